@@ -1,0 +1,402 @@
+/*
+ * tto.c -- CPU oracle of the TokenTiming verification path (arXiv 2510.15545).
+ *
+ * TEST INFRASTRUCTURE: the plain, slow, obviously-correct definition that the
+ * CUDA path is checked against. Only the tests, the smoke check and the
+ * benchmark's CPU legs may load it. It shares nothing with the CUDA library.
+ *
+ * Readings of the paper taken here (each one is listed with its reason in the
+ * design notes of the repository):
+ *  - p is the target distribution, q the draft one, accept while
+ *    u < min(1, p/q) (Alg. 4 naming; §3 and Alg. 2 swap the letters).
+ *  - Band: |i - j| <= w_eff with w_eff = max(w, |k - m|), so (k, m) is always
+ *    reachable; w < 0 means no band (§4.1 band, Alg. 1).
+ *  - Backtrack ties: prefer (i-1, j-1), then (i-1, j), then (i, j-1).
+ *  - Token distance is Levenshtein over the tokens' UTF-8 bytes (App. F, and
+ *    the byte-level resolution of the fragmented-tokenization study).
+ *  - Transfer: target position j takes the draft token with the largest i
+ *    aligned to it (terminal rule for many-to-one, copy rule for one-to-many,
+ *    App. A.2); its probability is the one-hot probability of that sampled
+ *    draft token (Limitations).
+ *  - After a rejection at j the next token is drawn from the normalised
+ *    residual max(0, p_j - q_j) (Alg. 4); with the one-hot q this is p_j with
+ *    the rejected token's mass reduced to max(0, p_j(t) - q_hat_j).
+ *  - Uniforms: Philox4x64-10, counter (position, stream, request, 0), key
+ *    (seed, 0), u = top 24 bits * 2^-24; stream 0 = accept, 1 = resample.
+ */
+#include "tto.h"
+
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ST_ID_RANGE 1
+#define ST_TOO_LONG 2
+#define ST_EMPTY 4
+#define ST_BAD_OFFSETS 8
+#define MAX_K 256
+#define MAX_M 512
+#define MAX_TOKEN_BYTES 256
+#define BOUNDARY_EPS 1e-6
+
+/* ------------------------------------------------------------------ App. F */
+
+int32_t tto_lev(const uint8_t* s, int32_t ns, const uint8_t* t, int32_t nt) {
+  /* D(i,0) = i, D(0,j) = j; D(i,j) = min(D(i-1,j)+1, D(i,j-1)+1,
+   * D(i-1,j-1) + [s_i != t_j]); the distance is D(ns, nt). */
+  int32_t* D = (int32_t*)malloc(sizeof(int32_t) * (size_t)(ns + 1) * (size_t)(nt + 1));
+  int32_t W = nt + 1;
+  for (int32_t i = 0; i <= ns; ++i) D[i * W] = i;
+  for (int32_t j = 0; j <= nt; ++j) D[j] = j;
+  for (int32_t i = 1; i <= ns; ++i) {
+    for (int32_t j = 1; j <= nt; ++j) {
+      int32_t del = D[(i - 1) * W + j] + 1;
+      int32_t ins = D[i * W + (j - 1)] + 1;
+      int32_t sub = D[(i - 1) * W + (j - 1)] + (s[i - 1] == t[j - 1] ? 0 : 1);
+      int32_t best = del < ins ? del : ins;
+      D[i * W + j] = sub < best ? sub : best;
+    }
+  }
+  int32_t r = D[ns * W + nt];
+  free(D);
+  return r;
+}
+
+/* ------------------------------------------------------------------ Alg. 1 */
+
+#define DTW_INF ((int64_t)1 << 60)
+
+int64_t tto_dtw(int32_t k, int32_t m, const int32_t* d, int32_t w,
+                int32_t* path, int32_t* path_len) {
+  *path_len = 0;
+  if (k <= 0 || m <= 0) return -1;
+  int64_t band;
+  if (w < 0) {
+    band = (int64_t)k + m; /* no band */
+  } else {
+    int64_t gap = k > m ? k - m : m - k;
+    band = w > gap ? w : gap;
+  }
+  int64_t W = m + 1;
+  int64_t* C = (int64_t*)malloc(sizeof(int64_t) * (size_t)(k + 1) * (size_t)W);
+  for (int64_t x = 0; x < (int64_t)(k + 1) * W; ++x) C[x] = DTW_INF;
+  C[0] = 0; /* C_{0,0} = 0, every other border cell is infinite */
+  for (int32_t i = 1; i <= k; ++i) {
+    int64_t jlo = i - band > 1 ? i - band : 1;
+    int64_t jhi = i + band < m ? i + band : m;
+    for (int64_t j = jlo; j <= jhi; ++j) {
+      int64_t up = C[(i - 1) * W + j];
+      int64_t left = C[i * W + (j - 1)];
+      int64_t diag = C[(i - 1) * W + (j - 1)];
+      int64_t best = up < left ? up : left;
+      best = diag < best ? diag : best;
+      C[i * W + j] = best >= DTW_INF ? DTW_INF : best + d[(int64_t)(i - 1) * m + (j - 1)];
+    }
+  }
+  int64_t cstar = C[(int64_t)k * W + m];
+  if (cstar >= DTW_INF) {
+    free(C);
+    return -1;
+  }
+  /* Backtrack from (k, m) to (0, 0), collecting cells in reverse order. */
+  int32_t* rev = (int32_t*)malloc(sizeof(int32_t) * 2 * (size_t)(k + m));
+  int32_t L = 0;
+  int64_t i = k, j = m;
+  while (i != 0 || j != 0) {
+    rev[2 * L] = (int32_t)i;
+    rev[2 * L + 1] = (int32_t)j;
+    ++L;
+    /* candidates in preference order: diagonal, up, left */
+    int64_t bi = i - 1, bj = j - 1;
+    int64_t bc = (bi >= 0 && bj >= 0) ? C[bi * W + bj] : DTW_INF;
+    int64_t cu = (i - 1 >= 0) ? C[(i - 1) * W + j] : DTW_INF;
+    if (cu < bc) { bi = i - 1; bj = j; bc = cu; }
+    int64_t cl = (j - 1 >= 0) ? C[i * W + (j - 1)] : DTW_INF;
+    if (cl < bc) { bi = i; bj = j - 1; bc = cl; }
+    i = bi;
+    j = bj;
+  }
+  for (int32_t x = 0; x < L; ++x) { /* forward order, 0-based indices */
+    path[2 * x] = rev[2 * (L - 1 - x)] - 1;
+    path[2 * x + 1] = rev[2 * (L - 1 - x) + 1] - 1;
+  }
+  *path_len = L;
+  free(rev);
+  free(C);
+  return cstar;
+}
+
+/* ------------------------------------------------ Philox (Salmon et al. 2011) */
+
+static void mulhilo64(uint64_t a, uint64_t b, uint64_t* hi, uint64_t* lo) {
+  unsigned __int128 p = (unsigned __int128)a * (unsigned __int128)b;
+  *hi = (uint64_t)(p >> 64);
+  *lo = (uint64_t)p;
+}
+
+void tto_philox4x64_10(const uint64_t ctr[4], const uint64_t key[2], uint64_t out[4]) {
+  const uint64_t M0 = 0xD2E7470EE14C6C93ULL, M1 = 0xCA5A826395121157ULL;
+  const uint64_t W0 = 0x9E3779B97F4A7C15ULL, W1 = 0xBB67AE8584CAA73BULL;
+  uint64_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];
+  uint64_t k0 = key[0], k1 = key[1];
+  for (int r = 0; r < 10; ++r) {
+    uint64_t hi0, lo0, hi1, lo1;
+    mulhilo64(M0, c0, &hi0, &lo0);
+    mulhilo64(M1, c2, &hi1, &lo1);
+    uint64_t n0 = hi1 ^ c1 ^ k0, n1 = lo1, n2 = hi0 ^ c3 ^ k1, n3 = lo0;
+    c0 = n0; c1 = n1; c2 = n2; c3 = n3;
+    k0 += W0;
+    k1 += W1;
+  }
+  out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
+}
+
+double tto_uniform(uint64_t seed, uint64_t pos, uint64_t stream, uint64_t request) {
+  uint64_t ctr[4] = {pos, stream, request, 0}, key[2] = {seed, 0}, out[4];
+  tto_philox4x64_10(ctr, key, out);
+  return (double)(out[0] >> 40) * (1.0 / 16777216.0);
+}
+
+/* ------------------------------------------------------------------ softmax */
+
+static double load_logit(const void* row, int32_t dtype, int64_t x) {
+  if (dtype == 0) return (double)((const float*)row)[x];
+  /* bf16: the upper 16 bits of an IEEE binary32 */
+  uint32_t bits = (uint32_t)((const uint16_t*)row)[x] << 16;
+  float f;
+  memcpy(&f, &bits, sizeof f);
+  return (double)f;
+}
+
+static const void* row_ptr(const void* base, int32_t dtype, int64_t stride, int64_t r) {
+  size_t elem = dtype == 0 ? 4 : 2;
+  return (const char*)base + (size_t)r * (size_t)stride * elem;
+}
+
+double tto_logsumexp(const void* row, int32_t dtype, int64_t V, double T) {
+  double mx = -INFINITY;
+  for (int64_t x = 0; x < V; ++x) {
+    double z = load_logit(row, dtype, x) / T;
+    if (z > mx) mx = z;
+  }
+  double s = 0.0;
+  for (int64_t x = 0; x < V; ++x) s += exp(load_logit(row, dtype, x) / T - mx);
+  return mx + log(s);
+}
+
+void tto_softmax(const void* row, int32_t dtype, int64_t V, double T, double* p) {
+  double mx = -INFINITY;
+  for (int64_t x = 0; x < V; ++x) {
+    double z = load_logit(row, dtype, x) / T;
+    if (z > mx) mx = z;
+  }
+  double s = 0.0;
+  for (int64_t x = 0; x < V; ++x) {
+    p[x] = exp(load_logit(row, dtype, x) / T - mx);
+    s += p[x];
+  }
+  for (int64_t x = 0; x < V; ++x) p[x] /= s;
+}
+
+/* ------------------------------------------------------------ batched align */
+
+static int32_t offsets_ok(const int32_t* off, int32_t b) {
+  return off[b] >= 0 && off[b + 1] >= off[b];
+}
+
+void tto_align(int32_t B, const int32_t* draft_off, const int32_t* draft_ids,
+               const int32_t* target_off, const int32_t* target_ids,
+               const uint8_t* vd_bytes, const int64_t* vd_off, int32_t Vd,
+               const uint8_t* vt_bytes, const int64_t* vt_off, int32_t Vt,
+               int32_t w, int32_t* path, int32_t* path_len, int32_t* cost,
+               int32_t* map, int32_t* status) {
+  for (int32_t b = 0; b < B; ++b) {
+    path_len[b] = 0;
+    cost[b] = -1;
+    if (!offsets_ok(draft_off, b) || !offsets_ok(target_off, b)) {
+      status[b] = ST_BAD_OFFSETS;
+      continue;
+    }
+    int32_t d0 = draft_off[b], k = draft_off[b + 1] - d0;
+    int32_t t0 = target_off[b], m = target_off[b + 1] - t0;
+    int32_t st = 0;
+    for (int32_t j = 0; j < m; ++j) map[t0 + j] = -1;
+    if (k == 0 || m == 0) st |= ST_EMPTY;
+    if (k > MAX_K || m > MAX_M) st |= ST_TOO_LONG;
+    /* length checks first; only then every token is looked at, OR-ing flags */
+    int32_t skip_tokens = st != 0;
+    for (int32_t i = 0; i < k && !skip_tokens; ++i) {
+      int32_t id = draft_ids[d0 + i];
+      if (id < 0 || id >= Vd) st |= ST_ID_RANGE;
+      else if (vd_off[id + 1] - vd_off[id] > MAX_TOKEN_BYTES) st |= ST_TOO_LONG;
+    }
+    for (int32_t j = 0; j < m && !skip_tokens; ++j) {
+      int32_t id = target_ids[t0 + j];
+      if (id < 0 || id >= Vt) st |= ST_ID_RANGE;
+      else if (vt_off[id + 1] - vt_off[id] > MAX_TOKEN_BYTES) st |= ST_TOO_LONG;
+    }
+    status[b] = st;
+    if (st) continue;
+    /* local cost d(x_i, y_j) for every cell (the band only reads some) */
+    int32_t* d = (int32_t*)malloc(sizeof(int32_t) * (size_t)k * (size_t)m);
+    for (int32_t i = 0; i < k; ++i) {
+      int32_t a = draft_ids[d0 + i];
+      for (int32_t j = 0; j < m; ++j) {
+        int32_t c = target_ids[t0 + j];
+        d[(int64_t)i * m + j] =
+            tto_lev(vd_bytes + vd_off[a], (int32_t)(vd_off[a + 1] - vd_off[a]),
+                    vt_bytes + vt_off[c], (int32_t)(vt_off[c + 1] - vt_off[c]));
+      }
+    }
+    int32_t* pb = path + 2 * ((int64_t)d0 + t0);
+    int32_t L = 0;
+    int64_t cs = tto_dtw(k, m, d, w, pb, &L);
+    free(d);
+    path_len[b] = L;
+    cost[b] = (int32_t)cs;
+    /* map[j] = largest draft index aligned to target index j */
+    for (int32_t x = 0; x < L; ++x) {
+      int32_t i = pb[2 * x], j = pb[2 * x + 1];
+      if (i > map[t0 + j]) map[t0 + j] = i;
+    }
+  }
+}
+
+/* ---------------------------------------------------------------- transfer */
+
+void tto_transfer(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                  const int32_t* target_off, const int32_t* map,
+                  const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                  const float* draft_probs, double T_d, double* q_hat, int32_t* status) {
+  for (int32_t b = 0; b < B; ++b) {
+    if (!offsets_ok(draft_off, b) || !offsets_ok(target_off, b)) {
+      status[b] = ST_BAD_OFFSETS;
+      continue;
+    }
+    int32_t d0 = draft_off[b], k = draft_off[b + 1] - d0;
+    int32_t t0 = target_off[b], m = target_off[b + 1] - t0;
+    int32_t st = 0;
+    if (k == 0 || m == 0) st |= ST_EMPTY;
+    int32_t skip_tokens = st != 0;
+    for (int32_t j = 0; j < m && !skip_tokens; ++j)
+      if (map[t0 + j] < 0 || map[t0 + j] >= k) st |= ST_ID_RANGE;
+    for (int32_t i = 0; i < k && !skip_tokens && !draft_probs; ++i)
+      if (draft_cols[d0 + i] < 0 || draft_cols[d0 + i] >= V) st |= ST_ID_RANGE;
+    status[b] = st;
+    for (int32_t j = 0; j < m; ++j) q_hat[t0 + j] = 0.0;
+    if (st) continue;
+    for (int32_t j = 0; j < m; ++j) {
+      int64_t r = (int64_t)d0 + map[t0 + j];
+      if (draft_probs) {
+        q_hat[t0 + j] = (double)draft_probs[r];
+      } else {
+        const void* row = row_ptr(draft_logits, dtype, row_stride, r);
+        double lse = tto_logsumexp(row, dtype, V, T_d);
+        q_hat[t0 + j] = exp(load_logit(row, dtype, draft_cols[r]) / T_d - lse);
+      }
+    }
+  }
+}
+
+/* ------------------------------------------------------------------ verify */
+
+void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                const double* q_hat, const void* target_logits, int32_t dtype_t,
+                int64_t stride_t, int32_t V_t, double T_t,
+                const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                int32_t full_q, uint64_t seed, uint64_t request_base,
+                int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
+                int32_t* status, int32_t* boundary) {
+  double* p = (double*)malloc(sizeof(double) * (size_t)V_t);
+  double* q = full_q ? (double*)malloc(sizeof(double) * (size_t)V_d) : NULL;
+  double* r = (double*)malloc(sizeof(double) * (size_t)V_t);
+  for (int32_t b = 0; b < B; ++b) {
+    accepted[b] = 0;
+    next_token[b] = -1;
+    boundary[b] = 0;
+    if (!offsets_ok(target_off, b)) {
+      status[b] = ST_BAD_OFFSETS;
+      continue;
+    }
+    int32_t t0 = target_off[b], m = target_off[b + 1] - t0;
+    int64_t row0 = (int64_t)t0 + b; /* request b owns target rows row0 .. row0+m */
+    int32_t st = 0;
+    if (m == 0) st |= ST_EMPTY;
+    if (m > MAX_M) st |= ST_TOO_LONG;
+    int32_t skip_tokens = st != 0;
+    for (int32_t j = 0; j < m && !skip_tokens; ++j)
+      if (target_cols[t0 + j] < 0 || target_cols[t0 + j] >= V_t) st |= ST_ID_RANGE;
+    if (full_q && !skip_tokens) {
+      if (!offsets_ok(draft_off, b)) {
+        st |= ST_BAD_OFFSETS;
+      } else {
+        int32_t k = draft_off[b + 1] - draft_off[b];
+        for (int32_t j = 0; j < m; ++j)
+          if (map[t0 + j] < 0 || map[t0 + j] >= k) st |= ST_ID_RANGE;
+      }
+    }
+    status[b] = st;
+    if (st) continue;
+
+    /* p_hat_j = p_j(t_j) for every target position; lse of all m+1 rows */
+    for (int32_t j = 0; j <= m; ++j) {
+      const void* row = row_ptr(target_logits, dtype_t, stride_t, row0 + j);
+      double l = tto_logsumexp(row, dtype_t, V_t, T_t);
+      if (lse) lse[row0 + j] = l;
+      if (j < m) p_hat[t0 + j] = exp(load_logit(row, dtype_t, target_cols[t0 + j]) / T_t - l);
+    }
+
+    /* sequential accept, stop at the first rejection */
+    int32_t a = 0;
+    for (int32_t j = 0; j < m; ++j) {
+      double u = tto_uniform(seed, (uint64_t)j, 0, request_base + (uint64_t)b);
+      double ph = p_hat[t0 + j], qh = q_hat[t0 + j];
+      double ratio = qh > 0.0 ? ph / qh : (ph > 0.0 ? INFINITY : 0.0);
+      double acc = ratio < 1.0 ? ratio : 1.0;
+      if (fabs(u - acc) < BOUNDARY_EPS) boundary[b] |= 1;
+      if (u < acc) ++a;
+      else break;
+    }
+    accepted[b] = a;
+
+    /* the residual (or bonus) row a */
+    const void* prow = row_ptr(target_logits, dtype_t, stride_t, row0 + a);
+    tto_softmax(prow, dtype_t, V_t, T_t, p);
+    if (a < m) {
+      if (full_q) {
+        const void* qrow = row_ptr(draft_logits, dtype_d, stride_d,
+                                   (int64_t)draft_off[b] + map[t0 + a]);
+        tto_softmax(qrow, dtype_d, V_d, T_d, q);
+        for (int32_t x = 0; x < V_t; ++x) r[x] = p[x] > q[x] ? p[x] - q[x] : 0.0;
+      } else {
+        int32_t t = target_cols[t0 + a];
+        for (int32_t x = 0; x < V_t; ++x) r[x] = p[x];
+        double rt = p[t] - q_hat[t0 + a];
+        r[t] = rt > 0.0 ? rt : 0.0;
+      }
+    } else {
+      for (int32_t x = 0; x < V_t; ++x) r[x] = p[x];
+    }
+    double Z = 0.0;
+    for (int32_t x = 0; x < V_t; ++x) Z += r[x];
+    if (!(Z > 0.0)) { /* degenerate residual: fall back to the row itself */
+      for (int32_t x = 0; x < V_t; ++x) r[x] = p[x];
+      Z = 0.0;
+      for (int32_t x = 0; x < V_t; ++x) Z += r[x];
+    }
+    double u2 = tto_uniform(seed, (uint64_t)a, 1, request_base + (uint64_t)b);
+    double theta = u2 * Z, cum = 0.0;
+    int32_t pick = -1, last_pos = -1;
+    for (int32_t x = 0; x < V_t; ++x) {
+      cum += r[x];
+      if (r[x] > 0.0) last_pos = x;
+      if (fabs(theta - cum) < BOUNDARY_EPS * Z) boundary[b] |= 2;
+      if (pick < 0 && cum > theta) pick = x;
+    }
+    next_token[b] = pick >= 0 ? pick : last_pos;
+  }
+  free(p);
+  free(q);
+  free(r);
+}

@@ -1,0 +1,81 @@
+/*
+ * tto.h -- CPU oracle of the TokenTiming verification path (arXiv 2510.15545).
+ *
+ * TEST INFRASTRUCTURE. This library is the slow, plain reference that the CUDA
+ * path is compared against. Only the test suite, the smoke check and the
+ * benchmark's CPU-baseline / reference legs load it; the product path never
+ * does. It shares no code, header or constant with the CUDA library.
+ *
+ * Arithmetic is fp64 throughout; every routine is the textbook form of the
+ * passage it cites. Indices are 0-based in all arrays.
+ *
+ * Per-request status bits (the same values the CUDA library documents):
+ *   1 id out of range, 2 too long, 4 empty request, 8 bad CSR offsets.
+ * Boundary bits (oracle only): 1 = some accept draw u_j lay within 1e-6 of
+ * min(1, p/q); 2 = the residual draw u' lay within 1e-6 of a CDF breakpoint.
+ */
+#ifndef TTO_H
+#define TTO_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* App. F: Levenshtein distance between byte strings, unit costs. */
+int32_t tto_lev(const uint8_t* s, int32_t ns, const uint8_t* t, int32_t nt);
+
+/* Alg. 1 on a given k x m local cost matrix d (row-major, d[i*m+j] =
+ * d(x_{i+1}, y_{j+1})). w < 0: no band. Writes the optimal path as 0-based
+ * (i, j) pairs in forward order (capacity k+m pairs) and returns C* (or -1). */
+int64_t tto_dtw(int32_t k, int32_t m, const int32_t* d, int32_t w,
+                int32_t* path, int32_t* path_len);
+
+/* Philox4x64-10 (Salmon et al., SC'11) of one counter block. */
+void tto_philox4x64_10(const uint64_t ctr[4], const uint64_t key[2], uint64_t out[4]);
+
+/* Uniform in [0,1): top 24 bits of the first Philox word times 2^-24, for
+ * counter (pos, stream, request, 0) and key (seed, 0). */
+double tto_uniform(uint64_t seed, uint64_t pos, uint64_t stream, uint64_t request);
+
+/* Two-pass fp64 softmax of row/T (row: fp32 or bf16 values, dtype 0 / 1). */
+void tto_softmax(const void* row, int32_t dtype, int64_t V, double T, double* p_out);
+double tto_logsumexp(const void* row, int32_t dtype, int64_t V, double T);
+
+/* Batched DTW alignment (§4.1, Alg. 1, App. F). Outputs are per request:
+ * path pairs at pair offset draft_off[b] + target_off[b], path_len[b],
+ * cost[b] = C*, map[j] = max{i : (i,j) on the path} for the request's target
+ * positions, status[b]. */
+void tto_align(int32_t B, const int32_t* draft_off, const int32_t* draft_ids,
+               const int32_t* target_off, const int32_t* target_ids,
+               const uint8_t* vd_bytes, const int64_t* vd_off, int32_t Vd,
+               const uint8_t* vt_bytes, const int64_t* vt_off, int32_t Vt,
+               int32_t w, int32_t* path, int32_t* path_len, int32_t* cost,
+               int32_t* map, int32_t* status);
+
+/* MapProbabilities (Alg. 2, App. A.2): q_hat[j] = probability of the mapped
+ * draft token d_{map[j]} under its own draft row at temperature T_d, or
+ * draft_probs[row] when draft_probs is not NULL. */
+void tto_transfer(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                  const int32_t* target_off, const int32_t* map,
+                  const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                  const float* draft_probs, double T_d, double* q_hat, int32_t* status);
+
+/* Verification (Alg. 2 accept loop, Alg. 4 residual): accept target token j
+ * while u_j < min(1, p_j / q_hat_j); then sample the next token from the
+ * normalised residual of row a (or from the bonus row when all m were
+ * accepted). full_q != 0: homogeneous vocabulary, residual max(0, p - q) with
+ * q the full draft row map[a]. */
+void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                const double* q_hat, const void* target_logits, int32_t dtype_t,
+                int64_t stride_t, int32_t V_t, double T_t,
+                const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                int32_t full_q, uint64_t seed, uint64_t request_base,
+                int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
+                int32_t* status, int32_t* boundary);
+
+#ifdef __cplusplus
+}
+#endif
+#endif
