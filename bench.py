@@ -1,0 +1,477 @@
+#!/usr/bin/env python
+"""Benchmark of the TokenTiming verification step on GB300.
+
+One step = one tt_step over a batch: DTW alignment of every request, one pass
+over the mapped draft rows and all target rows, and the per-request
+accept / residual-sampling decision. Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the CPU oracle, timed on the host
+
+Under torchrun every rank runs its own batch (requests are independent; no
+collective on the data path) and the timed region is bracketed by barriers;
+the reported time is the maximum over ranks (weak scaling).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "b64_g8_v152k"
+METRIC = "verified draft positions/sec (batch×γ) and HBM GB/s vs 8 TB/s; DTW pairs/sec"
+UNIT = "positions/s"
+L2_BYTES = 129 * 1024 * 1024
+FALLBACK_HBM_GBS = 6800.0
+ROWPASS_SOURCES = ["paper_2510_15545_gb300/csrc/rowpass.cu",
+                   "paper_2510_15545_gb300/csrc/tt_device.cuh",
+                   "paper_2510_15545_gb300/csrc/tt_launch.h"]
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["mine", "reference"], default="mine")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="CPU work budget of the oracle baseline sample")
+    return ap.parse_args(argv)
+
+
+# ----------------------------------------------------------- multi-process
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, ws, local
+
+
+def dist_init(ws, backend):
+    import torch.distributed as dist
+    if ws > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend)
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(value: float, ws: int, device=None) -> float:
+    """Largest value over ranks (the slowest rank sets the job's time)."""
+    if ws <= 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64,
+                     device=device if device is not None else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value: float, ws: int, device=None) -> float:
+    if ws <= 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64,
+                     device=device if device is not None else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons, kept with host
+    timestamps so that only the samples inside the timed region count."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, period_ms: int = 50):
+        self.samples = []
+        self.proc = None
+        self.thread = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                 "-i", str(gpu_index), "-lms", str(period_ms)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.perf_counter(), [x.strip() for x in line.split(",")]))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float) -> dict:
+        inside = [s for t, s in self.samples if t0 <= t <= t1]
+        note = "samples inside the timed region"
+        if not inside and self.samples:  # a very short region: nearest samples
+            inside = [min(self.samples, key=lambda ts: abs(ts[0] - 0.5 * (t0 + t1)))[1]]
+            note = "nearest sample to a timed region shorter than the sampling period"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for s in inside:
+            try:
+                sm.append(float(s[1]))
+                smax.append(float(s[2]))
+            except (ValueError, IndexError):
+                continue
+            for n, v in zip(names, s[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": sorted(reasons),
+                "samples": len(inside), "note": note}
+
+
+# ----------------------------------------------------------------- helpers
+
+def measured_hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def rowpass_source_hash() -> str:
+    h = hashlib.sha256()
+    for rel in ROWPASS_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str):
+    """DRAM bytes per row-pass launch from the committed ncu summary, if it was
+    taken on the current row-pass source."""
+    path = os.path.join(ROOT, "profiles", "rowpass_%s.md" % workload)
+    try:
+        txt = open(path).read()
+    except OSError:
+        return None
+    vals = {}
+    for line in txt.splitlines():
+        if ":" in line and line.strip().startswith("- "):
+            k, v = line.strip()[2:].split(":", 1)
+            vals[k.strip()] = v.strip().strip("`")
+    if vals.get("source_sha256") != rowpass_source_hash():
+        return None
+    try:
+        return float(vals["traffic_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+def algorithmic_bytes(wl, mp) -> dict:
+    """Bytes the step must read once: every distinct mapped draft row and all
+    m_b + 1 target rows of every request."""
+    import numpy as np
+    esz_d = wl.draft_logits.element_size()
+    esz_t = wl.target_logits.element_size()
+    rows_d = 0
+    for b in range(wl.B):
+        t0, t1 = int(wl.target_off[b]), int(wl.target_off[b + 1])
+        rows_d += len(np.unique(mp[t0:t1]))
+    d = rows_d * wl.draft_logits.shape[1] * esz_d
+    t = (wl.n_target + wl.B) * wl.target_logits.shape[1] * esz_t
+    return {"draft_rows": rows_d, "target_rows": wl.n_target + wl.B, "draft_bytes": d,
+            "target_bytes": t, "total": d + t}
+
+
+def default_steps(name: str) -> int:
+    return {"b1_g4_v32k": 20000, "b64_g8_v152k": 20000, "b256_g16_v152k_bf16": 3000,
+            "dtw_4096x64": 1000, "b1024_g8_v201k_bf16": 1000}.get(name, 1000)
+
+
+def oracle_sample_rate(wl, budget_s: float, rank: int = 0):
+    """Times the oracle (as it stands) over requests of the workload, cycling
+    through them until the CPU budget is spent; returns positions/s and a note."""
+    import oracle
+    oracle.build()
+    order = list(range(wl.B))
+    subs = {}
+    done_req, positions, elapsed, passes = 0, 0, 0.0, 0
+    while elapsed < budget_s:
+        b = order[done_req % wl.B]
+        if b not in subs:
+            subs[b] = wl.subset([b])
+        sw = subs[b]
+        t = time.perf_counter()
+        oracle.step(sw, request_base=b)
+        elapsed += time.perf_counter() - t
+        positions += int(sw.draft_off[-1])
+        done_req += 1
+    sample = ("%d requests of the %s batch (cycling from request 0), oracle single-threaded, "
+              "fp64, %.1f s of CPU time" % (done_req, wl.spec.name, elapsed))
+    return positions / elapsed, sample, done_req, elapsed
+
+
+# -------------------------------------------------------------- my arm
+
+def run_mine(args):
+    import numpy as np
+    import torch
+
+    rank, ws, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist_init(ws, "nccl")
+    import paper_2510_15545_gb300 as tt
+    from paper_2510_15545_gb300 import workload as W
+    tt.load(build_if_missing=(rank == 0 or ws == 1))
+    barrier(ws)
+    tt.load()
+
+    name = args.workload
+    K = args.steps if args.steps is not None else default_steps(name)
+    Wm = max(3, args.warmup)
+    wl = W.make_workload(name, seed=rank, device=str(dev))
+    inp = tt.device_inputs(wl, dev)
+    prm = inp["params"]
+    prm.request_base = rank * wl.B
+    batch, vd, vt = inp["batch"], inp["vd"], inp["vt"]
+    dl, tl = inp["draft_logits"], inp["target_logits"]
+    stream = torch.cuda.current_stream(dev)
+
+    # one untimed step with every output: mapped draft rows, acceptance
+    full = tt.tt_step(batch, vd, vt, dl, tl, prm)
+    torch.cuda.synchronize(dev)
+    mp = full["map"].cpu().numpy()
+    acc = full["accepted"].cpu().numpy()
+    assert int((full["status"] != 0).sum()) == 0, "a request failed"
+    ab = algorithmic_bytes(wl, mp)
+    m = np.diff(wl.target_off)
+
+    call = tt.StepCall(batch, vd, vt, dl, tl, prm, out=tt.step_outputs(batch, dev, full=False),
+                       stream=stream)
+    # stage events on a strided subset of the timed steps
+    stride = max(1, math.ceil(K / 2000))
+    sampled = list(range(0, K, stride))
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in sampled]
+    for e4 in ev:
+        for e in e4:
+            e.record(stream)
+    handles = [[e.cuda_event for e in e4] for e4 in ev]
+
+    for _ in range(Wm):
+        call()
+    torch.cuda.synchronize(dev)
+
+    clocks = ClockSampler(local)
+    time.sleep(0.3)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    barrier(ws)
+    torch.cuda.synchronize(dev)
+    h0 = time.perf_counter()
+    t_start.record(stream)
+    si = 0
+    for i in range(K):
+        if si < len(sampled) and sampled[si] == i:
+            call(handles[si])
+            si += 1
+        else:
+            call()
+    t_end.record(stream)
+    torch.cuda.synchronize(dev)
+    h1 = time.perf_counter()
+    barrier(ws)
+    time.sleep(0.2)
+    clocks.stop()
+    sec = t_start.elapsed_time(t_end) / 1e3
+    sec_max = max_over_ranks(sec, ws, dev)
+    align_ms = statistics.mean(e4[0].elapsed_time(e4[1]) for e4 in ev)
+    row_ms = statistics.mean(e4[1].elapsed_time(e4[2]) for e4 in ev)
+    dec_ms = statistics.mean(e4[2].elapsed_time(e4[3]) for e4 in ev)
+
+    positions = wl.n_draft  # verified draft positions per step (batch x gamma)
+    value = positions * K * ws / sec_max
+    peak, peak_kind = measured_hbm_peak()
+    achieved = ab["total"] / (row_ms / 1e3) / 1e9
+    step_gbs = ab["total"] / (sec / K) / 1e9
+    traffic = profiled_traffic(name)
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(tt, wl, inp, prm, dev, stream, K, ws)
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        rate, sample, nreq, el = oracle_sample_rate(wl, args.cpu_seconds)
+        cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
+
+    clk = clocks.summary(h0, h1)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": K,
+        "warmup": Wm, "ms_per_step": sec_max * 1e3 / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": wl.spec.dtype.__repr__().split(".")[-1]
+        .replace("float32", "f32").replace("bfloat16", "bf16"),
+        "data": "synthetic (seeded byte-string vocabularies, greedy re-encoding, Zipf logits)",
+        "config": {"workload": name, "batch_per_gpu": wl.B, "gamma": wl.spec.k,
+                   "V_d": wl.spec.V_d, "V_t": wl.spec.V_t,
+                   "logits_cols": [int(dl.shape[1]), int(tl.shape[1])],
+                   "target_tokens_per_gpu": wl.n_target, "window": prm.window,
+                   "parallelism": "dp%d (independent requests per GPU)" % ws,
+                   "l2": "inputs %.0f MB exceed the 129 MB L2; no flush between steps"
+                         % ((dl.numel() * dl.element_size() + tl.numel() * tl.element_size()) / 1e6)
+                   if ab["total"] > L2_BYTES else "inputs fit in L2",
+                   "accept_rate": float(acc.sum() / max(1, m.sum())),
+                   "mean_accepted": float(acc.mean())},
+        "hbm_gbs_step": step_gbs,
+        "dtw_pairs_per_s": wl.B / (align_ms / 1e3),
+        "stage_ms": {"align": align_ms, "rowpass": row_ms, "decide": dec_ms,
+                     "sampled_steps": len(sampled)},
+        "roofline": {"bound": "hbm", "kernel": "rowpass_kernel", "achieved": achieved,
+                     "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                     "peak_kind": "%s copy bandwidth (hbm_gbs)" % peak_kind,
+                     "traffic": traffic, "algorithmic_bytes": ab["total"],
+                     "vs_nominal_8tbs": achieved / 8000.0},
+        "gpu_launches": 3 * K,
+        "clocks": clk,
+    }
+    if e2e is not None:
+        line["e2e"] = e2e
+    if cpu is not None:
+        line["cpu_baseline"] = cpu
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_e2e(tt, wl, inp, prm, dev, stream, K, ws):
+    """The same metric through the public API with the step's inputs in pinned
+    host memory: every step copies ids, offsets and logits host -> device,
+    runs tt_step and reads the results back."""
+    import torch
+    batch = inp["batch"]
+    dev_tensors = [batch.draft_off, batch.draft_ids, batch.target_off, batch.target_ids,
+                   batch.draft_cols, batch.target_cols, inp["draft_logits"], inp["target_logits"]]
+    dev_tensors = [t for t in dev_tensors if t is not None]
+    host = [t.cpu().pin_memory() for t in dev_tensors]
+    out = tt.step_outputs(batch, dev, full=False)
+    res_host = [torch.empty_like(out[k], device="cpu").pin_memory()
+                for k in ("accepted", "next_token", "status")]
+    call = tt.StepCall(batch, inp["vd"], inp["vt"], inp["draft_logits"], inp["target_logits"], prm,
+                       out=out, stream=stream)
+    h2d = sum(t.numel() * t.element_size() for t in host)
+    d2h = sum(t.numel() * t.element_size() for t in res_host)
+
+    def one():
+        for d, h in zip(dev_tensors, host):
+            d.copy_(h, non_blocking=True)
+        call()
+        for h, k in zip(res_host, ("accepted", "next_token", "status")):
+            h.copy_(out[k], non_blocking=True)
+        stream.synchronize()
+
+    for _ in range(3):
+        one()
+    t0 = time.perf_counter()
+    one()
+    est = time.perf_counter() - t0
+    n = max(3, min(K, int(math.ceil(3.0 / max(est, 1e-6)))))
+    barrier(ws)
+    t0 = time.perf_counter()
+    for _ in range(n):
+        one()
+    sec = time.perf_counter() - t0
+    sec = max_over_ranks(sec, ws, dev)
+    return {"value": wl.n_draft * n * ws / sec, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": n, "ms_per_step": sec * 1e3 / n,
+            "api": "pinned host tensors -> copy_(non_blocking) -> tt_step -> copy_ back -> sync"}
+
+
+# ---------------------------------------------------------- reference arm
+
+def run_reference(args):
+    """The CPU oracle as it stands, on the host cores, on the same workload and
+    metric: each step is a bounded sample of the batch's requests."""
+    rank, ws, local = dist_env()
+    if rank != 0:
+        return
+    from paper_2510_15545_gb300 import workload as W
+    import oracle
+    oracle.build()
+    name = args.workload
+    K = args.steps if args.steps is not None else 5
+    Wm = max(3, args.warmup)
+    wl = W.make_workload(name, seed=0, device="cpu")
+    per_step = {"b1_g4_v32k": 1, "b64_g8_v152k": 4, "b256_g16_v152k_bf16": 2,
+                "dtw_4096x64": 16, "b1024_g8_v201k_bf16": 2}.get(name, 2)
+    subs = []
+    for s in range(K + Wm):
+        idx = [((s * per_step) + i) % wl.B for i in range(per_step)]
+        subs.append((idx[0], wl.subset(idx)))
+    for s in range(Wm):
+        b0, sw = subs[s]
+        oracle.step(sw, request_base=b0)
+    t0 = time.perf_counter()
+    pos = 0
+    for s in range(Wm, Wm + K):
+        b0, sw = subs[s]
+        oracle.step(sw, request_base=b0)
+        pos += int(sw.draft_off[-1])
+    sec = time.perf_counter() - t0
+    value = pos / sec
+    sample = ("%d requests of the %s batch per step, oracle single-threaded, fp64"
+              % (per_step, name))
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": ws, "steps": K, "warmup": Wm, "ms_per_step": sec * 1e3 / K,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": name, "requests_per_step": per_step},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_mine(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,202 @@
+/*
+ * tt.h -- C ABI of the TokenTiming verification hot path on one NVIDIA GB300
+ * (sm_103a). TokenTiming: arXiv 2510.15545 ("TokenTiming: A Dynamic Alignment
+ * Method for Universal Speculative Decoding Model Pairs").
+ *
+ * One verification step of a batch of B independent requests:
+ *   (a) align   -- Dynamic Token Warping (§4.1, Alg. 1) between each request's
+ *                  draft tokens D = (d_1..d_k) and its proxy target tokens
+ *                  T = (t_1..t_m) = encode_t(decode_d(D)) (§4.2, App. A.1),
+ *                  with the Levenshtein distance over the tokens' UTF-8 bytes as
+ *                  the local cost (App. F) and a Sakoe-Chiba band (§4.1);
+ *   (b) transfer -- MapProbabilities (Alg. 2, App. A.2): target position j
+ *                  takes the draft probability of the last draft token aligned
+ *                  to it (terminal rule / copy rule), one-hot (Limitations);
+ *   (c) verify  -- speculative sampling (§4.2 verification, Alg. 4): accept t_j
+ *                  while u_j < min(1, p(t_j)/q(t_j)), stop at the first
+ *                  rejection, then draw the next token from the normalised
+ *                  residual max(0, p - q) over the whole target vocabulary (or
+ *                  from the bonus row m+1 when all m were accepted).
+ * Here p is the target distribution and q the draft one (Alg. 4's naming).
+ *
+ * Conventions shared by every entry point:
+ *  - Every pointer is a DEVICE pointer owned by the caller, unless stated
+ *    otherwise; the library allocates nothing. Scratch space is the caller's
+ *    `workspace` (size from tt_workspace_bytes).
+ *  - Calls are asynchronous on `stream` (a cudaStream_t, NULL = the legacy
+ *    default stream). Nothing synchronises; the caller does.
+ *  - Call-level errors come back as tt_status before anything is launched.
+ *    Per-request problems are reported in status[b] (bits below); a failed
+ *    request yields accepted[b] = 0 and next_token[b] = -1. Kernels never trap.
+ *  - Requests are CSR batches: request b owns draft tokens
+ *    draft_off[b] .. draft_off[b+1]-1 and target tokens
+ *    target_off[b] .. target_off[b+1]-1 (k_b and m_b of them). It owns the draft
+ *    logits rows with the same indices (row i is the distribution d_i was drawn
+ *    from) and the m_b + 1 target logits rows target_off[b] + b ..
+ *    target_off[b+1] + b (row j scores t_{j+1}; the last one is the bonus row).
+ *  - All indices in inputs and outputs are 0-based.
+ *  - Uniforms: Philox4x64-10 (Salmon et al., SC'11), key (seed, 0), counter
+ *    (position j, stream, request_base + b, 0), u = (top 24 bits of word 0) *
+ *    2^-24; stream 0 draws the accept uniforms, stream 1 the resampling one.
+ */
+#ifndef TT_H
+#define TT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TT_MAX_K 256          /* longest draft sequence per request */
+#define TT_MAX_M 512          /* longest proxy target sequence per request */
+#define TT_MAX_TOKEN_BYTES 256 /* longest byte string of one token */
+
+typedef enum {
+  TT_OK = 0,
+  TT_ERR_INVALID_ARG = 1, /* a NULL required pointer, a bad size or alignment */
+  TT_ERR_UNSUPPORTED = 2, /* valid but outside what the kernels handle */
+  TT_ERR_CUDA = 3         /* a CUDA launch failed; see tt_last_cuda_error() */
+} tt_status;
+
+/* Bits of status[b]. */
+#define TT_REQ_OK 0
+#define TT_REQ_ID_OUT_OF_RANGE 1 /* a token id / logits column / map entry out of range */
+#define TT_REQ_TOO_LONG 2        /* k > min(max_k, TT_MAX_K), m > min(max_m, TT_MAX_M) or a
+                                    token longer than TT_MAX_TOKEN_BYTES */
+#define TT_REQ_EMPTY 4           /* k == 0 or m == 0 */
+#define TT_REQ_BAD_OFFSETS 8     /* CSR offsets decreasing or outside [0, n_draft/n_target] */
+#define TT_REQ_NOT_FINITE 16     /* a logits row gave a non-finite normaliser */
+
+typedef enum { TT_F32 = 0, TT_BF16 = 1 } tt_dtype;
+
+/* A token byte-string table: token id v spells bytes[offsets[v] .. offsets[v+1]). */
+typedef struct {
+  const uint8_t* bytes;   /* device, [n_bytes] */
+  const int64_t* offsets; /* device, [n_tokens + 1]; a token whose range is not inside
+                             [0, n_bytes] is reported as TT_REQ_ID_OUT_OF_RANGE */
+  int32_t n_tokens;
+  int64_t n_bytes;
+} tt_vocab;
+
+/* Row-major logits rows: row r starts at element r * row_stride. data must be
+ * 16-byte aligned and row_stride * element size a multiple of 16 bytes. */
+typedef struct {
+  const void* data; /* device */
+  int32_t dtype;    /* tt_dtype */
+  int32_t n_cols;   /* V: width of a row (the vocabulary the row scores) */
+  int64_t row_stride; /* elements between row starts, >= n_cols */
+  int64_t n_rows;   /* rows available at data */
+} tt_logits;
+
+typedef struct {
+  int32_t window;      /* Sakoe-Chiba half-width w >= 0 (the paper settles on 8,
+                          App. G); negative = no band. The band used for a request
+                          is max(w, |k - m|) so that (k, m) stays reachable. */
+  float temp_draft;    /* T_d > 0: draft rows are softmax(z / T_d) */
+  float temp_target;   /* T_t > 0: target rows are softmax(z / T_t) */
+  int32_t full_q;      /* 0: one-hot transfer (the paper's); 1: homogeneous
+                          vocabularies, residual max(0, p - q) against the full
+                          draft row (standard speculative decoding, Alg. 4);
+                          needs draft and target rows of the same width */
+  uint64_t seed;       /* Philox key */
+  uint64_t request_base; /* global index of request 0 in the Philox counter */
+  void* const* events; /* host array of 4 cudaEvent_t or NULL: tt_step records
+                          them before align, before the row pass, before the
+                          decision kernel and after it (profiling only) */
+} tt_params;
+
+typedef struct {
+  int32_t B;          /* requests */
+  int32_t n_draft;    /* sum of k_b = draft_off[B] */
+  int32_t n_target;   /* sum of m_b = target_off[B] */
+  int32_t max_k;      /* bound on k_b used to size on-chip buffers (<= TT_MAX_K) */
+  int32_t max_m;      /* bound on m_b (<= TT_MAX_M) */
+  const int32_t* draft_off;   /* [B+1] */
+  const int32_t* draft_ids;   /* [n_draft] ids into the draft vocab table */
+  const int32_t* draft_cols;  /* [n_draft] column of d_i in its logits row; NULL = draft_ids */
+  const int32_t* target_off;  /* [B+1] */
+  const int32_t* target_ids;  /* [n_target] ids into the target vocab table */
+  const int32_t* target_cols; /* [n_target] column of t_j in its logits row; NULL = target_ids */
+} tt_batch;
+
+/* Outputs of tt_step. accepted, next_token and status are required; the rest
+ * may be NULL. */
+typedef struct {
+  int32_t* accepted;   /* [B] a_b, number of target tokens accepted (0..m_b) */
+  int32_t* next_token; /* [B] column sampled from the residual / bonus row */
+  int32_t* status;     /* [B] TT_REQ_* bits */
+  int32_t* path;       /* [2 * (n_draft + n_target)] (i, j) pairs; request b's
+                          path starts at pair draft_off[b] + target_off[b] */
+  int32_t* path_len;   /* [B] pairs on the path (<= k_b + m_b - 1) */
+  int32_t* cost;       /* [B] C* = accumulated cost of the path, -1 if failed */
+  int32_t* map;        /* [n_target] draft index aligned to each target token */
+  float* q_hat;        /* [n_target] transferred draft probability q(t_j) */
+  float* p_hat;        /* [n_target] target probability p(t_j) */
+  float* lse;          /* [n_target + B] natural log-normaliser of every target row */
+} tt_step_out;
+
+/* Bytes of scratch the transfer / verify / step calls need for this batch and
+ * these row widths. 256-byte aligned sizes; pass a 256-byte aligned pointer. */
+size_t tt_workspace_bytes(const tt_batch* batch, int32_t V_d, int32_t V_t);
+
+/* (a) DTW alignment (§4.1, Alg. 1; App. F token distance).
+ * Per request: local cost d(i,j) = Levenshtein distance between the byte
+ * strings of d_i (in vd) and t_j (in vt), for cells inside the band;
+ * C_{0,0} = 0, border and out-of-band cells infinite,
+ * C_{i,j} = d(i,j) + min(C_{i-1,j}, C_{i,j-1}, C_{i-1,j-1}); backtrack from
+ * (k, m) taking the smallest predecessor, ties broken diagonal, then (i-1, j),
+ * then (i, j-1). Writes path/path_len/cost/map/status; map[j] is the largest
+ * draft index on the path in column j. Uses batch ids (not cols). Needs no
+ * workspace. TT_ERR_UNSUPPORTED when the on-chip tile for max_k x max_m (and
+ * the band) does not fit in shared memory. */
+tt_status tt_align(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
+                   const tt_params* prm, int32_t* path, int32_t* path_len, int32_t* cost,
+                   int32_t* map, int32_t* status, void* stream);
+
+/* (b) Transfer (Alg. 2 MapProbabilities, App. A.2, Limitations).
+ * q_hat[j] = softmax(draft row map[j] / T_d) at column draft_cols[map[j]],
+ * or draft_probs[draft_off[b] + map[j]] when draft_probs (fp32 [n_draft],
+ * device) is not NULL, in which case `draft` may be NULL. Writes q_hat and
+ * status. */
+tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits* draft,
+                      const float* draft_probs, const tt_params* prm, void* workspace,
+                      size_t workspace_bytes, float* q_hat, int32_t* status, void* stream);
+
+/* (c) Verification (§4.2, Alg. 2 accept loop, Alg. 4 residual).
+ * Reads the m_b + 1 target rows of every request once. p_hat[j] =
+ * softmax(target row j / T_t) at target_cols[j]; accept while
+ * u_j < min(1, p_hat[j] / q_hat[j]) (q_hat = 0 accepts when p_hat > 0);
+ * a_b = accepted count; next token from row a_b: residual max(0, p - q)
+ * (one-hot q = q_hat e_{t}, or the full draft row map[a_b] when full_q), or
+ * the bonus row itself when a_b = m_b; inverse CDF in column order, smallest x
+ * whose running mass exceeds u' * Z. `draft` and `map` are read only when
+ * full_q. p_hat and lse may be NULL. */
+tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* target,
+                    const tt_logits* draft, const int32_t* map, const tt_params* prm,
+                    void* workspace, size_t workspace_bytes, int32_t* accepted,
+                    int32_t* next_token, float* p_hat, float* lse, int32_t* status,
+                    void* stream);
+
+/* (a)+(b)+(c) fused: align, one streaming pass over the needed draft rows and
+ * all target rows, then the per-request decision, as three kernels on
+ * `stream`. Same results as tt_align -> tt_transfer -> tt_verify. */
+tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
+                  const tt_logits* draft, const float* draft_probs, const tt_logits* target,
+                  const tt_params* prm, void* workspace, size_t workspace_bytes,
+                  const tt_step_out* out, void* stream);
+
+/* Static text for a tt_status. */
+const char* tt_status_string(tt_status s);
+
+/* cudaError_t of the last failed launch in this process (0 if none). */
+int32_t tt_last_cuda_error(void);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int32_t tt_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TT_H */

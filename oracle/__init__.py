@@ -219,7 +219,8 @@ def step(wl, *, window: Optional[int] = None, temp_draft: Optional[float] = None
                 temp_target=temp_target, seed=seed, request_base=request_base, full_q=full_q,
                 draft_off=wl.draft_off, mp=al["map"], draft_logits=wl.draft_logits,
                 temp_draft=temp_draft)
-    status = al["status"] | tr["status"] | ve["status"]
+    # the fused step reports the alignment's problems first, else the later stages'
+    status = np.where(al["status"] != 0, al["status"], tr["status"] | ve["status"])
     out = dict(al)
     out.update(q_hat=tr["q_hat"], p_hat=ve["p_hat"], lse=ve["lse"], accepted=ve["accepted"],
                next_token=ve["next_token"], boundary=ve["boundary"], status=status)

@@ -332,7 +332,8 @@ void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols
         st |= ST_BAD_OFFSETS;
       } else {
         int32_t k = draft_off[b + 1] - draft_off[b];
-        for (int32_t j = 0; j < m; ++j)
+        if (k == 0) st |= ST_EMPTY;
+        for (int32_t j = 0; j < m && k > 0; ++j)
           if (map[t0 + j] < 0 || map[t0 + j] >= k) st |= ST_ID_RANGE;
       }
     }

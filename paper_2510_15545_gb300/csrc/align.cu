@@ -1,0 +1,298 @@
+// align.cu -- Dynamic Token Warping between draft and proxy target tokens
+// (§4.1, Alg. 1) with the byte-level Levenshtein token distance (App. F).
+//
+// One warp per request (sequence pair), several pairs per CTA. Per pair:
+//  1. stage the tokens' byte strings in shared memory (packed 8-byte words);
+//  2. fill the banded local-cost tile d(i,j) with all 32 lanes (bit-parallel
+//     edit distance for tokens of <= 8 bytes, a plain DP otherwise);
+//  3. sweep the anti-diagonals i + j = s: every cell of a diagonal depends
+//     only on the two previous diagonals, kept in three rotating shared
+//     buffers; each cell's choice of predecessor overwrites its cost in the
+//     tile (diagonal, then (i-1,j), then (i,j-1) on ties);
+//  4. backtrack from (k, m) on one lane, then write path, C*, the map
+//     i*(j) = max{i : (i,j) on the path} and the needed-draft-row flags.
+#include <cstdint>
+
+#include "tt_device.cuh"
+#include "tt_launch.h"
+
+namespace tt {
+
+namespace {
+
+// Bit i set iff byte i of the packed string P equals c.
+__device__ __forceinline__ uint32_t eq_mask8(uint64_t P, uint32_t c) {
+  uint32_t cc = c * 0x01010101u;
+  uint32_t lo = __vcmpeq4(uint32_t(P), cc), hi = __vcmpeq4(uint32_t(P >> 32), cc);
+  // gather the low bit of each 0x00/0xFF byte into 4 consecutive bits
+  uint32_t blo = (((lo & 0x01010101u) * 0x00204081u) >> 21) & 0xFu;
+  uint32_t bhi = (((hi & 0x01010101u) * 0x00204081u) >> 21) & 0xFu;
+  return blo | (bhi << 4);
+}
+
+// Edit distance of two byte strings of at most 8 bytes, packed little-endian,
+// by the bit-parallel column recurrence of Myers (1999) in Hyyro's form for
+// global distance: one pass over the text, one 8-bit vector per column.
+__device__ __forceinline__ int lev_packed8(uint64_t P, int lp, uint64_t T, int lt) {
+  if (lp == 0) return lt;
+  if (lt == 0) return lp;
+  const uint32_t mask = (1u << lp) - 1u, hb = 1u << (lp - 1);
+  uint32_t Pv = mask, Mv = 0;
+  int score = lp;
+  for (int x = 0; x < lt; ++x) {
+    uint32_t Eq = eq_mask8(P, uint32_t(T >> (8 * x)) & 0xFFu) & mask;
+    uint32_t Xv = Eq | Mv;
+    uint32_t Xh = (((Eq & Pv) + Pv) ^ Pv) | Eq;
+    uint32_t Ph = Mv | ~(Xh | Pv);
+    uint32_t Mh = Pv & Xh;
+    score += int((Ph & hb) != 0) - int((Mh & hb) != 0);
+    Ph = (Ph << 1) | 1u;  // row 0 of the edit table grows by one per column
+    Mh <<= 1;
+    Pv = Mh | ~(Xv | Ph);
+    Mv = Ph & Xv;
+  }
+  return score;
+}
+
+// Edit distance by the textbook row recurrence, for tokens longer than 8
+// bytes (bytes read from the global tables; ns, nt <= TT_MAX_TOKEN_BYTES).
+__device__ int lev_rows(const uint8_t* s, int ns, const uint8_t* t, int nt) {
+  if (ns > nt) {  // keep the row short
+    const uint8_t* u = s; s = t; t = u;
+    int n = ns; ns = nt; nt = n;
+  }
+  uint16_t row[TT_MAX_TOKEN_BYTES + 1];
+  for (int i = 0; i <= ns; ++i) row[i] = uint16_t(i);
+  for (int j = 1; j <= nt; ++j) {
+    uint8_t tj = t[j - 1];
+    int diag = row[0];
+    row[0] = uint16_t(j);
+    for (int i = 1; i <= ns; ++i) {
+      int up = row[i];
+      int v = min(min(up + 1, int(row[i - 1]) + 1), diag + (s[i - 1] == tj ? 0 : 1));
+      diag = up;
+      row[i] = uint16_t(v);
+    }
+  }
+  return row[ns];
+}
+
+struct PairSmem {
+  uint64_t* tok;  // [K + M] packed bytes (valid when len <= 8)
+  int32_t* diag;  // [3 * (K + 2)] rotating anti-diagonals, indexed by i
+  uint32_t* path; // [K + M] backtracked cells (i << 16 | j), reverse order
+  uint16_t* tile; // [K * TW] cost, then direction
+  uint16_t* len;  // [K + M] token byte lengths
+};
+
+__device__ __forceinline__ PairSmem carve(char* base, int K, int M, int TW) {
+  PairSmem s;
+  size_t off = 0;
+  s.tok = reinterpret_cast<uint64_t*>(base + off);
+  off += sizeof(uint64_t) * (K + M);
+  s.diag = reinterpret_cast<int32_t*>(base + off);
+  off += sizeof(int32_t) * 3 * (K + 2);
+  s.path = reinterpret_cast<uint32_t*>(base + off);
+  off += sizeof(uint32_t) * (K + M);
+  s.tile = reinterpret_cast<uint16_t*>(base + off);
+  off += sizeof(uint16_t) * size_t(K) * TW;
+  s.len = reinterpret_cast<uint16_t*>(base + off);
+  return s;
+}
+
+__global__ void __launch_bounds__(kAlignWarpsMax * 32)
+    align_kernel(AlignArgs a) {
+  extern __shared__ __align__(16) char smem_raw[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * a.warps_per_block + warp;
+  if (b >= a.B) return;
+  const int K = a.max_k, M = a.max_m, TW = a.tile_w;
+  PairSmem sm = carve(smem_raw + size_t(warp) * a.smem_per_warp, K, M, TW);
+
+  if (!csr_ok(a.draft_off, b, a.n_draft) || !csr_ok(a.target_off, b, a.n_target)) {
+    if (lane == 0) {
+      a.status[b] = TT_REQ_BAD_OFFSETS;
+      if (a.path_len) a.path_len[b] = 0;
+      if (a.cost) a.cost[b] = -1;
+    }
+    return;
+  }
+  const int d0 = a.draft_off[b], k = a.draft_off[b + 1] - d0;
+  const int t0 = a.target_off[b], m = a.target_off[b + 1] - t0;
+  if (a.excl) {  // scored column of each of the request's m + 1 target rows
+    for (int j = lane; j <= m; j += 32) {
+      int col = -1;
+      if (j < m) {
+        const int c = a.target_cols[t0 + j];
+        col = (c >= 0 && c < a.V_t) ? c : -1;
+      }
+      a.excl[t0 + b + j] = col;
+    }
+  }
+
+  int st = 0;
+  if (k == 0 || m == 0) st |= TT_REQ_EMPTY;
+  if (k > K || m > M || k > TT_MAX_K || m > TT_MAX_M) st |= TT_REQ_TOO_LONG;
+  if (st == 0) {
+    // stage every token: length and (if <= 8 bytes) its packed bytes
+    int flag = 0;
+    for (int x = lane; x < k + m; x += 32) {
+      const bool is_d = x < k;
+      const int id = is_d ? a.draft_ids[d0 + x] : a.target_ids[t0 + x - k];
+      const tt_vocab& v = is_d ? a.vd : a.vt;
+      uint16_t ln = 0;
+      uint64_t packed = 0;
+      if (id < 0 || id >= v.n_tokens) {
+        flag |= TT_REQ_ID_OUT_OF_RANGE;
+      } else {
+        const int64_t o0 = v.offsets[id], o1 = v.offsets[id + 1];
+        const int64_t n = o1 - o0;
+        if (o0 < 0 || o1 > v.n_bytes || n < 0) {
+          flag |= TT_REQ_ID_OUT_OF_RANGE;
+        } else if (n > TT_MAX_TOKEN_BYTES) {
+          flag |= TT_REQ_TOO_LONG;
+        } else {
+          ln = uint16_t(n);
+          if (n <= 8)
+            for (int y = 0; y < n; ++y) packed |= uint64_t(v.bytes[o0 + y]) << (8 * y);
+        }
+      }
+      sm.len[x] = ln;
+      sm.tok[x] = packed;
+    }
+    st = __reduce_or_sync(0xffffffffu, flag);
+  }
+  if (st != 0) {
+    for (int j = lane; j < m; j += 32)
+      if (a.map) a.map[t0 + j] = -1;
+    for (int i = lane; i < k; i += 32)
+      if (a.need) a.need[d0 + i] = 0;
+    if (lane == 0) {
+      a.status[b] = st;
+      if (a.path_len) a.path_len[b] = 0;
+      if (a.cost) a.cost[b] = -1;
+    }
+    return;
+  }
+
+  const int W0 = a.window < 0 ? k + m : max(a.window, abs(k - m));  // band half-width
+  const int tw = min(m, 2 * W0 + 1);                                 // tile cells per row
+
+  // 1. banded local costs; row i (1-based) holds j = jlo(i) .. jhi(i)
+  for (int idx = lane; idx < k * tw; idx += 32) {
+    const int i = idx / tw + 1, c = idx - (i - 1) * tw;
+    const int jlo = max(1, i - W0), j = jlo + c;
+    if (j > min(m, i + W0)) continue;
+    const int ld = sm.len[i - 1], lt = sm.len[k + j - 1];
+    int d;
+    if (ld <= 8 && lt <= 8) {
+      // pattern = the longer string, text = the shorter (fewer steps)
+      d = ld >= lt ? lev_packed8(sm.tok[i - 1], ld, sm.tok[k + j - 1], lt)
+                   : lev_packed8(sm.tok[k + j - 1], lt, sm.tok[i - 1], ld);
+    } else {
+      const int di = a.draft_ids[d0 + i - 1], ti = a.target_ids[t0 + j - 1];
+      d = lev_rows(a.vd.bytes + a.vd.offsets[di], ld, a.vt.bytes + a.vt.offsets[ti], lt);
+    }
+    sm.tile[size_t(i - 1) * TW + c] = uint16_t(d);
+  }
+
+  // 2. anti-diagonal sweep; buffer s % 3 holds C(i, s - i) at index i
+  int32_t* D[3] = {sm.diag, sm.diag + (K + 2), sm.diag + 2 * (K + 2)};
+  for (int i = lane; i <= k + 1; i += 32) {
+    D[0][i] = i == 0 ? 0 : kInf;  // s = 0: C(0,0) = 0
+    D[1][i] = kInf;               // s = 1: border cells only
+  }
+  __syncwarp();
+  for (int s = 2; s <= k + m; ++s) {
+    int32_t* cur = D[s % 3];
+    const int32_t* p1 = D[(s + 2) % 3];
+    const int32_t* p2 = D[(s + 1) % 3];
+    const int lo = max(max(1, s - m), (s - W0 + 1) >> 1);  // ceil((s - W0) / 2)
+    const int hi = min(min(k, s - 1), (s + W0) >> 1);
+    for (int i = lo + lane; i <= hi; i += 32) {
+      const int j = s - i;
+      const int up = p1[i - 1], left = p1[i], dg = p2[i - 1];
+      int best = dg, dir = 0;
+      if (up < best) { best = up; dir = 1; }
+      if (left < best) { best = left; dir = 2; }
+      uint16_t* cell = sm.tile + size_t(i - 1) * TW + (j - max(1, i - W0));
+      cur[i] = best >= kInf ? kInf : best + int(*cell);
+      *cell = uint16_t(dir);
+    }
+    if (lane == 0) {  // guards: neighbours just outside the diagonal read as infinite
+      if (lo - 1 >= 0) cur[lo - 1] = kInf;
+      if (hi + 1 <= k + 1) cur[hi + 1] = kInf;
+    }
+    __syncwarp();
+  }
+  const int cstar = D[(k + m) % 3][k];
+
+  // 3. backtrack on lane 0, from (k, m) to (1, 1)
+  int L = 0;
+  if (lane == 0) {
+    int i = k, j = m;
+    while (i > 0 && j > 0 && L < k + m) {
+      sm.path[L++] = (uint32_t(i) << 16) | uint32_t(j);
+      const int dir = sm.tile[size_t(i - 1) * TW + (j - max(1, i - W0))];
+      if (dir == 0) { --i; --j; }
+      else if (dir == 1) { --i; }
+      else { --j; }
+    }
+  }
+  L = __shfl_sync(0xffffffffu, L, 0);
+  for (int i = lane; i < k; i += 32)
+    if (a.need) a.need[d0 + i] = 0;
+  __syncwarp();
+
+  // 4. outputs in forward order
+  int32_t* pout = a.path ? a.path + 2 * (size_t(d0) + t0) : nullptr;
+  for (int x = lane; x < L; x += 32) {
+    const uint32_t cell = sm.path[L - 1 - x];
+    const int i = int(cell >> 16), j = int(cell & 0xffffu);
+    if (pout) {
+      pout[2 * x] = i - 1;
+      pout[2 * x + 1] = j - 1;
+    }
+    // last cell of column j on the path carries the largest i
+    const bool last_in_col = x == L - 1 || int(sm.path[L - 2 - x] & 0xffffu) != j;
+    if (last_in_col) {
+      if (a.map) a.map[t0 + j - 1] = i - 1;
+      if (a.need) a.need[d0 + i - 1] = 1;
+    }
+  }
+  if (lane == 0) {
+    a.status[b] = 0;
+    if (a.path_len) a.path_len[b] = L;
+    if (a.cost) a.cost[b] = cstar;
+  }
+}
+
+}  // namespace
+
+size_t align_smem_per_warp(int max_k, int max_m, int tile_w) {
+  size_t n = sizeof(uint64_t) * (max_k + max_m) + sizeof(int32_t) * 3 * (max_k + 2) +
+             sizeof(uint32_t) * (max_k + max_m) + sizeof(uint16_t) * size_t(max_k) * tile_w +
+             sizeof(uint16_t) * (max_k + max_m);
+  return (n + 15) & ~size_t(15);
+}
+
+int align_tile_width(int max_k, int max_m, int window) {
+  const int W0 = window < 0 ? max_k + max_m : max(window, max(max_k, max_m) - 1);
+  return min(max_m, 2 * W0 + 1);
+}
+
+cudaError_t launch_align(const AlignArgs& args, cudaStream_t stream) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(align_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kAlignSmemMax);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  const int blocks = (args.B + args.warps_per_block - 1) / args.warps_per_block;
+  const size_t smem = args.smem_per_warp * size_t(args.warps_per_block);
+  align_kernel<<<blocks, args.warps_per_block * 32, smem, stream>>>(args);
+  return cudaGetLastError();
+}
+
+}  // namespace tt

@@ -1,0 +1,389 @@
+// api.cu -- the extern "C" entry points declared in include/tt.h: argument
+// validation (before anything touches the GPU), workspace carving and the
+// launch sequences of align / transfer / verify / step.
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+
+#include "tt_device.cuh"
+#include "tt_launch.h"
+
+namespace {
+
+using namespace tt;
+
+int g_last_cuda_error = 0;
+
+tt_status cuda_fail(cudaError_t e) {
+  g_last_cuda_error = int(e);
+  return TT_ERR_CUDA;
+}
+
+int sm_count_current() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 148;
+  if (dev < 64 && cached[dev] > 0) return cached[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    n = 148;
+  if (dev < 64) cached[dev] = n;
+  return n;
+}
+
+bool batch_ok(const tt_batch* b) {
+  if (!b || b->B < 0 || b->n_draft < 0 || b->n_target < 0) return false;
+  if (b->B == 0) return true;
+  if (!b->draft_off || !b->target_off) return false;
+  if (b->max_k < 1 || b->max_k > TT_MAX_K || b->max_m < 1 || b->max_m > TT_MAX_M) return false;
+  if (int64_t(b->n_target) + b->B > INT32_MAX) return false;
+  return true;
+}
+
+bool dtype_ok(int32_t dt) { return dt == TT_F32 || dt == TT_BF16; }
+
+// Logits rows usable by the vectorised row pass.
+bool logits_ok(const tt_logits* L, int64_t rows_needed) {
+  if (!L || !L->data || !dtype_ok(L->dtype)) return false;
+  if (L->n_cols < 1 || int64_t(L->n_cols) > int64_t(kMaxChunksPerRow) * kChunk) return false;
+  if (L->row_stride < L->n_cols || L->n_rows < rows_needed) return false;
+  const int64_t esz = L->dtype == TT_F32 ? 4 : 2;
+  if ((reinterpret_cast<uintptr_t>(L->data) & 15) != 0) return false;
+  if ((L->row_stride * esz) % 16 != 0) return false;
+  return true;
+}
+
+bool params_ok(const tt_params* p) {
+  if (!p) return false;
+  if (!(p->temp_draft > 0.f) || !std::isfinite(p->temp_draft)) return false;
+  if (!(p->temp_target > 0.f) || !std::isfinite(p->temp_target)) return false;
+  if (p->full_q != 0 && p->full_q != 1) return false;
+  return true;
+}
+
+bool vocab_ok(const tt_vocab* v) {
+  return v && v->bytes && v->offsets && v->n_tokens >= 1 && v->n_bytes >= 0;
+}
+
+float log2e_over(float T) { return float(1.4426950408889634 / double(T)); }
+
+RowSet rowset(const tt_logits* L, Partial* part, const uint8_t* need, float T) {
+  RowSet r;
+  r.data = static_cast<const char*>(L->data);
+  r.stride_bytes = L->row_stride * (L->dtype == TT_F32 ? 4 : 2);
+  r.V = L->n_cols;
+  r.nch = n_chunks(L->n_cols);
+  r.scale = log2e_over(T);
+  r.part = part;
+  r.need = need;
+  return r;
+}
+
+RowSet no_rows() {
+  RowSet r;
+  std::memset(&r, 0, sizeof r);
+  r.nch = 1;
+  return r;
+}
+
+void record(const tt_params* p, int i, cudaStream_t s) {
+  if (p->events && p->events[i]) cudaEventRecord(static_cast<cudaEvent_t>(p->events[i]), s);
+}
+
+tt_status fill_align_args(const tt_batch* bt, const tt_vocab* vd, const tt_vocab* vt,
+                          const tt_params* prm, AlignArgs& a) {
+  std::memset(&a, 0, sizeof a);
+  a.B = bt->B;
+  a.n_draft = bt->n_draft;
+  a.n_target = bt->n_target;
+  a.max_k = bt->max_k;
+  a.max_m = bt->max_m;
+  a.window = prm->window;
+  a.draft_off = bt->draft_off;
+  a.draft_ids = bt->draft_ids;
+  a.target_off = bt->target_off;
+  a.target_ids = bt->target_ids;
+  a.vd = *vd;
+  a.vt = *vt;
+  a.tile_w = align_tile_width(bt->max_k, bt->max_m, prm->window);
+  a.smem_per_warp = align_smem_per_warp(bt->max_k, bt->max_m, a.tile_w);
+  if (a.smem_per_warp > size_t(kAlignSmemMax)) return TT_ERR_UNSUPPORTED;
+  int wpb = int(size_t(96 * 1024) / a.smem_per_warp);
+  wpb = wpb < 1 ? 1 : (wpb > kAlignWarpsMax ? kAlignWarpsMax : wpb);
+  a.warps_per_block = wpb;
+  return TT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t tt_workspace_bytes(const tt_batch* batch, int32_t V_d, int32_t V_t) {
+  if (!batch || batch->B < 0 || batch->n_draft < 0 || batch->n_target < 0) return 0;
+  return workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d < 0 ? 0 : V_d,
+                          V_t < 0 ? 0 : V_t)
+      .bytes;
+}
+
+tt_status tt_align(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
+                   const tt_params* prm, int32_t* path, int32_t* path_len, int32_t* cost,
+                   int32_t* map, int32_t* status, void* stream) {
+  if (!batch_ok(batch) || !params_ok(prm)) return TT_ERR_INVALID_ARG;
+  if (batch->B == 0) return TT_OK;
+  if (!vocab_ok(vd) || !vocab_ok(vt) || !status) return TT_ERR_INVALID_ARG;
+  if ((batch->n_draft > 0 && !batch->draft_ids) || (batch->n_target > 0 && !batch->target_ids))
+    return TT_ERR_INVALID_ARG;
+  AlignArgs a;
+  tt_status st = fill_align_args(batch, vd, vt, prm, a);
+  if (st != TT_OK) return st;
+  a.path = path;
+  a.path_len = path_len;
+  a.cost = cost;
+  a.map = map;
+  a.status = status;
+  cudaError_t e = launch_align(a, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TT_OK : cuda_fail(e);
+}
+
+tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits* draft,
+                      const float* draft_probs, const tt_params* prm, void* workspace,
+                      size_t workspace_bytes, float* q_hat, int32_t* status, void* stream) {
+  if (!batch_ok(batch) || !params_ok(prm)) return TT_ERR_INVALID_ARG;
+  if (batch->B == 0) return TT_OK;
+  if (!q_hat || !status || (batch->n_target > 0 && !map)) return TT_ERR_INVALID_ARG;
+  const bool from_logits = draft_probs == nullptr;
+  if (from_logits && !logits_ok(draft, batch->n_draft)) return TT_ERR_INVALID_ARG;
+  const int32_t* cols = batch->draft_cols ? batch->draft_cols : batch->draft_ids;
+  if (from_logits && batch->n_draft > 0 && !cols) return TT_ERR_INVALID_ARG;
+  const int V_d = from_logits ? draft->n_cols : 0;
+  const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d, 0).bytes;
+  if (from_logits && (!workspace || workspace_bytes < need ||
+                      (reinterpret_cast<uintptr_t>(workspace) & 255) != 0))
+    return TT_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d, 0);
+
+  DecideArgs d;
+  std::memset(&d, 0, sizeof d);
+  d.B = batch->B;
+  d.n_draft = batch->n_draft;
+  d.n_target = batch->n_target;
+  d.max_m = batch->max_m;
+  d.mode_transfer_only = 1;
+  d.draft_off = batch->draft_off;
+  d.draft_cols = cols;
+  d.target_off = batch->target_off;
+  d.map = map;
+  d.draft_probs = draft_probs;
+  d.d = from_logits ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
+  d.t = no_rows();
+  d.dt_d = from_logits ? draft->dtype : TT_F32;
+  d.status = status;
+  d.q_hat_out = q_hat;
+  cudaError_t e;
+  if (from_logits) {
+    PrepArgs p;
+    std::memset(&p, 0, sizeof p);
+    p.B = batch->B;
+    p.n_draft = batch->n_draft;
+    p.n_target = batch->n_target;
+    p.draft_off = batch->draft_off;
+    p.target_off = batch->target_off;
+    p.map = map;
+    p.need = ws.need_d;
+    if ((e = launch_prep(p, s)) != cudaSuccess) return cuda_fail(e);
+    RowPassArgs r;
+    std::memset(&r, 0, sizeof r);
+    r.d = d.d;
+    r.t = no_rows();
+    r.items_d = int64_t(batch->n_draft) * d.d.nch;
+    r.items_t = 0;
+    if ((e = launch_rowpass(r, draft->dtype, TT_F32, s, sm_count_current())) != cudaSuccess)
+      return cuda_fail(e);
+  }
+  if ((e = launch_decide(d, s)) != cudaSuccess) return cuda_fail(e);
+  return TT_OK;
+}
+
+tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* target,
+                    const tt_logits* draft, const int32_t* map, const tt_params* prm,
+                    void* workspace, size_t workspace_bytes, int32_t* accepted,
+                    int32_t* next_token, float* p_hat, float* lse, int32_t* status,
+                    void* stream) {
+  if (!batch_ok(batch) || !params_ok(prm)) return TT_ERR_INVALID_ARG;
+  if (batch->B == 0) return TT_OK;
+  if (!accepted || !next_token || !status) return TT_ERR_INVALID_ARG;
+  if (batch->n_target > 0 && !q_hat) return TT_ERR_INVALID_ARG;
+  const int32_t* tcols = batch->target_cols ? batch->target_cols : batch->target_ids;
+  if (batch->n_target > 0 && !tcols) return TT_ERR_INVALID_ARG;
+  if (!logits_ok(target, int64_t(batch->n_target) + batch->B)) return TT_ERR_INVALID_ARG;
+  const bool full_q = prm->full_q != 0;
+  if (full_q) {
+    if (!logits_ok(draft, batch->n_draft) || draft->n_cols != target->n_cols) return TT_ERR_INVALID_ARG;
+    if (batch->n_target > 0 && !map) return TT_ERR_INVALID_ARG;
+  }
+  const int V_d = full_q ? draft->n_cols : 0;
+  const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d,
+                                       target->n_cols).bytes;
+  if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
+    return TT_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d,
+                                  target->n_cols);
+  PrepArgs p;
+  std::memset(&p, 0, sizeof p);
+  p.B = batch->B;
+  p.n_draft = batch->n_draft;
+  p.n_target = batch->n_target;
+  p.V_t = target->n_cols;
+  p.draft_off = batch->draft_off;
+  p.target_off = batch->target_off;
+  p.target_cols = tcols;
+  p.map = map;
+  p.excl = ws.excl;
+  p.need = full_q ? ws.need_d : nullptr;
+  cudaError_t e;
+  if ((e = launch_prep(p, s)) != cudaSuccess) return cuda_fail(e);
+
+  RowPassArgs r;
+  std::memset(&r, 0, sizeof r);
+  r.t = rowset(target, ws.part_t, nullptr, prm->temp_target);
+  r.items_t = (int64_t(batch->n_target) + batch->B) * r.t.nch;
+  r.d = full_q ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
+  r.items_d = full_q ? int64_t(batch->n_draft) * r.d.nch : 0;
+  r.excl = ws.excl;
+  if ((e = launch_rowpass(r, full_q ? draft->dtype : TT_F32, target->dtype, s,
+                          sm_count_current())) != cudaSuccess)
+    return cuda_fail(e);
+
+  DecideArgs d;
+  std::memset(&d, 0, sizeof d);
+  d.B = batch->B;
+  d.n_draft = batch->n_draft;
+  d.n_target = batch->n_target;
+  d.max_m = batch->max_m;
+  d.full_q = full_q ? 1 : 0;
+  d.draft_off = batch->draft_off;
+  d.target_off = batch->target_off;
+  d.target_cols = tcols;
+  d.map = map;
+  d.q_hat_in = q_hat;
+  d.d = r.d;
+  d.t = r.t;
+  d.dt_d = full_q ? draft->dtype : TT_F32;
+  d.dt_t = target->dtype;
+  d.seed = prm->seed;
+  d.request_base = prm->request_base;
+  d.accepted = accepted;
+  d.next_token = next_token;
+  d.status = status;
+  d.p_hat = p_hat;
+  d.lse = lse;
+  if ((e = launch_decide(d, s)) != cudaSuccess) return cuda_fail(e);
+  return TT_OK;
+}
+
+tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
+                  const tt_logits* draft, const float* draft_probs, const tt_logits* target,
+                  const tt_params* prm, void* workspace, size_t workspace_bytes,
+                  const tt_step_out* out, void* stream) {
+  if (!batch_ok(batch) || !params_ok(prm)) return TT_ERR_INVALID_ARG;
+  if (!out || !out->accepted || !out->next_token || !out->status) return TT_ERR_INVALID_ARG;
+  if (batch->B == 0) return TT_OK;
+  if (!vocab_ok(vd) || !vocab_ok(vt)) return TT_ERR_INVALID_ARG;
+  if ((batch->n_draft > 0 && !batch->draft_ids) || (batch->n_target > 0 && !batch->target_ids))
+    return TT_ERR_INVALID_ARG;
+  const bool full_q = prm->full_q != 0;
+  const bool from_logits = draft_probs == nullptr || full_q;
+  if (!logits_ok(target, int64_t(batch->n_target) + batch->B)) return TT_ERR_INVALID_ARG;
+  if (from_logits && !logits_ok(draft, batch->n_draft)) return TT_ERR_INVALID_ARG;
+  if (full_q && draft->n_cols != target->n_cols) return TT_ERR_INVALID_ARG;
+  const int V_d = from_logits ? draft->n_cols : 0;
+  const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d,
+                                       target->n_cols).bytes;
+  if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
+    return TT_ERR_INVALID_ARG;
+  const int32_t* dcols = batch->draft_cols ? batch->draft_cols : batch->draft_ids;
+  const int32_t* tcols = batch->target_cols ? batch->target_cols : batch->target_ids;
+  AlignArgs a;
+  tt_status st = fill_align_args(batch, vd, vt, prm, a);
+  if (st != TT_OK) return st;
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d,
+                                  target->n_cols);
+  int32_t* map = out->map ? out->map : ws.map;
+  a.path = out->path;
+  a.path_len = out->path_len;
+  a.cost = out->cost;
+  a.map = map;
+  a.status = out->status;
+  a.need = from_logits ? ws.need_d : nullptr;
+  a.target_cols = tcols;
+  a.V_t = target->n_cols;
+  a.excl = ws.excl;
+
+  cudaError_t e;
+  record(prm, 0, s);
+  if ((e = launch_align(a, s)) != cudaSuccess) return cuda_fail(e);
+  record(prm, 1, s);
+
+  RowPassArgs r;
+  std::memset(&r, 0, sizeof r);
+  r.t = rowset(target, ws.part_t, nullptr, prm->temp_target);
+  r.items_t = (int64_t(batch->n_target) + batch->B) * r.t.nch;
+  r.d = from_logits ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
+  r.items_d = from_logits ? int64_t(batch->n_draft) * r.d.nch : 0;
+  r.excl = ws.excl;
+  if ((e = launch_rowpass(r, from_logits ? draft->dtype : TT_F32, target->dtype, s,
+                          sm_count_current())) != cudaSuccess)
+    return cuda_fail(e);
+  record(prm, 2, s);
+
+  DecideArgs d;
+  std::memset(&d, 0, sizeof d);
+  d.B = batch->B;
+  d.n_draft = batch->n_draft;
+  d.n_target = batch->n_target;
+  d.max_m = batch->max_m;
+  d.full_q = full_q ? 1 : 0;
+  d.draft_off = batch->draft_off;
+  d.draft_cols = dcols;
+  d.target_off = batch->target_off;
+  d.target_cols = tcols;
+  d.map = map;
+  d.q_hat_in = nullptr;
+  d.draft_probs = full_q ? nullptr : draft_probs;
+  d.d = r.d;
+  d.t = r.t;
+  d.dt_d = from_logits ? draft->dtype : TT_F32;
+  d.dt_t = target->dtype;
+  d.status_in = out->status;
+  d.seed = prm->seed;
+  d.request_base = prm->request_base;
+  d.accepted = out->accepted;
+  d.next_token = out->next_token;
+  d.status = out->status;
+  d.q_hat_out = out->q_hat;
+  d.p_hat = out->p_hat;
+  d.lse = out->lse;
+  if ((e = launch_decide(d, s)) != cudaSuccess) return cuda_fail(e);
+  record(prm, 3, s);
+  return TT_OK;
+}
+
+const char* tt_status_string(tt_status s) {
+  switch (s) {
+    case TT_OK: return "ok";
+    case TT_ERR_INVALID_ARG: return "invalid argument";
+    case TT_ERR_UNSUPPORTED: return "unsupported configuration";
+    case TT_ERR_CUDA: return "CUDA launch failure";
+  }
+  return "unknown status";
+}
+
+int32_t tt_last_cuda_error(void) { return g_last_cuda_error; }
+
+int32_t tt_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,180 @@
+// tt_device.cuh -- device helpers and the workspace layout shared by the
+// kernels of the TokenTiming verification path (sm_103a).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/tt.h"
+
+namespace tt {
+
+constexpr int kChunk = 8192;         // logits elements per row chunk (one partial)
+constexpr int kRowThreads = 256;     // threads of the row-pass and decision blocks
+constexpr int32_t kInf = 0x3fffffff; // "infinite" accumulated DTW cost
+
+// -------------------------------------------------------------- workspace
+
+__host__ __device__ inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+__host__ __device__ inline int n_chunks(int V) { return V <= 0 ? 0 : (V + kChunk - 1) / kChunk; }
+
+// Partial of one row chunk: m = max of s_x = z_x * log2(e) / T over the chunk,
+// s = sum of 2^(s_x - m) over the chunk (target rows leave out their scored
+// token, whose term is rebuilt exactly by the decision kernel).
+struct Partial {
+  float m;
+  float s;
+};
+
+struct Workspace {
+  Partial* part_d;   // [n_draft * nch_d]
+  Partial* part_t;   // [(n_target + B) * nch_t]
+  uint8_t* need_d;   // [n_draft]: draft row is mapped by some target position
+  int32_t* map;      // [n_target] alignment map when the caller keeps none
+  float* q_hat;      // [n_target] transferred probabilities when the caller keeps none
+  int32_t* status;   // [B] per-request status between kernels
+  int32_t* excl;     // [n_target + B] scored column of each target row (-1: bonus row)
+  size_t bytes;
+};
+
+__host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_draft, int n_target,
+                                                      int V_d, int V_t) {
+  Workspace w;
+  char* p = static_cast<char*>(base);
+  size_t off = 0;
+  auto take = [&](size_t n) {
+    char* r = p ? p + off : nullptr;
+    off = align256(off + n);
+    return r;
+  };
+  w.part_d = reinterpret_cast<Partial*>(take(sizeof(Partial) * size_t(n_draft) * n_chunks(V_d)));
+  w.part_t = reinterpret_cast<Partial*>(
+      take(sizeof(Partial) * size_t(n_target + B) * n_chunks(V_t)));
+  w.need_d = reinterpret_cast<uint8_t*>(take(size_t(n_draft)));
+  w.map = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * size_t(n_target)));
+  w.q_hat = reinterpret_cast<float*>(take(sizeof(float) * size_t(n_target)));
+  w.status = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * size_t(B)));
+  w.excl = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (size_t(n_target) + B)));
+  w.bytes = off;
+  return w;
+}
+
+// ------------------------------------------------------------------ loads
+
+__device__ __forceinline__ float bf16_to_f32(uint16_t h) {
+  return __uint_as_float(uint32_t(h) << 16);
+}
+
+template <int DT>
+__device__ __forceinline__ float load_logit(const void* row, int64_t x) {
+  if constexpr (DT == TT_F32) {
+    return __ldg(static_cast<const float*>(row) + x);
+  } else {
+    return bf16_to_f32(__ldg(static_cast<const unsigned short*>(row) + x));
+  }
+}
+
+// 16-byte streaming load that does not allocate in L1.
+__device__ __forceinline__ uint4 ld_stream_v4(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// -------------------------------------------------------------- reductions
+
+// Merge two (max, sum-of-2^(s - max)) pairs.
+__device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2) {
+  if (m2 > m) {
+    s = s2 + (m == -INFINITY ? 0.f : s * ex2_approx(m - m2));
+    m = m2;
+  } else if (m2 != -INFINITY) {
+    s += s2 * ex2_approx(m2 - m);
+  }
+}
+
+__device__ __forceinline__ void warp_merge_ms(float& m, float& s) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    merge_ms(m, s, m2, s2);
+  }
+}
+
+__device__ __forceinline__ double warp_sum_d(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float warp_max_f(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Log2-normaliser of a row from its chunk partials, computed by one warp:
+// returns (M, S) with sum over the row of 2^(s_x - M) = S (excluding what the
+// partials exclude). S accumulates in fp64.
+__device__ __forceinline__ void row_norm_warp(const Partial* part, int nch, int lane, float& M,
+                                              double& S) {
+  float mx = -INFINITY;
+  for (int c = lane; c < nch; c += 32) mx = fmaxf(mx, part[c].m);
+  mx = warp_max_f(mx);
+  double acc = 0.0;
+  if (mx != -INFINITY) {
+    for (int c = lane; c < nch; c += 32) {
+      Partial p = part[c];
+      if (p.m != -INFINITY) acc += double(p.s) * double(ex2_approx(p.m - mx));
+    }
+  }
+  M = mx;
+  S = warp_sum_d(acc);
+}
+
+// ----------------------------------------------------------------- Philox
+
+__device__ __forceinline__ void philox4x64_10(uint64_t c[4], uint64_t k0, uint64_t k1) {
+  const uint64_t M0 = 0xD2E7470EE14C6C93ULL, M1 = 0xCA5A826395121157ULL;
+  const uint64_t W0 = 0x9E3779B97F4A7C15ULL, W1 = 0xBB67AE8584CAA73BULL;
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    uint64_t lo0 = M0 * c[0], hi0 = __umul64hi(M0, c[0]);
+    uint64_t lo1 = M1 * c[2], hi1 = __umul64hi(M1, c[2]);
+    uint64_t n0 = hi1 ^ c[1] ^ k0, n2 = hi0 ^ c[3] ^ k1;
+    c[0] = n0;
+    c[1] = lo1;
+    c[2] = n2;
+    c[3] = lo0;
+    k0 += W0;
+    k1 += W1;
+  }
+}
+
+// u in [0,1): top 24 bits of word 0 of Philox4x64-10 at counter
+// (pos, stream, request, 0), key (seed, 0). Exact in fp32 and fp64.
+__device__ __forceinline__ double philox_uniform(uint64_t seed, uint64_t pos, uint64_t stream,
+                                                 uint64_t request) {
+  uint64_t c[4] = {pos, stream, request, 0};
+  philox4x64_10(c, seed, 0);
+  return double(c[0] >> 40) * (1.0 / 16777216.0);
+}
+
+// ------------------------------------------------------------ CSR helpers
+
+// Offsets of request b are usable: 0 <= off[b] <= off[b+1] <= n.
+__device__ __forceinline__ bool csr_ok(const int32_t* off, int b, int n) {
+  int a = off[b], e = off[b + 1];
+  return a >= 0 && a <= e && e <= n;
+}
+
+}  // namespace tt

@@ -234,6 +234,32 @@ class Workload:
     def max_m(self) -> int:
         return int(np.diff(self.target_off).max(initial=0))
 
+    def subset(self, idx) -> "Workload":
+        """Requests ``idx`` as a workload of their own (logits copied to the CPU)."""
+        idx = [int(b) for b in idx]
+        d_rows, t_rows, d_ids, t_ids, d_cols, t_cols = [], [], [], [], [], []
+        d_off, t_off = [0], [0]
+        for b in idx:
+            d0, d1 = int(self.draft_off[b]), int(self.draft_off[b + 1])
+            o0, o1 = int(self.target_off[b]), int(self.target_off[b + 1])
+            d_rows.extend(range(d0, d1))
+            t_rows.extend(range(o0 + b, o1 + b + 1))
+            d_ids.append(self.draft_ids[d0:d1])
+            d_cols.append(self.draft_cols[d0:d1])
+            t_ids.append(self.target_ids[o0:o1])
+            t_cols.append(self.target_cols[o0:o1])
+            d_off.append(d_off[-1] + d1 - d0)
+            t_off.append(t_off[-1] + o1 - o0)
+
+        def cat(xs):
+            return np.concatenate(xs).astype(np.int32) if xs else np.zeros(0, np.int32)
+        dl = self.draft_logits[torch.as_tensor(d_rows, device=self.draft_logits.device)].cpu()
+        tl = self.target_logits[torch.as_tensor(t_rows, device=self.target_logits.device)].cpu()
+        return dataclasses.replace(self, draft_off=np.array(d_off, np.int32),
+                                   target_off=np.array(t_off, np.int32), draft_ids=cat(d_ids),
+                                   target_ids=cat(t_ids), draft_cols=cat(d_cols),
+                                   target_cols=cat(t_cols), draft_logits=dl, target_logits=tl)
+
     def request(self, b: int) -> dict:
         d0, d1 = int(self.draft_off[b]), int(self.draft_off[b + 1])
         t0, t1 = int(self.target_off[b]), int(self.target_off[b + 1])
@@ -361,7 +387,8 @@ def make_workload(name: str, *, B: Optional[int] = None, seed: int = 0,
 
     target_logits = _gen_rows(spec, n_target + B, V_tl, gen, device)
     if spec.corr_frac > 0:
-        _correlate(spec, target_logits, draft_logits, draft_off, target_off, vd, vt, rng, device)
+        _correlate(spec, target_logits, draft_logits, draft_off, target_off, draft_ids_flat,
+                   target_ids, vd, vt, rng, device)
 
     if spec.verify_V:
         draft_cols = (draft_ids_flat % spec.verify_V).astype(np.int32)
@@ -376,10 +403,21 @@ def make_workload(name: str, *, B: Optional[int] = None, seed: int = 0,
                     target_logits=target_logits.to(spec.dtype))
 
 
-def _correlate(spec, target_logits, draft_logits, draft_off, target_off, vd, vt, rng, device):
-    """Makes ``corr_frac`` of the target rows correlated (coefficient ``corr_rho``)
-    with the draft row at the proportional position of the same request, through
-    the injection that sends a target string to the draft id spelling it."""
+def _source_rows(vd, vt, d_ids, t_ids) -> np.ndarray:
+    """For each target token, the draft token holding its last byte (tokenizer
+    bookkeeping of the re-encoding, not an alignment)."""
+    ends = np.cumsum([len(vd.strings[i]) for i in d_ids])
+    t_ends = np.cumsum([len(vt.strings[i]) for i in t_ids])
+    return np.searchsorted(ends, t_ends - 1, side="right").clip(max=len(d_ids) - 1)
+
+
+def _correlate(spec, target_logits, draft_logits, draft_off, target_off, draft_ids, target_ids,
+               vd, vt, rng, device):
+    """Makes the target rows of a fraction ``corr_frac`` of the requests
+    correlated (coefficient ``corr_rho``) with the draft row holding the same
+    bytes, through the injection that sends a target string to the draft id
+    spelling it: z_t = rho * z_d + sqrt(1 - rho^2) * sd(z_d) * N(0, 1). The
+    bonus row follows the last draft row."""
     inj = np.full(vt.n_tokens, -1, dtype=np.int64)
     for tid, s in enumerate(vt.strings):
         did = vd.index.get(s)
@@ -390,18 +428,20 @@ def _correlate(spec, target_logits, draft_logits, draft_off, target_off, vd, vt,
     from_d = torch.as_tensor(inj[have], device=device)
     rho = spec.corr_rho
     B = len(draft_off) - 1
-    for b in range(B):
-        k = int(draft_off[b + 1] - draft_off[b])
-        m = int(target_off[b + 1] - target_off[b])
-        for j in range(m + 1):
-            if rng.random() >= spec.corr_frac:
-                continue
-            i = min(k - 1, (j * k) // max(m, 1))
-            r_t = int(target_off[b]) + b + j
-            r_d = int(draft_off[b]) + i
-            row = target_logits[r_t]
-            src = draft_logits[r_d, from_d]
-            row[have_t] = rho * src + math.sqrt(1 - rho * rho) * row[have_t]
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(rng.integers(0, 2**31)))
+    chosen = rng.random(B) < spec.corr_frac
+    for b in np.nonzero(chosen)[0]:
+        d0, d1 = int(draft_off[b]), int(draft_off[b + 1])
+        t0, t1 = int(target_off[b]), int(target_off[b + 1])
+        src = _source_rows(vd, vt, draft_ids[d0:d1], target_ids[t0:t1])
+        src = np.concatenate([src, [d1 - d0 - 1]])
+        for j, i in enumerate(src):
+            zd = draft_logits[d0 + int(i), from_d]
+            sd = float(zd.std())
+            noise = torch.randn(zd.shape, generator=gen, device=device) * sd
+            row = target_logits[t0 + b + j]
+            row[have_t] = rho * zd + math.sqrt(1 - rho * rho) * noise
 
 
 def homogeneous_workload(B: int, k: int, V: int, *, seed: int = 0, device: str = "cpu",
