@@ -69,6 +69,11 @@ def dist_init(ws, backend):
         dist.init_process_group(backend=backend)
 
 
+def request_base(rank: int, batch: int) -> int:
+    """Global index of a rank's first request: ranks own disjoint Philox streams."""
+    return rank * batch
+
+
 def barrier(ws):
     if ws > 1:
         import torch.distributed as dist
@@ -264,7 +269,7 @@ def run_mine(args):
     wl = W.make_workload(name, seed=rank, device=str(dev))
     inp = tt.device_inputs(wl, dev)
     prm = inp["params"]
-    prm.request_base = rank * wl.B
+    prm.request_base = request_base(rank, wl.B)
     batch, vd, vt = inp["batch"], inp["vd"], inp["vt"]
     dl, tl = inp["draft_logits"], inp["target_logits"]
     stream = torch.cuda.current_stream(dev)

@@ -274,13 +274,13 @@ def _affine_perm_ranks(gen: torch.Generator, R: int, V: int, device) -> torch.Te
     """1-based ranks under a random affine permutation x -> (a x + c) mod V per
     row (a coprime to V): a cheap stand-in for an independent random
     permutation of the vocabulary in every row."""
-    a = torch.randint(1, V, (R,), generator=gen, device="cpu", dtype=torch.int64).numpy()
+    a = torch.randint(1, V, (R,), generator=gen, device=device, dtype=torch.int64).cpu().numpy()
     bad = np.gcd(a, V) != 1
     while bad.any():  # step to the next candidate; 1 is always coprime
         a[bad] = a[bad] % (V - 1) + 1
         bad = np.gcd(a, V) != 1
     a = torch.from_numpy(a)
-    c = torch.randint(0, V, (R,), generator=gen, device="cpu", dtype=torch.int64)
+    c = torch.randint(0, V, (R,), generator=gen, device=device, dtype=torch.int64).cpu()
     x = torch.arange(V, device=device, dtype=torch.int64)
     return ((x[None, :] * a.to(device)[:, None] + c.to(device)[:, None]) % V) + 1
 

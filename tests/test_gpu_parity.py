@@ -160,18 +160,25 @@ def test_transfer_and_verify_ragged_widths(dtype, V):
     gen = torch.Generator().manual_seed(V)
     dl = (torch.randn((nd, V), generator=gen) * 2.5).to(dtype)
     tl = (torch.randn((nt + B, V), generator=gen) * 2.5).to(dtype)
+    # rows start on 16-byte boundaries (the row pass's contract): pad the stride
+    pad = -V % 8
+
+    def padded(x):
+        st = torch.full((x.shape[0], V + pad), float("nan"), dtype=dtype, device="cuda")
+        st[:, :V] = x.cuda()
+        return st[:, :V]
     d_cols = rng.integers(0, V, size=nd).astype(np.int32)
     t_cols = rng.integers(0, V, size=nt).astype(np.int32)
     mp = np.concatenate([np.sort(rng.integers(0, k, size=m)) for m in ms]).astype(np.int32)
     batch = tt.Batch.from_host(d_off, d_cols, t_off, t_cols, device="cuda")
     prm = tt.Params(temp_draft=0.8, temp_target=1.3, seed=7)
     mp_d = torch.as_tensor(mp, device="cuda")
-    gt = to_np(tt.tt_transfer(batch, mp_d, prm, draft_logits=dl.cuda()))
+    gt = to_np(tt.tt_transfer(batch, mp_d, prm, draft_logits=padded(dl)))
     ot = oracle.transfer(d_off, d_cols, t_off, mp, dl, 0.8)
     assert np.array_equal(gt["status"], ot["status"])
     assert np.max(np.abs(gt["q_hat"][:nt] - ot["q_hat"])) <= TOL
     q = torch.as_tensor(gt["q_hat"][:nt], device="cuda")
-    gv = to_np(tt.tt_verify(batch, q, tl.cuda(), prm))
+    gv = to_np(tt.tt_verify(batch, q, padded(tl), prm))
     ov = oracle.verify(t_off, t_cols, gt["q_hat"][:nt].astype(np.float64), tl, temp_target=1.3,
                        seed=7)
     g = dict(gv, _target_off=t_off, _draft_off=d_off)
