@@ -68,6 +68,10 @@ typedef enum {
 #define TT_REQ_EMPTY 4           /* k == 0 or m == 0 */
 #define TT_REQ_BAD_OFFSETS 8     /* CSR offsets decreasing or outside [0, n_draft/n_target] */
 #define TT_REQ_NOT_FINITE 16     /* a logits row gave a non-finite normaliser */
+#define TT_REQ_TIMEOUT 32        /* a pipeline wait in the row pass gave up (bounded waits);
+                                    the step's results are not valid */
+#define TT_REQ_INTERNAL 64       /* an internal bounds check in a kernel failed (the access
+                                    was skipped); the step's results are not valid */
 
 typedef enum { TT_F32 = 0, TT_BF16 = 1 } tt_dtype;
 

@@ -103,6 +103,9 @@ __device__ __forceinline__ PairSmem carve(char* base, int K, int M, int TW) {
 __global__ void __launch_bounds__(kAlignWarpsMax * 32)
     align_kernel(AlignArgs a) {
   extern __shared__ __align__(16) char smem_raw[];
+  // the row pass may start streaming target rows now; it waits for this grid
+  // before it reads the needed-draft-row flags
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * a.warps_per_block + warp;
   if (b >= a.B) return;
@@ -119,17 +122,6 @@ __global__ void __launch_bounds__(kAlignWarpsMax * 32)
   }
   const int d0 = a.draft_off[b], k = a.draft_off[b + 1] - d0;
   const int t0 = a.target_off[b], m = a.target_off[b + 1] - t0;
-  if (a.excl) {  // scored column of each of the request's m + 1 target rows
-    for (int j = lane; j <= m; j += 32) {
-      int col = -1;
-      if (j < m) {
-        const int c = a.target_cols[t0 + j];
-        col = (c >= 0 && c < a.V_t) ? c : -1;
-      }
-      a.excl[t0 + b + j] = col;
-    }
-  }
-
   int st = 0;
   if (k == 0 || m == 0) st |= TT_REQ_EMPTY;
   if (k > K || m > M || k > TT_MAX_K || m > TT_MAX_M) st |= TT_REQ_TOO_LONG;
@@ -281,14 +273,12 @@ int align_tile_width(int max_k, int max_m, int window) {
   return min(max_m, 2 * W0 + 1);
 }
 
+cudaError_t preload_align() {
+  return cudaFuncSetAttribute(align_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              kAlignSmemMax);
+}
+
 cudaError_t launch_align(const AlignArgs& args, cudaStream_t stream) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(align_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kAlignSmemMax);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
   const int blocks = (args.B + args.warps_per_block - 1) / args.warps_per_block;
   const size_t smem = args.smem_per_warp * size_t(args.warps_per_block);
   align_kernel<<<blocks, args.warps_per_block * 32, smem, stream>>>(args);

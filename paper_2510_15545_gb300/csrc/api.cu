@@ -1,6 +1,7 @@
 // api.cu -- the extern "C" entry points declared in include/tt.h: argument
 // validation (before anything touches the GPU), workspace carving and the
 // launch sequences of align / transfer / verify / step.
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -13,10 +14,27 @@ namespace {
 using namespace tt;
 
 int g_last_cuda_error = 0;
+std::atomic<int32_t> g_epoch{0x2b6f1000};  // tags each call's row-pass error word
+
+int32_t next_epoch() { return ++g_epoch; }
 
 tt_status cuda_fail(cudaError_t e) {
   g_last_cuda_error = int(e);
   return TT_ERR_CUDA;
+}
+
+// Loads all kernels on the current device once, before the first launch there.
+cudaError_t ensure_loaded() {
+  static bool done[64] = {false};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev >= 0 && dev < 64 && done[dev]) return cudaSuccess;
+  if ((e = preload_align()) != cudaSuccess) return e;
+  if ((e = preload_rowpass()) != cudaSuccess) return e;
+  if ((e = preload_decide()) != cudaSuccess) return e;
+  if (dev >= 0 && dev < 64) done[dev] = true;
+  return cudaSuccess;
 }
 
 int sm_count_current() {
@@ -74,6 +92,7 @@ RowSet rowset(const tt_logits* L, Partial* part, const uint8_t* need, float T) {
   r.V = L->n_cols;
   r.nch = n_chunks(L->n_cols);
   r.scale = log2e_over(T);
+  r.n_rows = L->n_rows;
   r.part = part;
   r.need = need;
   return r;
@@ -141,7 +160,8 @@ tt_status tt_align(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt
   a.cost = cost;
   a.map = map;
   a.status = status;
-  cudaError_t e = launch_align(a, static_cast<cudaStream_t>(stream));
+  cudaError_t e = ensure_loaded();
+  if (e == cudaSuccess) e = launch_align(a, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? TT_OK : cuda_fail(e);
 }
 
@@ -180,7 +200,8 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   d.dt_d = from_logits ? draft->dtype : TT_F32;
   d.status = status;
   d.q_hat_out = q_hat;
-  cudaError_t e;
+  cudaError_t e = ensure_loaded();
+  if (e != cudaSuccess) return cuda_fail(e);
   if (from_logits) {
     PrepArgs p;
     std::memset(&p, 0, sizeof p);
@@ -198,10 +219,14 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
     r.t = no_rows();
     r.items_d = int64_t(batch->n_draft) * d.d.nch;
     r.items_t = 0;
-    if ((e = launch_rowpass(r, draft->dtype, TT_F32, s, sm_count_current())) != cudaSuccess)
+    r.err = ws.err;
+    r.epoch = next_epoch();
+    d.err = ws.err;
+    d.epoch = r.epoch;
+    if ((e = launch_rowpass(r, draft->dtype, TT_F32, s, sm_count_current(), true)) != cudaSuccess)
       return cuda_fail(e);
   }
-  if ((e = launch_decide(d, s)) != cudaSuccess) return cuda_fail(e);
+  if ((e = launch_decide(d, s, from_logits)) != cudaSuccess) return cuda_fail(e);
   return TT_OK;
 }
 
@@ -230,30 +255,34 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d,
                                   target->n_cols);
-  PrepArgs p;
-  std::memset(&p, 0, sizeof p);
-  p.B = batch->B;
-  p.n_draft = batch->n_draft;
-  p.n_target = batch->n_target;
-  p.V_t = target->n_cols;
-  p.draft_off = batch->draft_off;
-  p.target_off = batch->target_off;
-  p.target_cols = tcols;
-  p.map = map;
-  p.excl = ws.excl;
-  p.need = full_q ? ws.need_d : nullptr;
-  cudaError_t e;
-  if ((e = launch_prep(p, s)) != cudaSuccess) return cuda_fail(e);
-
+  cudaError_t e = ensure_loaded();
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (full_q) {  // the residual needs the mapped draft rows' normalisers
+    PrepArgs p;
+    std::memset(&p, 0, sizeof p);
+    p.B = batch->B;
+    p.n_draft = batch->n_draft;
+    p.n_target = batch->n_target;
+    p.draft_off = batch->draft_off;
+    p.target_off = batch->target_off;
+    p.map = map;
+    p.need = ws.need_d;
+    if ((e = launch_prep(p, s)) != cudaSuccess) return cuda_fail(e);
+  }
   RowPassArgs r;
   std::memset(&r, 0, sizeof r);
   r.t = rowset(target, ws.part_t, nullptr, prm->temp_target);
   r.items_t = (int64_t(batch->n_target) + batch->B) * r.t.nch;
   r.d = full_q ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
   r.items_d = full_q ? int64_t(batch->n_draft) * r.d.nch : 0;
-  r.excl = ws.excl;
+  r.B = batch->B;
+  r.n_target = batch->n_target;
+  r.target_off = batch->target_off;
+  r.target_cols = tcols;
+  r.err = ws.err;
+  r.epoch = next_epoch();
   if ((e = launch_rowpass(r, full_q ? draft->dtype : TT_F32, target->dtype, s,
-                          sm_count_current())) != cudaSuccess)
+                          sm_count_current(), true)) != cudaSuccess)
     return cuda_fail(e);
 
   DecideArgs d;
@@ -279,7 +308,9 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   d.status = status;
   d.p_hat = p_hat;
   d.lse = lse;
-  if ((e = launch_decide(d, s)) != cudaSuccess) return cuda_fail(e);
+  d.err = ws.err;
+  d.epoch = r.epoch;
+  if ((e = launch_decide(d, s, true)) != cudaSuccess) return cuda_fail(e);
   return TT_OK;
 }
 
@@ -319,11 +350,9 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   a.map = map;
   a.status = out->status;
   a.need = from_logits ? ws.need_d : nullptr;
-  a.target_cols = tcols;
-  a.V_t = target->n_cols;
-  a.excl = ws.excl;
 
-  cudaError_t e;
+  cudaError_t e = ensure_loaded();
+  if (e != cudaSuccess) return cuda_fail(e);
   record(prm, 0, s);
   if ((e = launch_align(a, s)) != cudaSuccess) return cuda_fail(e);
   record(prm, 1, s);
@@ -334,9 +363,17 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   r.items_t = (int64_t(batch->n_target) + batch->B) * r.t.nch;
   r.d = from_logits ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
   r.items_d = from_logits ? int64_t(batch->n_draft) * r.d.nch : 0;
-  r.excl = ws.excl;
+  r.B = batch->B;
+  r.n_target = batch->n_target;
+  r.target_off = batch->target_off;
+  r.target_cols = tcols;
+  r.err = ws.err;
+  r.epoch = next_epoch();
+  // programmatic dependent launch: target rows stream while the alignment runs
+  // (unless stage events sit between the kernels)
+  const bool pdl = prm->events == nullptr;
   if ((e = launch_rowpass(r, from_logits ? draft->dtype : TT_F32, target->dtype, s,
-                          sm_count_current())) != cudaSuccess)
+                          sm_count_current(), pdl)) != cudaSuccess)
     return cuda_fail(e);
   record(prm, 2, s);
 
@@ -367,7 +404,9 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   d.q_hat_out = out->q_hat;
   d.p_hat = out->p_hat;
   d.lse = out->lse;
-  if ((e = launch_decide(d, s)) != cudaSuccess) return cuda_fail(e);
+  d.err = ws.err;
+  d.epoch = r.epoch;
+  if ((e = launch_decide(d, s, pdl)) != cudaSuccess) return cuda_fail(e);
   record(prm, 3, s);
   return TT_OK;
 }

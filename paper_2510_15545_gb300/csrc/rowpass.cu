@@ -1,13 +1,19 @@
-// rowpass.cu -- one streaming pass over logits rows: per row chunk of kChunk
-// elements, the maximum m of s_x = z_x * log2(e) / T and the sum of 2^(s_x - m).
+// rowpass.cu -- one streaming pass over logits rows: per chunk of kChunk
+// columns, the maximum m of s_x = z_x * log2(e) / T and the sum of 2^(s_x - m).
 //
-// These partials are everything the softmax normalisers of Alg. 2 / Alg. 4
-// need (log2 sum_x 2^s_x = M + log2 sum_c s_c 2^(m_c - M)), and they double as
-// the coarse level of the residual inverse CDF, so every logit is read from HBM
-// exactly once. Draft rows that no target position maps to are skipped.
+// These partials are all the softmax normalisers of Alg. 2 / Alg. 4 need
+// (log2 sum_x 2^s_x = M + log2 sum_c s_c 2^(m_c - M)) and they are the coarse
+// level of the residual's inverse CDF, so every logit is read from HBM once.
 // Target row j < m leaves its scored token t_j out of the sum; the decision
-// kernel adds that one term back exactly (no cancellation when the residual
-// removes it).
+// kernel adds that one term back exactly. Draft rows that no target position
+// maps to are skipped.
+//
+// Warp-specialised pipeline, several CTAs per SM: one producer lane streams
+// chunks into a ring of shared-memory stages with 1-D bulk copies
+// (cp.async.bulk, completion counted on an mbarrier per stage); each of the 8
+// consumer warps owns every 8th stage, reduces one whole chunk at a time from
+// shared memory (no block barrier) and frees the stage. Every wait is bounded in time; on timeout the kernel sets
+// an error word that the decision kernel turns into a per-request status.
 #include <algorithm>
 #include <cstdint>
 
@@ -18,169 +24,367 @@ namespace tt {
 
 namespace {
 
-template <int DT>
-struct Vec;
-template <>
-struct Vec<TT_F32> {
-  static constexpr int kElems = 4;
-  static constexpr uint32_t kNegInf = 0xff800000u;
-};
-template <>
-struct Vec<TT_BF16> {
-  static constexpr int kElems = 8;
-  static constexpr uint32_t kNegInf = 0xff80ff80u;  // two bf16 -inf
+constexpr int kConsumerWarps = 8;
+constexpr int kThreads = (kConsumerWarps + 1) * 32;
+constexpr int kRingBytes = 64 * 1024;  // three CTAs per SM fit
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
+
+struct Desc {
+  int64_t row;    // < 0: no more work for this consumer warp
+  int32_t chunk;
+  int32_t n;      // columns in the chunk
+  int32_t n_smem; // leading columns delivered by the bulk copy (rest read directly)
+  int32_t excl;   // column (within the row) left out of the sum, -1 = none
+  int32_t set;    // 0 draft rows, 1 target rows
+  int32_t pad;
 };
 
-template <int DT>
-__device__ __forceinline__ float elem(const uint4& v, int q) {
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-  if constexpr (DT == TT_F32) {
-    return __uint_as_float(w[q]);
-  } else {
-    const uint32_t x = w[q >> 1];
-    return __uint_as_float((q & 1) ? (x & 0xffff0000u) : (x << 16));
+// Stage s is always refilled for the same consumer warp (s mod kConsumerWarps),
+// so a warp never waits on a stage more than one phase ahead of it: an
+// mbarrier parity wait cannot tell phase n from phase n + 2.
+template <int DTD, int DTT>
+struct Ring {
+  static constexpr int kEsz = (DTD == TT_F32 || DTT == TT_F32) ? 4 : 2;
+  static constexpr int kStageBytes = kChunk * kEsz;
+  static constexpr int kStages = kRingBytes / kStageBytes;
+  static constexpr size_t kSmem = size_t(kRingBytes) + kStages * (2 * sizeof(uint64_t) + sizeof(Desc));
+  static_assert(kStages % kConsumerWarps == 0, "each stage belongs to one consumer warp");
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Waits for the phase of the given parity to complete; false after kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t i = 1; i < (1u << 30); ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63) == 0 && global_ns() - t0 > kWaitLimitNs) return false;
   }
+  return false;
+}
+__device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32_t bytes,
+                                              uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
-// Replaces element q (0..VEC-1) of a vector by raw bits, with selects only
-// (no dynamic register indexing).
+// Scored column of target row r (-1 for a bonus row or an unusable entry):
+// request b owns rows target_off[b] + b .. target_off[b+1] + b.
+__device__ int target_excl(const RowPassArgs& a, int64_t r) {
+  if (!a.target_off || a.B <= 0) return -1;
+  int lo = 0, hi = a.B - 1;
+  while (lo < hi) {  // largest b with target_off[b] + b <= r
+    const int mid = (lo + hi + 1) >> 1;
+    if (int64_t(a.target_off[mid]) + mid <= r) lo = mid;
+    else hi = mid - 1;
+  }
+  const int b = lo;
+  const int t0 = a.target_off[b], t1 = a.target_off[b + 1];
+  if (t0 < 0 || t1 < t0 || t1 > a.n_target) return -1;
+  const int64_t j = r - (int64_t(t0) + b);
+  if (j < 0 || j >= t1 - t0) return -1;
+  const int c = a.target_cols[t0 + j];
+  return (c >= 0 && c < a.t.V) ? c : -1;
+}
+
 template <int DT>
-__device__ __forceinline__ void set_elem_bits(uint4& v, int q, uint32_t bits) {
+__device__ __forceinline__ float lane_elem(const uint4& v, int q) {
   if constexpr (DT == TT_F32) {
-    v.x = q == 0 ? bits : v.x;
-    v.y = q == 1 ? bits : v.y;
-    v.z = q == 2 ? bits : v.z;
-    v.w = q == 3 ? bits : v.w;
+    return __uint_as_float(q == 0 ? v.x : q == 1 ? v.y : q == 2 ? v.z : v.w);
   } else {
     const int h = q >> 1;
-    const bool high = (q & 1) != 0;
-    auto upd = [&](uint32_t x) {
-      return high ? ((x & 0x0000ffffu) | (bits << 16)) : ((x & 0xffff0000u) | (bits & 0xffffu));
-    };
-    v.x = h == 0 ? upd(v.x) : v.x;
-    v.y = h == 1 ? upd(v.y) : v.y;
-    v.z = h == 2 ? upd(v.z) : v.z;
-    v.w = h == 3 ? upd(v.w) : v.w;
+    const uint32_t w = h == 0 ? v.x : h == 1 ? v.y : h == 2 ? v.z : v.w;
+    return __uint_as_float((q & 1) ? (w & 0xffff0000u) : (w << 16));
+  }
+}
+
+// One consumer warp reduces one chunk held in shared memory (plus a ragged
+// tail of fewer than 16 bytes read directly) to (max, sum of 2^(s - max)).
+// The stage is read twice (max, then sum) rather than held in registers.
+template <int DT, bool PLAIN>
+__device__ __forceinline__ void reduce_stage(const uint4* sv, const Desc& d, float scale,
+                                             int lane, float& mx, float& sum) {
+  constexpr int VEC = DT == TT_F32 ? 4 : 8;  // elements per 16 bytes
+  constexpr int NV = kChunk / (VEC * 32);    // 16-byte vectors per lane
+#pragma unroll 4
+  for (int v = 0; v < NV; ++v) {
+    const uint4 w = sv[v * 32 + lane];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) {
+      const int e = (v * 32 + lane) * VEC + q;
+      if (PLAIN || (e < d.n_smem && e != d.excl)) mx = fmaxf(mx, lane_elem<DT>(w, q) * scale);
+    }
+  }
+  if (mx == -INFINITY) return;
+#pragma unroll 4
+  for (int v = 0; v < NV; ++v) {
+    const uint4 w = sv[v * 32 + lane];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) {
+      const int e = (v * 32 + lane) * VEC + q;
+      if (PLAIN || (e < d.n_smem && e != d.excl))
+        sum += ex2_approx(fmaf(lane_elem<DT>(w, q), scale, -mx));
+    }
   }
 }
 
 template <int DT>
-__device__ __forceinline__ void process_chunk(const RowSet& S, int64_t r, int c, int excl_col,
-                                              float* red_m, float* red_s) {
-  constexpr int VEC = Vec<DT>::kElems;
-  constexpr int NV = kChunk / (VEC * kRowThreads);
-  constexpr int ESZ = DT == TT_F32 ? 4 : 2;
-  const int tid = threadIdx.x;
-  const char* row = S.data + r * S.stride_bytes;
-  const int c0 = c * kChunk;
-  const int n = min(kChunk, S.V - c0);
-
-  uint4 buf[NV];
-#pragma unroll
-  for (int v = 0; v < NV; ++v) {
-    const int e = (v * kRowThreads + tid) * VEC;
-    if (e + VEC <= n) {
-      buf[v] = ld_stream_v4(row + size_t(c0 + e) * ESZ);
-    } else {
-      buf[v] = make_uint4(Vec<DT>::kNegInf, Vec<DT>::kNegInf, Vec<DT>::kNegInf,
-                          Vec<DT>::kNegInf);
-#pragma unroll
-      for (int q = 0; q < VEC; ++q) {  // ragged tail of the row
-        if (e + q < n) {
-          const uint32_t bits = DT == TT_F32
-              ? __ldg(reinterpret_cast<const unsigned int*>(row) + c0 + e + q)
-              : uint32_t(__ldg(reinterpret_cast<const unsigned short*>(row) + c0 + e + q));
-          set_elem_bits<DT>(buf[v], q, bits);
-        }
-      }
-    }
-  }
-  const int ex = excl_col - c0;  // the scored token leaves the sum
-  if (ex >= 0 && ex < n) {
-#pragma unroll
-    for (int v = 0; v < NV; ++v) {
-      const int e = (v * kRowThreads + tid) * VEC;
-      if (ex >= e && ex < e + VEC)
-        set_elem_bits<DT>(buf[v], ex - e, DT == TT_F32 ? 0xff800000u : 0xff80u);
-    }
-  }
-
+__device__ __forceinline__ void reduce_chunk(const char* stage, const Desc& d, const RowSet& S,
+                                             int lane, float& m_out, float& s_out) {
+  const uint4* sv = reinterpret_cast<const uint4*>(stage);
   const float scale = S.scale;
-  float mx = -INFINITY;
-#pragma unroll
-  for (int v = 0; v < NV; ++v)
-#pragma unroll
-    for (int q = 0; q < VEC; ++q) mx = fmaxf(mx, elem<DT>(buf[v], q) * scale);
-  float sum = 0.f;
-  if (mx != -INFINITY) {
-#pragma unroll
-    for (int v = 0; v < NV; ++v)
-#pragma unroll
-      for (int q = 0; q < VEC; ++q) sum += ex2_approx(fmaf(elem<DT>(buf[v], q), scale, -mx));
+  // ragged tail: at most 7 columns beyond the bulk copy, one per lane
+  float ztail = -INFINITY;
+  const int tail = d.n - d.n_smem;
+  if (lane < tail) {
+    const int e = d.n_smem + lane;
+    if (e != d.excl) {
+      const char* row = S.data + d.row * S.stride_bytes;
+      ztail = load_logit<DT>(row, int64_t(d.chunk) * kChunk + e) * scale;
+    }
   }
-  warp_merge_ms(mx, sum);
-  const int warp = tid >> 5, lane = tid & 31;
-  if (lane == 0) {
-    red_m[warp] = mx;
-    red_s[warp] = sum;
+  float mx = ztail, sum = 0.f;
+  if (d.n_smem == kChunk && d.excl < 0) {
+    reduce_stage<DT, true>(sv, d, scale, lane, mx, sum);
+  } else {
+    reduce_stage<DT, false>(sv, d, scale, lane, mx, sum);
+  }
+  if (ztail != -INFINITY) sum += ex2_approx(ztail - mx);
+  m_out = mx;
+  s_out = sum;
+}
+
+template <int DTD, int DTT>
+__global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
+  using R = Ring<DTD, DTT>;
+  extern __shared__ __align__(128) char smem[];
+  char* stages = smem;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kRingBytes);
+  uint64_t* empty = full + R::kStages;
+  Desc* desc = reinterpret_cast<Desc*>(empty + R::kStages);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < R::kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
-  if (warp == 0) {
-    float m2 = lane < kRowThreads / 32 ? red_m[lane] : -INFINITY;
-    float s2 = lane < kRowThreads / 32 ? red_s[lane] : 0.f;
-    warp_merge_ms(m2, s2);
-    if (lane == 0) S.part[r * S.nch + c] = Partial{m2, s2};
-  }
-}
 
-template <int DTD, int DTT>
-__global__ void __launch_bounds__(kRowThreads) rowpass_kernel(RowPassArgs a) {
-  __shared__ float red_m[2][kRowThreads / 32];
-  __shared__ float red_s[2][kRowThreads / 32];
-  const int64_t total = a.items_t + a.items_d;
-  int it = 0;
-  // target items first: they do not depend on the alignment
-  for (int64_t item = blockIdx.x; item < total; item += gridDim.x) {
-    if (item < a.items_t) {
-      const int64_t r = item / a.t.nch;
-      const int c = int(item - r * a.t.nch);
-      const int excl = a.excl ? a.excl[r] : -1;
-      process_chunk<DTT>(a.t, r, c, excl, red_m[it & 1], red_s[it & 1]);
-    } else {
-      const int64_t di = item - a.items_t;
-      const int64_t r = di / a.d.nch;
-      const int c = int(di - r * a.d.nch);
-      if (a.d.need && !a.d.need[r]) continue;
-      process_chunk<DTD>(a.d, r, c, -1, red_m[it & 1], red_s[it & 1]);
+  if (warp == kConsumerWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      // this CTA's share: a block of target items, then a block of draft items
+      const int64_t G = gridDim.x, g = blockIdx.x;
+      const int64_t t_lo = a.items_t * g / G, t_hi = a.items_t * (g + 1) / G;
+      const int64_t d_lo = a.items_d * g / G, d_hi = a.items_d * (g + 1) / G;
+      bool ok = true, waited = false;
+      int it = 0;
+      int64_t cached_row = -1;
+      int cached_excl = -1;
+      for (int64_t item = t_lo; ok && item < t_hi + (d_hi - d_lo); ++item) {
+        Desc d;
+        const RowSet* S;
+        int esz;
+        if (item < t_hi) {
+          S = &a.t;
+          esz = DTT == TT_F32 ? 4 : 2;
+          d.row = item / a.t.nch;
+          d.chunk = int(item - d.row * a.t.nch);
+          d.set = 1;
+          if (d.row != cached_row) {
+            cached_row = d.row;
+            cached_excl = a.excl ? a.excl[d.row] : target_excl(a, d.row);
+          }
+          const int ex = cached_excl - d.chunk * kChunk;
+          d.excl = (cached_excl >= 0 && ex >= 0 && ex < kChunk) ? ex : -1;
+        } else {
+          if (!waited) {  // draft rows need the alignment's flags
+            grid_dependency_wait();
+            waited = true;
+          }
+          const int64_t di = d_lo + (item - t_hi);
+          S = &a.d;
+          esz = DTD == TT_F32 ? 4 : 2;
+          d.row = di / a.d.nch;
+          d.chunk = int(di - d.row * a.d.nch);
+          d.set = 0;
+          d.excl = -1;
+          if (a.d.need && !a.d.need[d.row]) continue;
+        }
+        const int c0 = d.chunk * kChunk;
+        d.n = min(kChunk, S->V - c0);
+        const uint32_t bytes = uint32_t(d.n * esz) & ~15u;  // bulk copies move 16-byte units
+        d.n_smem = int(bytes) / esz;
+        const int s = it % R::kStages;
+        const uint32_t par = ((it / R::kStages) & 1) ^ 1;
+        if (!mbar_wait(&empty[s], par)) {
+          report_error(a.err, a.epoch, TT_REQ_TIMEOUT);
+          ok = false;
+          break;
+        }
+        // every bulk copy is checked against the tensor before it is issued
+        const char* src = S->data + d.row * S->stride_bytes + size_t(c0) * esz;
+        const bool copy_ok = d.row >= 0 && d.row < S->n_rows && c0 >= 0 && d.n > 0 &&
+                             (reinterpret_cast<uintptr_t>(src) & 15) == 0 &&
+                             bytes <= uint32_t(R::kStageBytes);
+        if (!copy_ok) {
+          report_error(a.err, a.epoch, TT_REQ_INTERNAL);
+          d.n = 0;
+          d.n_smem = 0;
+        }
+        desc[s] = d;
+        if (copy_ok && bytes > 0) {
+          mbar_arrive_expect_tx(&full[s], bytes);
+          bulk_copy_g2s(stages + size_t(s) * R::kStageBytes, src, bytes, &full[s]);
+        } else {
+          mbar_arrive(&full[s]);
+        }
+        ++it;
+      }
+      if (!waited) grid_dependency_wait();  // this grid ends after the one before it
+      // one end marker per consumer warp
+      for (int w = 0; ok && w < kConsumerWarps; ++w) {
+        const int s = it % R::kStages;
+        const uint32_t par = ((it / R::kStages) & 1) ^ 1;
+        if (!mbar_wait(&empty[s], par)) {
+          report_error(a.err, a.epoch, TT_REQ_TIMEOUT);
+          ok = false;
+          break;
+        }
+        desc[s].row = -1;
+        mbar_arrive(&full[s]);
+        ++it;
+      }
+      grid_launch_dependents();
     }
-    ++it;
+    return;
+  }
+
+  // -------------------------------------------------------------- consumers
+  for (int it = warp;; it += kConsumerWarps) {
+    const int s = it % R::kStages;
+    const uint32_t par = (it / R::kStages) & 1;
+    if (!mbar_wait(&full[s], par)) {
+      if (lane == 0) report_error(a.err, a.epoch, TT_REQ_TIMEOUT);
+      break;
+    }
+    const Desc d = desc[s];
+    if (d.row < 0) break;
+    const char* stage = stages + size_t(s) * R::kStageBytes;
+    float m, sum;
+    if (d.set) {
+      reduce_chunk<DTT>(stage, d, a.t, lane, m, sum);
+    } else {
+      reduce_chunk<DTD>(stage, d, a.d, lane, m, sum);
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[s]);  // the stage's bytes are consumed
+    warp_merge_ms(m, sum);
+    if (lane == 0) {
+      const RowSet& S = d.set ? a.t : a.d;
+      S.part[d.row * S.nch + d.chunk] = Partial{m, sum};
+    }
   }
 }
 
 template <int DTD, int DTT>
-cudaError_t launch_rowpass_t(const RowPassArgs& a, cudaStream_t stream, int sm_count) {
+int& resident_per_sm() {
   static int per_sm = 0;
-  if (per_sm == 0) {
-    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &per_sm, rowpass_kernel<DTD, DTT>, kRowThreads, 0);
-    if (e != cudaSuccess) return e;
-    if (per_sm < 1) per_sm = 1;
-  }
+  return per_sm;
+}
+
+template <int DTD, int DTT>
+cudaError_t preload_t() {
+  using R = Ring<DTD, DTT>;
+  cudaError_t e = cudaFuncSetAttribute(rowpass_kernel<DTD, DTT>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(R::kSmem));
+  if (e != cudaSuccess) return e;
+  int per_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rowpass_kernel<DTD, DTT>, kThreads,
+                                                    R::kSmem);
+  if (e != cudaSuccess) return e;
+  resident_per_sm<DTD, DTT>() = per_sm < 1 ? 1 : per_sm;
+  return cudaSuccess;
+}
+
+template <int DTD, int DTT>
+cudaError_t launch_rowpass_t(const RowPassArgs& a, cudaStream_t stream, int sm_count, bool pdl) {
+  using R = Ring<DTD, DTT>;
+  const int per_sm = resident_per_sm<DTD, DTT>();
+  if (per_sm == 0) return cudaErrorNotReady;  // preload_rowpass() was not called
   const int64_t total = a.items_t + a.items_d;
   if (total == 0) return cudaSuccess;
   const int64_t grid = std::min<int64_t>(total, int64_t(sm_count) * per_sm);
-  rowpass_kernel<DTD, DTT><<<unsigned(grid), kRowThreads, 0, stream>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(grid));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = R::kSmem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, rowpass_kernel<DTD, DTT>, a);
 }
 
 }  // namespace
 
+cudaError_t preload_rowpass() {
+  cudaError_t e;
+  if ((e = preload_t<TT_F32, TT_F32>()) != cudaSuccess) return e;
+  if ((e = preload_t<TT_F32, TT_BF16>()) != cudaSuccess) return e;
+  if ((e = preload_t<TT_BF16, TT_F32>()) != cudaSuccess) return e;
+  return preload_t<TT_BF16, TT_BF16>();
+}
+
 cudaError_t launch_rowpass(const RowPassArgs& a, int dt_d, int dt_t, cudaStream_t stream,
-                           int sm_count) {
-  if (dt_d == TT_F32 && dt_t == TT_F32) return launch_rowpass_t<TT_F32, TT_F32>(a, stream, sm_count);
-  if (dt_d == TT_F32 && dt_t == TT_BF16) return launch_rowpass_t<TT_F32, TT_BF16>(a, stream, sm_count);
-  if (dt_d == TT_BF16 && dt_t == TT_F32) return launch_rowpass_t<TT_BF16, TT_F32>(a, stream, sm_count);
-  return launch_rowpass_t<TT_BF16, TT_BF16>(a, stream, sm_count);
+                           int sm_count, bool pdl) {
+  if (dt_d == TT_F32 && dt_t == TT_F32) return launch_rowpass_t<TT_F32, TT_F32>(a, stream, sm_count, pdl);
+  if (dt_d == TT_F32 && dt_t == TT_BF16) return launch_rowpass_t<TT_F32, TT_BF16>(a, stream, sm_count, pdl);
+  if (dt_d == TT_BF16 && dt_t == TT_F32) return launch_rowpass_t<TT_BF16, TT_F32>(a, stream, sm_count, pdl);
+  return launch_rowpass_t<TT_BF16, TT_BF16>(a, stream, sm_count, pdl);
 }
 
 }  // namespace tt

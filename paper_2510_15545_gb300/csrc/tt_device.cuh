@@ -5,11 +5,11 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
-#include "../../include/tt.h"
+#include "tt.h"
 
 namespace tt {
 
-constexpr int kChunk = 8192;         // logits elements per row chunk (one partial)
+constexpr int kChunk = 2048;         // logits columns per row chunk (one partial)
 constexpr int kRowThreads = 256;     // threads of the row-pass and decision blocks
 constexpr int32_t kInf = 0x3fffffff; // "infinite" accumulated DTW cost
 
@@ -34,6 +34,7 @@ struct Workspace {
   float* q_hat;      // [n_target] transferred probabilities when the caller keeps none
   int32_t* status;   // [B] per-request status between kernels
   int32_t* excl;     // [n_target + B] scored column of each target row (-1: bonus row)
+  int32_t* err;      // two words: epoch of a call whose row pass failed, and why
   size_t bytes;
 };
 
@@ -55,6 +56,7 @@ __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_d
   w.q_hat = reinterpret_cast<float*>(take(sizeof(float) * size_t(n_target)));
   w.status = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * size_t(B)));
   w.excl = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (size_t(n_target) + B)));
+  w.err = reinterpret_cast<int32_t*>(take(2 * sizeof(int32_t)));
   w.bytes = off;
   return w;
 }
@@ -167,6 +169,13 @@ __device__ __forceinline__ double philox_uniform(uint64_t seed, uint64_t pos, ui
   uint64_t c[4] = {pos, stream, request, 0};
   philox4x64_10(c, seed, 0);
   return double(c[0] >> 40) * (1.0 / 16777216.0);
+}
+
+// Records a failure of call `epoch` (TT_REQ_TIMEOUT / TT_REQ_INTERNAL bits).
+__device__ __forceinline__ void report_error(int32_t* err, int32_t epoch, int32_t bits) {
+  if (!err) return;
+  atomicOr(&err[1], bits);
+  atomicExch(&err[0], epoch);
 }
 
 // ------------------------------------------------------------ CSR helpers

@@ -5,7 +5,7 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
-#include "../../include/tt.h"
+#include "tt.h"
 
 namespace tt {
 
@@ -13,7 +13,7 @@ struct Partial;
 
 constexpr int kAlignWarpsMax = 4;             // sequence pairs per align CTA
 constexpr int kAlignSmemMax = 200 * 1024;     // dynamic shared memory cap of one align CTA
-constexpr int kMaxChunksPerRow = 256;         // rows up to 256 * 8192 = 2,097,152 columns
+constexpr int kMaxChunksPerRow = 1024;        // rows up to 1024 * 2048 = 2,097,152 columns
 
 struct AlignArgs {
   int B, n_draft, n_target, max_k, max_m, window;
@@ -28,9 +28,6 @@ struct AlignArgs {
   int32_t* map;
   int32_t* status;
   uint8_t* need;               // needed draft rows (may be NULL)
-  const int32_t* target_cols;  // with excl: columns of the scored target tokens
-  int V_t;                     // width of the target rows (excl only)
-  int32_t* excl;               // [n_target + B] scored column of each target row, -1 if none (may be NULL)
   int warps_per_block, tile_w;
   size_t smem_per_warp;
 };
@@ -42,6 +39,7 @@ struct RowSet {
   int V;
   int nch;
   float scale;  // log2(e) / T
+  int64_t n_rows;
   Partial* part;
   const uint8_t* need;  // rows to visit (NULL = all)
 };
@@ -49,7 +47,13 @@ struct RowSet {
 struct RowPassArgs {
   RowSet d, t;
   int64_t items_d, items_t;  // rows * chunks of each family (0 = family absent)
-  const int32_t* excl;       // [target rows]: column left out of the sum, -1 = none
+  const int32_t* excl;       // [target rows] column left out of the sum, or NULL: found
+                             // from target_off / target_cols
+  int B, n_target;
+  const int32_t* target_off;
+  const int32_t* target_cols;
+  int32_t* err;              // err[0] = epoch of a failed call, err[1] = its TT_REQ_* bits
+  int32_t epoch;             // identifies this call
 };
 
 struct DecideArgs {
@@ -64,6 +68,8 @@ struct DecideArgs {
   RowSet d, t;
   int dt_d, dt_t;
   const int32_t* status_in;  // status of an earlier stage (align) or NULL
+  int32_t* err;              // row-pass error words (NULL when no row pass ran)
+  int32_t epoch;
   uint64_t seed, request_base;
   int32_t* accepted;
   int32_t* next_token;
@@ -74,21 +80,25 @@ struct DecideArgs {
 };
 
 struct PrepArgs {
-  int B, n_draft, n_target, V_t;
+  int B, n_draft, n_target;
   const int32_t* draft_off;
   const int32_t* target_off;
-  const int32_t* target_cols;
   const int32_t* map;
-  uint8_t* need;   // written from map when not NULL
-  int32_t* excl;   // written from target_cols when not NULL
+  uint8_t* need;   // needed-draft-row flags, written from map
 };
 
 size_t align_smem_per_warp(int max_k, int max_m, int tile_w);
 int align_tile_width(int max_k, int max_m, int window);
 cudaError_t launch_align(const AlignArgs& args, cudaStream_t stream);
 cudaError_t launch_rowpass(const RowPassArgs& args, int dt_d, int dt_t, cudaStream_t stream,
-                           int sm_count);
-cudaError_t launch_decide(const DecideArgs& args, cudaStream_t stream);
+                           int sm_count, bool pdl);
+cudaError_t launch_decide(const DecideArgs& args, cudaStream_t stream, bool pdl);
 cudaError_t launch_prep(const PrepArgs& args, cudaStream_t stream);
+
+// Loads every kernel of the library on the current device and sets its launch
+// attributes, so that no module is loaded lazily inside a dependent-launch chain.
+cudaError_t preload_align();
+cudaError_t preload_rowpass();
+cudaError_t preload_decide();
 
 }  // namespace tt
