@@ -168,13 +168,12 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
       if (j < m) {  // add back the scored token's term, left out by the row pass
         const double x = double(zt) * double(a.t.scale);
         const float Mx = fmaxf(M, float(x));
-        S = (M == -INFINITY ? 0.0 : S * exp2(double(M) - double(Mx))) + exp2(x - double(Mx));
+        S = (M == -INFINITY ? 0.0 : S * exp2_split(double(M) - double(Mx))) +
+            exp2_split(x - double(Mx));
         M = Mx;
-        lse2 = double(M) + log2(S);
-        ph = exp2(x - lse2);
-      } else {
-        lse2 = double(M) + log2(S);
+        ph = exp2_split(x - double(M)) * double(__frcp_rn(float(S)));
       }
+      lse2 = double(M) + log2_split(S);
       if (!isfinite(lse2)) nonfinite = 1;
       if (lane == 0) {
         s_M[j] = M;
@@ -193,9 +192,10 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
       float M;
       double S;
       row_norm_warp(a.d.part + row * a.d.nch, a.d.nch, lane, M, S);
-      const double lse2 = double(M) + log2(S);
-      if (!isfinite(lse2)) nonfinite = 1;
-      if (lane == 0) s_q[j] = exp2(double(zd) * double(a.d.scale) - lse2);
+      if (!(S > 0.0) || !isfinite(S) || M == -INFINITY) nonfinite = 1;
+      if (lane == 0)
+        s_q[j] = exp2_split(double(zd) * double(a.d.scale) - double(M)) *
+                 double(__frcp_rn(float(S)));
     }
   }
   if (__syncthreads_or(nonfinite)) {
@@ -228,11 +228,9 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
 
   // ------------------------- accept: u_j < min(1, p/q), first failure stops
   const uint64_t req = a.request_base + uint64_t(b);
-  if (tid < m) {
+  if (tid < m) {  // for u < 1, u < min(1, p/q) holds exactly when u q < p
     const double u = philox_uniform(a.seed, uint64_t(tid), 0, req);
-    const double p = s_p[tid], q = s_q[tid];
-    const double ratio = q > 0.0 ? p / q : (p > 0.0 ? INFINITY : 0.0);
-    if (!(u < fmin(1.0, ratio))) atomicMin(&s_a, tid);
+    if (!(u * s_q[tid] < s_p[tid])) atomicMin(&s_a, tid);
   }
   __syncthreads();
   const int acc = s_a;
@@ -240,7 +238,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
   const int col_t = acc < m ? s_col[acc] : -1;
   const float Mt = s_M[acc];
   const double St = s_S[acc];
-  const float invSt = float(1.0 / St);
+  const float invSt = __frcp_rn(float(St));
   const float scale_t = a.t.scale;
   const char* trow = a.t.data + row * a.t.stride_bytes;
   const int nch = a.t.nch;
@@ -265,7 +263,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
     __syncthreads();
   }
   const float Md = s_dM;
-  const float invSd = float(1.0 / s_dS);
+  const float invSd = __frcp_rn(float(s_dS));
   const float scale_d = a.d.scale;
   // residual mass of column x (logit z) of row a in mode md, fp32
   auto r_of = [&](int x, float z, int md) -> float {
@@ -292,7 +290,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
     } else {
       for (int c = tid; c < nch; c += kDecThreads) {
         const Partial P = a.t.part[row * nch + c];
-        double R = P.m == -INFINITY ? 0.0 : double(P.s) * double(ex2_approx(P.m - Mt)) / St;
+        double R = P.m == -INFINITY ? 0.0 : double(P.s * ex2_approx(P.m - Mt) * invSt);
         if (col_t >= 0 && col_t / kChunk == c) R += mode == 1 ? r_t : s_p[acc];
         s_R[c] = R;
       }
@@ -445,9 +443,8 @@ __global__ void __launch_bounds__(kDecThreads) transfer_kernel(DecideArgs a) {
       float M;
       double S;
       row_norm_warp(a.d.part + row * a.d.nch, a.d.nch, lane, M, S);
-      const double lse2 = double(M) + log2(S);
-      if (!isfinite(lse2)) nonfinite = 1;
-      qh = exp2(double(zd) * double(a.d.scale) - lse2);
+      if (!(S > 0.0) || !isfinite(S) || M == -INFINITY) nonfinite = 1;
+      qh = exp2_split(double(zd) * double(a.d.scale) - double(M)) * double(__frcp_rn(float(S)));
     }
     if (lane == 0) s_q[j] = qh;
   }

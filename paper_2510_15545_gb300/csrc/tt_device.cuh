@@ -126,21 +126,62 @@ __device__ __forceinline__ float warp_max_f(float v) {
 
 // Log2-normaliser of a row from its chunk partials, computed by one warp:
 // returns (M, S) with sum over the row of 2^(s_x - M) = S (excluding what the
-// partials exclude). S accumulates in fp64.
+// partials exclude). S accumulates in fp64. Rows of up to 128 chunks are read
+// once (four partials per lane held in registers).
 __device__ __forceinline__ void row_norm_warp(const Partial* part, int nch, int lane, float& M,
                                               double& S) {
   float mx = -INFINITY;
-  for (int c = lane; c < nch; c += 32) mx = fmaxf(mx, part[c].m);
-  mx = warp_max_f(mx);
   double acc = 0.0;
-  if (mx != -INFINITY) {
-    for (int c = lane; c < nch; c += 32) {
-      Partial p = part[c];
-      if (p.m != -INFINITY) acc += double(p.s) * double(ex2_approx(p.m - mx));
+  if (nch <= 128) {
+    Partial p[4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int c = lane + 32 * r;
+      p[r] = c < nch ? part[c] : Partial{-INFINITY, 0.f};
+      mx = fmaxf(mx, p[r].m);
+    }
+    mx = warp_max_f(mx);
+    if (mx != -INFINITY) {
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+        if (p[r].m != -INFINITY) acc += double(p[r].s) * double(ex2_approx(p[r].m - mx));
+    }
+  } else {
+    for (int c = lane; c < nch; c += 32) mx = fmaxf(mx, part[c].m);
+    mx = warp_max_f(mx);
+    if (mx != -INFINITY) {
+      for (int c = lane; c < nch; c += 32) {
+        const Partial q = part[c];
+        if (q.m != -INFINITY) acc += double(q.s) * double(ex2_approx(q.m - mx));
+      }
     }
   }
   M = mx;
   S = warp_sum_d(acc);
+}
+
+__device__ __forceinline__ float lg2_approx(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// 2^y for an fp64 exponent: the split y = n + f (n integer, |f| <= 1/2) is
+// exact, 2^f comes from the SFU (relative error about 2^-22) and 2^n is built
+// from its exponent bits. Below 2^-1020 the result is 0.
+__device__ __forceinline__ double exp2_split(double y) {
+  if (!(y > -1020.0)) return 0.0;
+  const double n = rint(y);
+  const int ni = int(n);
+  const double scale = __hiloint2double((ni + 1023) << 20, 0);
+  return double(ex2_approx(float(y - n))) * scale;
+}
+
+// log2 of a positive fp64 value: exponent exactly, mantissa from the SFU.
+__device__ __forceinline__ double log2_split(double v) {
+  int e;
+  const double m = frexp(v, &e);  // v = m * 2^e, m in [1/2, 1)
+  return double(e) + double(lg2_approx(float(m)));
 }
 
 // ----------------------------------------------------------------- Philox
