@@ -191,6 +191,37 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
                   const tt_params* prm, void* workspace, size_t workspace_bytes,
                   const tt_step_out* out, void* stream);
 
+/* Device scratch, in bytes, that the library keeps for tt_step_noalloc. */
+#define TT_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+/* tt_step for callers that cannot allocate device memory. (The paper has no
+ * counterpart: this is a deployment aid of this library.)
+ * Some callers cannot call cudaMalloc or any other allocating routine where they
+ * run a verification step: runtimes whose device memory is owned by one arena
+ * that must not be bypassed, serving loops that must not stall on the
+ * allocator (cudaMalloc can synchronise the device), or foreign-language hosts
+ * that only hand over input and output buffers. Such callers cannot provide the
+ * `workspace` of tt_step. This entry point takes the same arguments minus the
+ * workspace and uses a fixed scratch array of TT_NOALLOC_SCRATCH_BYTES (16 MiB)
+ * compiled into the library: every GPU that loads the library holds those
+ * 16 MiB until the process exits. It allocates nothing.
+ *  - Batches that need more scratch than that (tt_workspace_bytes) are refused
+ *    with TT_ERR_UNSUPPORTED before anything touches the GPU; the five
+ *    workloads the library is measured on all fit.
+ *  - The first call on each device looks up the array's device address there
+ *    (cudaGetSymbolAddress, with that device current); make that first call
+ *    before any stream capture.
+ *  - Every call on a device shares the one array, which keeps the last call's
+ *    contents; each call clears the two words that must start at zero (the
+ *    row pass's error report) on `stream`, and writes every other scratch
+ *    value before reading it. Calls whose work overlaps on the GPU (two
+ *    streams, or two host threads) race on the array: order them.
+ * Results equal tt_step's for the same arguments. */
+tt_status tt_step_noalloc(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
+                          const tt_logits* draft, const float* draft_probs,
+                          const tt_logits* target, const tt_params* prm,
+                          const tt_step_out* out, void* stream);
+
 /* Static text for a tt_status. */
 const char* tt_status_string(tt_status s);
 

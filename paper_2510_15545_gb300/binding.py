@@ -58,7 +58,8 @@ class _StepOut(ctypes.Structure):
 
 _lib = None
 EXPORTS = ("tt_workspace_bytes", "tt_align", "tt_transfer", "tt_verify", "tt_step",
-           "tt_status_string", "tt_last_cuda_error", "tt_version")
+           "tt_step_noalloc", "tt_status_string", "tt_last_cuda_error", "tt_version")
+TT_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
 def lib_path() -> str:
@@ -92,6 +93,9 @@ def load(build_if_missing: bool = False):
     L.tt_step.argtypes = [P(_Batch), P(_Vocab), P(_Vocab), P(_Logits), c_p, P(_Logits),
                           P(_Params), c_p, ctypes.c_size_t, P(_StepOut), c_p]
     L.tt_step.restype = c_i32
+    L.tt_step_noalloc.argtypes = [P(_Batch), P(_Vocab), P(_Vocab), P(_Logits), c_p, P(_Logits),
+                                  P(_Params), P(_StepOut), c_p]
+    L.tt_step_noalloc.restype = c_i32
     L.tt_status_string.argtypes = [c_i32]
     L.tt_status_string.restype = ctypes.c_char_p
     L.tt_last_cuda_error.argtypes = []
@@ -365,6 +369,27 @@ def tt_step(batch: Batch, vd: VocabTable, vt: VocabTable, draft_logits, target_l
             params: Params, *, draft_probs=None, ws=None, out=None, stream=None) -> dict:
     return StepCall(batch, vd, vt, draft_logits, target_logits, params, draft_probs=draft_probs,
                     ws=ws, out=out, stream=stream)()
+
+
+def tt_step_noalloc(batch: Batch, vd: VocabTable, vt: VocabTable, draft_logits, target_logits,
+                    params: Params, *, draft_probs=None, out=None, stream=None) -> dict:
+    """tt_step without a workspace, for callers that cannot allocate device
+    memory: the library's own fixed scratch (TT_NOALLOC_SCRATCH_BYTES per GPU)
+    is used instead. Outputs are the caller's (allocated here only when not
+    given). Calls that overlap on the GPU share that scratch and must be ordered."""
+    dev = batch.target_off.device
+    o = out if out is not None else step_outputs(batch, dev)
+    keep = []
+    Ld, Lt = _logits(draft_logits), _logits(target_logits)
+    so = _StepOut(*[_ptr(o.get(k)) for k in STEP_OUTPUTS])
+    code = load().tt_step_noalloc(ctypes.byref(batch._c()), ctypes.byref(vd._c()),
+                                  ctypes.byref(vt._c()),
+                                  ctypes.byref(Ld) if Ld is not None else None,
+                                  _ptr(draft_probs), ctypes.byref(Lt),
+                                  ctypes.byref(params._c(keep)), ctypes.byref(so),
+                                  _stream(stream))
+    _check("tt_step_noalloc", code)
+    return o
 
 
 def tt_status_string(code: int) -> str:
