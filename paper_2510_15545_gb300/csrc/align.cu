@@ -106,6 +106,8 @@ __global__ void __launch_bounds__(kAlignWarpsMax * 32)
   // the row pass may start streaming target rows now; it waits for this grid
   // before it reads the needed-draft-row flags
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (a.work && blockIdx.x == 0 && threadIdx.x < kWorkShards)
+    a.work[threadIdx.x * kWorkStride] = 0ull;  // read after this grid ends
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * a.warps_per_block + warp;
   if (b >= a.B) return;
@@ -122,6 +124,9 @@ __global__ void __launch_bounds__(kAlignWarpsMax * 32)
   }
   const int d0 = a.draft_off[b], k = a.draft_off[b + 1] - d0;
   const int t0 = a.target_off[b], m = a.target_off[b + 1] - t0;
+  if (a.excl)  // the row pass leaves these columns out of its sums
+    for (int j = lane; j <= m; j += 32)
+      a.excl[int64_t(t0) + b + j] = j < m ? a.target_cols[t0 + j] : -1;
   int st = 0;
   if (k == 0 || m == 0) st |= TT_REQ_EMPTY;
   if (k > K || m > M || k > TT_MAX_K || m > TT_MAX_M) st |= TT_REQ_TOO_LONG;

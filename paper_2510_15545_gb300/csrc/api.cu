@@ -212,15 +212,17 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
     p.target_off = batch->target_off;
     p.map = map;
     p.need = ws.need_d;
+    p.work = ws.work;
     if ((e = launch_prep(p, s)) != cudaSuccess) return cuda_fail(e);
     RowPassArgs r;
     std::memset(&r, 0, sizeof r);
     r.d = d.d;
     r.t = no_rows();
-    r.items_d = int64_t(batch->n_draft) * d.d.nch;
-    r.items_t = 0;
+    r.rows_d = batch->n_draft;
+    r.rows_t = 0;
     r.err = ws.err;
     r.epoch = next_epoch();
+    r.work = ws.work;
     d.err = ws.err;
     d.epoch = r.epoch;
     if ((e = launch_rowpass(r, draft->dtype, TT_F32, s, sm_count_current(), true)) != cudaSuccess)
@@ -267,22 +269,26 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
     p.target_off = batch->target_off;
     p.map = map;
     p.need = ws.need_d;
+    p.work = ws.work;
     if ((e = launch_prep(p, s)) != cudaSuccess) return cuda_fail(e);
   }
   RowPassArgs r;
   std::memset(&r, 0, sizeof r);
   r.t = rowset(target, ws.part_t, nullptr, prm->temp_target);
-  r.items_t = (int64_t(batch->n_target) + batch->B) * r.t.nch;
+  r.rows_t = int64_t(batch->n_target) + batch->B;
   r.d = full_q ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
-  r.items_d = full_q ? int64_t(batch->n_draft) * r.d.nch : 0;
+  r.rows_d = full_q ? batch->n_draft : 0;
   r.B = batch->B;
   r.n_target = batch->n_target;
   r.target_off = batch->target_off;
   r.target_cols = tcols;
   r.err = ws.err;
   r.epoch = next_epoch();
+  r.work = full_q ? ws.work : nullptr;  // zeroed by the prep kernel
+  // the first kernel of the chain starts only after the caller's work is
+  // complete: it reads the logits before its grid-dependency wait
   if ((e = launch_rowpass(r, full_q ? draft->dtype : TT_F32, target->dtype, s,
-                          sm_count_current(), true)) != cudaSuccess)
+                          sm_count_current(), full_q)) != cudaSuccess)
     return cuda_fail(e);
 
   DecideArgs d;
@@ -350,6 +356,9 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   a.map = map;
   a.status = out->status;
   a.need = from_logits ? ws.need_d : nullptr;
+  a.work = ws.work;
+  a.target_cols = tcols;
+  a.excl = ws.excl;
 
   cudaError_t e = ensure_loaded();
   if (e != cudaSuccess) return cuda_fail(e);
@@ -360,15 +369,17 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   RowPassArgs r;
   std::memset(&r, 0, sizeof r);
   r.t = rowset(target, ws.part_t, nullptr, prm->temp_target);
-  r.items_t = (int64_t(batch->n_target) + batch->B) * r.t.nch;
+  r.rows_t = int64_t(batch->n_target) + batch->B;
   r.d = from_logits ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
-  r.items_d = from_logits ? int64_t(batch->n_draft) * r.d.nch : 0;
+  r.rows_d = from_logits ? batch->n_draft : 0;
   r.B = batch->B;
   r.n_target = batch->n_target;
   r.target_off = batch->target_off;
   r.target_cols = tcols;
   r.err = ws.err;
   r.epoch = next_epoch();
+  r.work = ws.work;       // zeroed by the alignment kernel
+  r.excl_late = ws.excl;  // written by the alignment kernel
   // programmatic dependent launch: target rows stream while the alignment runs
   // (unless stage events sit between the kernels)
   const bool pdl = prm->events == nullptr;

@@ -64,16 +64,6 @@ __device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
   return {hi, __fsub_rn(lo, __fsub_rn(hi, s.hi))};
 }
 
-// Compensated sum over the warp; every lane gets lane 0's result.
-__device__ __forceinline__ float warp_sum_comp(F2 v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const F2 w = {__shfl_xor_sync(0xffffffffu, v.hi, o), __shfl_xor_sync(0xffffffffu, v.lo, o)};
-    v = f2_add(v, w);
-  }
-  return __shfl_sync(0xffffffffu, __fadd_rn(v.hi, v.lo), 0);
-}
-
 // 2^(z * scale - M) with the exponent split exactly into n + f, |f| <= 1/2:
 // z * scale = xh + xl and xh - M = dh + dl are error-free transformations, so
 // only 2^f (from the SFU, relative error about 2^-22) is approximate.
@@ -85,43 +75,6 @@ __device__ __forceinline__ float exp2_scaled(float z, float scale, float M) {
   const float f = __fadd_rn(__fsub_rn(d.hi, n), __fadd_rn(d.lo, xl));
   if (!(n > -126.f)) return 0.f;
   return ex2_approx(f) * __int_as_float((int(n) + 127) << 23);
-}
-
-// Max and sum of 2^(m_c - max) * s_c of one row's partials (one warp; all
-// lanes get the same values). Rows of up to 128 chunks use the cached loads.
-__device__ __forceinline__ void row_stats(const Partial* part, int nch, const Partial (&cache)[4],
-                                          int lane, float& mx, float& S) {
-  float m = -INFINITY;
-  F2 acc = {0.f, 0.f};
-  if (nch <= 128) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) m = fmaxf(m, cache[i].m);
-    m = warp_max_f(m);
-    if (m != -INFINITY) {
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (cache[i].m != -INFINITY) acc = f2_add(acc, F2{cache[i].s * ex2_approx(cache[i].m - m), 0.f});
-    }
-  } else {
-    for (int c = lane; c < nch; c += 32) m = fmaxf(m, part[c].m);
-    m = warp_max_f(m);
-    if (m != -INFINITY)
-      for (int c = lane; c < nch; c += 32) {
-        const Partial q = part[c];
-        if (q.m != -INFINITY) acc = f2_add(acc, F2{q.s * ex2_approx(q.m - m), 0.f});
-      }
-  }
-  mx = m;
-  S = warp_sum_comp(acc);
-}
-
-__device__ __forceinline__ void load_cache(const Partial* part, int nch, int lane, bool valid,
-                                           Partial (&cache)[4]) {
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int c = lane + 32 * i;
-    cache[i] = (valid && nch <= 128 && c < nch) ? part[c] : Partial{-INFINITY, 0.f};
-  }
 }
 
 struct RowResult {
@@ -136,22 +89,141 @@ __device__ __forceinline__ RowResult with_token(float mx, float S, float zt, flo
   return {Mx, rest + exp2_scaled(zt, scale, Mx)};
 }
 
-// One CTA (16 warps) per request: the warps share the row normalisers, the
-// accept draws run one thread per position, warp 0 picks the chunk and the
-// whole CTA re-reads it (4 columns per thread).
+__device__ __forceinline__ F2 f2_neg(F2 a) { return {-a.hi, -a.lo}; }
+
+// a * b as a normalised pair (the product's rounding error from a fused
+// multiply-add).
+__device__ __forceinline__ F2 f2_mul_f(F2 a, float b) {
+  const float p = __fmul_rn(a.hi, b);
+  const float e = fmaf(a.hi, b, -p);
+  const float lo = fmaf(a.lo, b, e);
+  const float hi = __fadd_rn(p, lo);
+  return {hi, __fsub_rn(lo, __fsub_rn(hi, p))};
+}
+
+// Order of normalised pairs (hi = fl(hi + lo)): lexicographic, which is the
+// order of their values. Intervals whose ends are the same pairs tile exactly.
+__device__ __forceinline__ bool f2_lt(F2 a, F2 b) {
+  return a.hi < b.hi || (a.hi == b.hi && a.lo < b.lo);
+}
+__device__ __forceinline__ bool f2_le(F2 a, F2 b) {
+  return a.hi < b.hi || (a.hi == b.hi && a.lo <= b.lo);
+}
+
+__device__ __forceinline__ F2 shfl_up_f2(F2 v, int o, int width) {
+  return {__shfl_up_sync(0xffffffffu, v.hi, o, width), __shfl_up_sync(0xffffffffu, v.lo, o, width)};
+}
+__device__ __forceinline__ F2 shfl_f2(F2 v, int src, int width) {
+  return {__shfl_sync(0xffffffffu, v.hi, src, width), __shfl_sync(0xffffffffu, v.lo, src, width)};
+}
+
+// Max / compensated sum over groups of WIDTH lanes (the whole warp calls).
+template <int WIDTH>
+__device__ __forceinline__ float group_max(float v) {
+#pragma unroll
+  for (int o = WIDTH / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o, WIDTH));
+  return v;
+}
+template <int WIDTH>
+__device__ __forceinline__ F2 group_sum(F2 v) {
+#pragma unroll
+  for (int o = WIDTH / 2; o > 0; o >>= 1) {
+    const F2 w = {__shfl_xor_sync(0xffffffffu, v.hi, o, WIDTH),
+                  __shfl_xor_sync(0xffffffffu, v.lo, o, WIDTH)};
+    v = f2_add(v, w);  // f2_add is commutative bit for bit: every lane ends equal
+  }
+  return v;
+}
+
+// Coarse level of the inverse CDF (Alg. 4): over chunk masses R(c), c in
+// [0, nch), in column order, the chunk where the running sum first exceeds
+// theta = u * Z, Z the total, and theta minus the mass before that chunk.
+// WIDTH lanes (sublane sl) take lane-contiguous ranges of chunks. theta past
+// the end by rounding gives the last chunk with mass and rel = +inf. Every lane
+// of the warp calls; results are per group.
+template <int WIDTH, class MassFn>
+__device__ __forceinline__ void coarse_pick(const MassFn& R, int nch, int lane, float u, int& chunk,
+                                            F2& rel, F2& Z) {
+  const int sl = lane & (WIDTH - 1);
+  const int per = (nch + WIDTH - 1) / WIDTH;
+  const int lo = min(nch, sl * per), hi = min(nch, lo + per);
+  F2 loc = {0.f, 0.f};
+  int last = -1;
+  for (int c = lo; c < hi; ++c) {
+    const F2 r = R(c);
+    loc = f2_add(loc, r);
+    if (r.hi > 0.f) last = c;
+  }
+  F2 incl = loc;
+#pragma unroll
+  for (int o = 1; o < WIDTH; o <<= 1) {
+    const F2 n = shfl_up_f2(incl, o, WIDTH);
+    if (sl >= o) incl = f2_add(n, incl);
+  }
+  const F2 prev = shfl_up_f2(incl, 1, WIDTH);
+  const F2 excl = sl == 0 ? F2{0.f, 0.f} : prev;
+  Z = shfl_f2(incl, WIDTH - 1, WIDTH);
+  const F2 th = f2_mul_f(Z, u);
+  int found = -1;
+  F2 r_rel = {INFINITY, 0.f};
+  if (f2_le(excl, th) && f2_lt(th, incl)) {
+    F2 cum = excl;
+    for (int c = lo; c < hi; ++c) {
+      const F2 r = R(c);
+      const F2 nx = f2_add(cum, r);
+      if (r.hi > 0.f && f2_lt(th, nx)) {
+        found = c;
+        r_rel = f2_add(th, f2_neg(cum));
+        break;
+      }
+      cum = nx;
+    }
+    if (found < 0) found = last;  // rounding inside the range: its last chunk with mass
+  }
+  const unsigned grp = (0xffffffffu >> (32 - WIDTH)) << (lane & ~(WIDTH - 1));
+  const unsigned hit = __ballot_sync(0xffffffffu, found >= 0) & grp;
+  int la = last;
+#pragma unroll
+  for (int o = WIDTH / 2; o > 0; o >>= 1) la = max(la, __shfl_xor_sync(0xffffffffu, la, o, WIDTH));
+  const int src = hit ? __ffs(hit) - 1 : (lane & ~(WIDTH - 1));
+  const int fc = __shfl_sync(0xffffffffu, found, src);
+  const F2 fr = shfl_f2(r_rel, src, 32);
+  if (hit) {
+    chunk = fc;
+    rel = fr;
+  } else {  // theta at the very top: the last chunk with mass
+    chunk = la < 0 ? 0 : la;
+    rel = {INFINITY, 0.f};
+  }
+}
+
+// One CTA (16 warps) per request.
+//  before the grid-dependency wait: checks of the caller's inputs, the map,
+//    the scored logits and both uniforms of every position;
+//  rows: one half-warp per row rebuilds the normaliser of each target row and
+//    each mapped draft row from the row-pass partials;
+//  accept test (one thread per position) and, for every candidate row, the
+//    coarse level of its residual (one half-warp per row), side by side;
+//  fine level: the whole CTA re-reads the chosen chunk of the accepted row.
 __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
-  __shared__ float s_p[TT_MAX_M], s_q[TT_MAX_M];
-  __shared__ int s_col[TT_MAX_M], s_map[TT_MAX_M];
-  __shared__ float s_M[TT_MAX_M + 1], s_S[TT_MAX_M + 1];
-  __shared__ double s_R[kMaxChunksPerRow];
-  __shared__ double s_wtot[kWarps], s_wpre[kWarps];
-  __shared__ int s_a, s_chunk, s_pick, s_last;
-  __shared__ double s_theta;
-  __shared__ float s_dM, s_dS;
+  __shared__ int s_col[TT_MAX_M], s_map[TT_MAX_M], s_first[TT_MAX_M], s_qi[TT_MAX_M];
+  __shared__ int s_task[TT_MAX_M];
+  __shared__ float s_zt[TT_MAX_M], s_zd[TT_MAX_M], s_u[TT_MAX_M];
+  __shared__ float s_p[TT_MAX_M], s_q[TT_MAX_M], s_DM[TT_MAX_M], s_DS[TT_MAX_M];
+  __shared__ float s_u2[TT_MAX_M + 1], s_M[TT_MAX_M + 1], s_S[TT_MAX_M + 1];
+  __shared__ int s_cchunk[TT_MAX_M + 1];
+  __shared__ F2 s_crel[TT_MAX_M + 1];
+  __shared__ unsigned char s_cmode[TT_MAX_M + 1];
+  __shared__ F2 s_R[kMaxChunksPerRow];
+  __shared__ F2 s_wtot[kWarps], s_wpre[kWarps + 1];
+  __shared__ int s_dcol[TT_MAX_K];
+  __shared__ int s_a, s_pick, s_last, s_nd, s_err, s_bad;
 
   const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int half = lane >> 4, hl = lane & 15;
   const bool want_draft = a.full_q || a.q_hat_in == nullptr;
   const bool q_from_logits = a.q_hat_in == nullptr && a.draft_probs == nullptr;
+  const bool draft_rows = q_from_logits || a.full_q;  // draft normalisers needed
 
   // ------------------------------------------ checks on the caller's inputs
   int st = 0, t0 = 0, m = 0, d0 = 0, k = 0;
@@ -168,164 +240,245 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
     if (m == 0 || (want_draft && k == 0)) st |= TT_REQ_EMPTY;
     if (m > a.max_m || m > TT_MAX_M) st |= TT_REQ_TOO_LONG;
   }
+  if (q_from_logits && k > TT_MAX_K) st |= TT_REQ_TOO_LONG;
   if (tid == 0) {
     s_a = m;
     s_pick = -1;
     s_last = -1;
-    s_dM = 0.f;
-    s_dS = 1.f;
+    s_nd = 0;
+    s_err = 0;
+    s_bad = 0;
   }
+  __syncthreads();
+  // One round of loads: the caller's columns and, read before the wait, the
+  // alignment's status and map (every CTA of the row pass between the two
+  // grids waits for the alignment grid before it lets this grid start; they
+  // are read through L2 only).
   int bad = 0;
   if (st == 0) {
     for (int j = tid; j < m; j += kDecThreads) {
       const int col = a.target_cols[t0 + j];
       s_col[j] = col;
-      if (col < 0 || col >= a.t.V) bad = 1;
+      if (col < 0 || col >= a.t.V) bad |= 1;
+      int i = j;
+      if (want_draft) {
+        i = __ldcg(a.map + t0 + j);
+        if (i < 0 || i >= k) bad |= 2;
+      }
+      s_map[j] = i;
     }
     if (q_from_logits)
       for (int i = tid; i < k; i += kDecThreads) {
         const int col = a.draft_cols[d0 + i];
-        if (col < 0 || col >= a.d.V) bad = 1;
+        s_dcol[i] = col;
+        if (col < 0 || col >= a.d.V) bad |= 1;
       }
   }
-  if (__syncthreads_or(bad)) st |= TT_REQ_ID_OUT_OF_RANGE;
+  const int s_in = a.status_in ? __ldcg(a.status_in + b) : 0;
+  if (bad) atomicOr(&s_bad, bad);
+  __syncthreads();
+  if (st == 0 && (s_bad & 1)) st |= TT_REQ_ID_OUT_OF_RANGE;
+  if (s_in != 0) st = s_in;  // the alignment's verdict comes first
+  if (st == 0 && (s_bad & 2)) st |= TT_REQ_ID_OUT_OF_RANGE;
+
+  const uint64_t req = a.request_base + uint64_t(b);
+  if (st == 0) {
+    for (int j = tid; j <= m; j += kDecThreads) {
+      s_u2[j] = float(philox_uniform(a.seed, uint64_t(j), 1, req));
+      if (j == m) continue;
+      int f = j;  // first position of this run of equal map entries
+      if (want_draft)
+        while (f > 0 && s_map[f - 1] == s_map[j]) --f;
+      s_first[j] = f;
+      s_u[j] = float(philox_uniform(a.seed, uint64_t(j), 0, req));
+      s_zt[j] = load_checked(a, a.t, a.dt_t, int64_t(t0) + b + j, s_col[j]);
+      // q of position j sits at s_q[s_qi[j]]: per position when given, per
+      // run when transferred from the draft logits here
+      s_qi[j] = q_from_logits ? f : j;
+      if (a.q_hat_in) {
+        s_q[j] = a.q_hat_in[t0 + j];
+      } else if (a.draft_probs) {
+        s_q[j] = a.draft_probs[int64_t(d0) + s_map[j]];
+      }
+      if (draft_rows && f == j) {
+        s_task[atomicAdd(&s_nd, 1)] = j;
+        if (q_from_logits)
+          s_zd[j] = load_checked(a, a.d, a.dt_d, int64_t(d0) + s_map[j], s_dcol[s_map[j]]);
+      }
+    }
+  }
+  __syncthreads();
 
   // ------------------------------ results of the kernels before this one
   grid_dependency_wait();
-  if (a.status_in) {
-    const int s_in = a.status_in[b];
-    if (s_in != 0) st = s_in;  // the alignment's verdict comes first
-  }
-  if (a.err && a.err[0] == a.epoch) st = a.err[1];  // the row pass failed
-  bad = 0;
-  if (st == 0 && want_draft)
-    for (int j = tid; j < m; j += kDecThreads) {
-      const int i = a.map[t0 + j];
-      s_map[j] = i;
-      if (i < 0 || i >= k) bad = 1;
-    }
-  if (__syncthreads_or(bad)) st |= TT_REQ_ID_OUT_OF_RANGE;
   if (st != 0) {
     if (tid == 0) {
+      const int e = (a.err && __ldcg(a.err) == a.epoch) ? __ldcg(a.err + 1) : 0;
       a.accepted[b] = 0;
       a.next_token[b] = -1;
-      a.status[b] = st;
+      a.status[b] = e ? e : st;
     }
     return;
   }
+  if (tid == 0 && a.err && __ldcg(a.err) == a.epoch) s_err = __ldcg(a.err + 1);
 
-  // ------ row normalisers, one warp per row: target rows 0..m, then the
-  // first row of each run of equal map entries (the copy rule reuses it)
+  // ------ row normalisers: target rows 0..m, then the first row of each run
+  // of equal map entries (the copy rule reuses it); a half-warp per row
   int nonfinite = 0;
-  const int n_tasks = m + 1 + (q_from_logits ? m : 0);
-  for (int task = warp; task < n_tasks; task += kWarps) {
+  const int n_tasks = m + 1 + s_nd;
+  for (int base = 2 * warp; base < n_tasks; base += 2 * kWarps) {
+    const int task = base + half;
+    const bool valid = task < n_tasks;
     const bool tgt = task <= m;
-    const int j = tgt ? task : task - (m + 1);
-    if (!tgt && j > 0 && s_map[j] == s_map[j - 1]) continue;
-    const int64_t row = tgt ? int64_t(t0) + b + j : int64_t(d0) + s_map[j];
-    const RowSet& R = tgt ? a.t : a.d;
-    const int dt = tgt ? a.dt_t : a.dt_d;
-    const Partial* part = R.part + row * R.nch;
-    // issue the loads first: the scored token's logit and the row's partials
+    int j = 0;
+    int64_t row = int64_t(t0) + b;
+    const RowSet* R = &a.t;
     float z = 0.f;
-    if (!tgt) z = load_checked(a, R, dt, row, a.draft_cols[row]);
-    else if (j < m) z = load_checked(a, R, dt, row, s_col[j]);
-    Partial cache[4];
-    load_cache(part, R.nch, lane, true, cache);
-    float mx, S;
-    row_stats(part, R.nch, cache, lane, mx, S);
-    if (tgt) {
-      float M = mx, Stot = S, ph = 0.f;
-      if (j < m) {  // add back the scored token's term, left out by the row pass
-        const RowResult rr = with_token(mx, S, z, R.scale);
-        M = rr.M;
-        Stot = rr.S;
-        ph = exp2_scaled(z, R.scale, M) * __frcp_rn(Stot);
+    if (valid) {
+      if (tgt) {
+        j = task;
+        row += j;
+        if (j < m) z = s_zt[j];
+      } else {
+        j = s_task[task - (m + 1)];
+        row = int64_t(d0) + s_map[j];
+        R = &a.d;
+        if (q_from_logits) z = s_zd[j];
       }
-      if (!(Stot > 0.f) || !isfinite(Stot) || isnan(M)) nonfinite = 1;
-      if (lane == 0) {
-        s_M[j] = M;
-        s_S[j] = Stot;
-        if (j < m) {
+    }
+    const int nch = valid ? R->nch : 0;
+    const Partial* part = R->part + row * R->nch;
+    const bool cached = nch <= 128;
+    Partial c8[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int c = hl + 16 * i;
+      c8[i] = (cached && c < nch) ? part[c] : Partial{-INFINITY, 0.f};
+    }
+    float lmx = -INFINITY;
+    if (cached) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) lmx = fmaxf(lmx, c8[i].m);
+    } else {
+      for (int c = hl; c < nch; c += 16) lmx = fmaxf(lmx, part[c].m);
+    }
+    const float mx = group_max<16>(lmx);
+    F2 acc = {0.f, 0.f};
+    if (mx != -INFINITY) {
+      if (cached) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          if (c8[i].m != -INFINITY) acc = f2_add(acc, F2{c8[i].s * ex2_approx(c8[i].m - mx), 0.f});
+      } else {
+        for (int c = hl; c < nch; c += 16) {
+          const Partial q = part[c];
+          if (q.m != -INFINITY) acc = f2_add(acc, F2{q.s * ex2_approx(q.m - mx), 0.f});
+        }
+      }
+    }
+    const F2 Ssum = group_sum<16>(acc);
+    const float S = __fadd_rn(Ssum.hi, Ssum.lo);
+    if (valid && hl == 0) {
+      if (tgt) {
+        float M = mx, St = S;
+        if (j < m) {  // add back the scored token's term, left out by the row pass
+          const RowResult rr = with_token(mx, S, z, R->scale);
+          M = rr.M;
+          St = rr.S;
+          const float ph = exp2_scaled(z, R->scale, M) * __frcp_rn(St);
           s_p[j] = ph;
           if (a.p_hat) a.p_hat[t0 + j] = ph;
         }
-        if (a.lse) a.lse[row] = (M + lg2_approx(Stot)) * 0.6931471805599453f;
+        if (!(St > 0.f) || !isfinite(St) || isnan(M)) nonfinite = 1;
+        s_M[j] = M;
+        s_S[j] = St;
+        if (a.lse) a.lse[row] = (M + lg2_approx(St)) * 0.6931471805599453f;
+      } else {
+        if (!(S > 0.f) || !isfinite(S) || mx == -INFINITY) nonfinite = 1;
+        s_DM[j] = mx;
+        s_DS[j] = S;
+        if (q_from_logits) s_q[j] = exp2_scaled(z, R->scale, mx) * __frcp_rn(S);
       }
-    } else {
-      if (!(S > 0.f) || !isfinite(S) || mx == -INFINITY) nonfinite = 1;
-      if (lane == 0) s_q[j] = exp2_scaled(z, R.scale, mx) * __frcp_rn(S);
     }
   }
-  if (__syncthreads_or(nonfinite)) {
+  if (__syncthreads_or(nonfinite) || s_err) {
     if (tid == 0) {
       a.accepted[b] = 0;
       a.next_token[b] = -1;
-      a.status[b] = TT_REQ_NOT_FINITE;
+      a.status[b] = s_err ? s_err : TT_REQ_NOT_FINITE;
     }
     return;
   }
-  for (int j = tid; j < m; j += kDecThreads) {
-    float qh;
-    if (a.q_hat_in) {
-      qh = a.q_hat_in[t0 + j];
-    } else if (a.draft_probs) {
-      qh = a.draft_probs[int64_t(d0) + s_map[j]];
-    } else {
-      int f = j;  // first position of this run of equal map entries
-      while (f > 0 && s_map[f - 1] == s_map[j]) --f;
-      qh = s_q[f];
-    }
-    if (a.q_hat_out) a.q_hat_out[t0 + j] = qh;
-    if (!q_from_logits) s_q[j] = qh;
-  }
-  __syncthreads();
-  if (q_from_logits) {  // copies of a run take the value of its first entry
-    for (int j = tid; j < m; j += kDecThreads) {
-      int f = j;
-      while (f > 0 && s_map[f - 1] == s_map[j]) --f;
-      if (f != j) s_q[j] = s_q[f];
-    }
-    __syncthreads();
-  }
 
   // --------------------------- accept while u_j q_j < p_j (u < 1 exactly)
-  const uint64_t req = a.request_base + uint64_t(b);
-  if (tid < m) {
-    const float u = float(philox_uniform(a.seed, uint64_t(tid), 0, req));
-    if (!(u * s_q[tid] < s_p[tid])) atomicMin(&s_a, tid);
+  for (int j = tid; j < m; j += kDecThreads) {
+    const float qh = s_q[s_qi[j]];
+    if (a.q_hat_out) a.q_hat_out[t0 + j] = qh;
+    if (!(s_u[j] * qh < s_p[j])) atomicMin(&s_a, j);
+  }
+
+  const int nch = a.t.nch;
+  const int V = a.t.V;
+  const float scale_t = a.t.scale;
+  // coarse level of every candidate row's residual, side by side with the
+  // accept test: one-hot q puts r_t = max(0, p_j - q_j) on t_j and p elsewhere
+  // (the row itself when that residual has no mass, and for the bonus row m)
+  if (!a.full_q) {
+    for (int base = 2 * warp; base <= m; base += 2 * kWarps) {
+      const int j0 = base + half;
+      const bool valid = j0 <= m;
+      const int j = valid ? j0 : m;
+      const Partial* part = a.t.part + (int64_t(t0) + b + j) * nch;
+      const float Mj = s_M[j], invS = __frcp_rn(s_S[j]);
+      const int ct = j < m ? s_col[j] / kChunk : -1;
+      const float pj = j < m ? s_p[j] : 0.f;
+      const float rt = j < m ? fmaxf(0.f, pj - s_q[s_qi[j]]) : 0.f;
+      auto base_mass = [&](int c) -> float {
+        const Partial P = part[c];
+        return P.m == -INFINITY ? 0.f : P.s * ex2_approx(P.m - Mj) * invS;
+      };
+      // does the one-hot residual have mass?
+      const int per = (nch + 15) / 16;
+      const int lo = min(nch, hl * per), hi = min(nch, lo + per);
+      bool pos = false;
+      for (int c = lo; c < hi && !pos; ++c) pos = base_mass(c) > 0.f;
+      const unsigned grp = 0xffffu << (lane & 16);
+      const bool any = (__ballot_sync(0xffffffffu, pos) & grp) != 0;
+      const int md = (j < m && (any || rt > 0.f)) ? 1 : 0;
+      const float extra = j < m ? (md == 1 ? rt : pj) : 0.f;
+      auto mass = [&](int c) -> F2 {
+        F2 r = {base_mass(c), 0.f};
+        if (c == ct) r = f2_add(r, F2{extra, 0.f});
+        return r;
+      };
+      int chunk;
+      F2 rel, Z;
+      coarse_pick<16>(mass, nch, lane, s_u2[j], chunk, rel, Z);
+      if (valid && hl == 0) {
+        s_cchunk[j] = chunk;
+        s_crel[j] = rel;
+        s_cmode[j] = (unsigned char)md;
+      }
+    }
   }
   __syncthreads();
   const int acc = s_a;
   const int64_t row = int64_t(t0) + b + acc;
-  const int nch = a.t.nch;
-  const int V = a.t.V;
   const int col_t = acc < m ? s_col[acc] : -1;
   const float Mt = s_M[acc];
   const float invSt = __frcp_rn(s_S[acc]);
-  const float scale_t = a.t.scale;
   const char* trow = a.t.data + row * a.t.stride_bytes;
   const float p_a = acc < m ? s_p[acc] : 0.f;
-  const float r_t = acc < m ? fmaxf(0.f, p_a - s_q[acc]) : 0.f;
-  int mode = acc < m ? (a.full_q ? 2 : 1) : 0;  // 0 the row itself, 1 one-hot, 2 full-q residual
+  const float r_t = acc < m ? fmaxf(0.f, p_a - s_q[s_qi[acc]]) : 0.f;
   const char* drow = nullptr;
-  if (mode == 2) {
-    const int64_t rd = int64_t(d0) + s_map[acc];
-    drow = a.d.data + rd * a.d.stride_bytes;
-    if (warp == 0) {
-      Partial c4[4];
-      load_cache(a.d.part + rd * a.d.nch, a.d.nch, lane, true, c4);
-      float Md, Sd;
-      row_stats(a.d.part + rd * a.d.nch, a.d.nch, c4, lane, Md, Sd);
-      if (lane == 0) {
-        s_dM = Md;
-        s_dS = Sd;
-      }
-    }
-    __syncthreads();
+  float Md = 0.f, invSd = 1.f;
+  if (a.full_q && acc < m) {
+    const int f = s_first[acc];
+    drow = a.d.data + (int64_t(d0) + s_map[acc]) * a.d.stride_bytes;
+    Md = s_DM[f];
+    invSd = __frcp_rn(s_DS[f]);
   }
-  const float Md = s_dM;
-  const float invSd = __frcp_rn(s_dS);
+  // 0 the row itself, 1 one-hot residual, 2 full-q residual max(0, p - q)
   auto r_of = [&](int x, float z, int md) -> float {
     const float p = ex2_approx(fmaf(z, scale_t, -Mt)) * invSt;
     if (md == 1) return x == col_t ? r_t : p;
@@ -335,89 +488,46 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
     }
     return p;
   };
-  const double u2 = philox_uniform(a.seed, uint64_t(acc), 1, req);
-
-  // ------------------------------- coarse level: the chunk holding u' * Z
-  for (int pass = 0; pass < 2; ++pass) {
-    if (mode == 2) {  // elementwise residual masses, one warp per chunk
+  if (a.full_q) {  // full-q residual: chunk masses from the logits themselves
+    const Partial* part = a.t.part + row * nch;
+    int md = acc < m ? 2 : 0;
+    if (md == 2) {
       for (int c = warp; c < nch; c += kWarps) {
-        F2 part = {0.f, 0.f};
+        F2 acc2 = {0.f, 0.f};
         const int hi_c = min(V, (c + 1) * kChunk);
         for (int x = c * kChunk + lane; x < hi_c; x += 32)
-          part = f2_add(part, F2{r_of(x, load_dt(trow, a.dt_t, x), 2), 0.f});
-        const float Rc = warp_sum_comp(part);
-        if (lane == 0) s_R[c] = double(Rc);
+          acc2 = f2_add(acc2, F2{r_of(x, load_dt(trow, a.dt_t, x), 2), 0.f});
+        const F2 Rc = group_sum<32>(acc2);
+        if (lane == 0) s_R[c] = Rc;
       }
-    } else {
-      for (int c = tid; c < nch; c += kDecThreads) {
-        const Partial P = a.t.part[row * nch + c];
-        double R = P.m == -INFINITY ? 0.0 : double(P.s * ex2_approx(P.m - Mt) * invSt);
-        if (col_t >= 0 && col_t / kChunk == c) R += mode == 1 ? r_t : p_a;
-        s_R[c] = R;
+      __syncthreads();
+    }
+    if (warp == 0) {
+      auto mass0 = [&](int c) -> F2 {
+        const Partial P = part[c];
+        F2 r = {P.m == -INFINITY ? 0.f : P.s * ex2_approx(P.m - Mt) * invSt, 0.f};
+        if (col_t >= 0 && c == col_t / kChunk) r = f2_add(r, F2{p_a, 0.f});
+        return r;
+      };
+      auto mass2 = [&](int c) -> F2 { return s_R[c]; };
+      int chunk;
+      F2 rel, Z;
+      if (md == 2) {
+        coarse_pick<32>(mass2, nch, lane, s_u2[acc], chunk, rel, Z);
+        if (!(Z.hi > 0.f)) md = 0;  // degenerate residual: the row itself
+      }
+      if (md == 0) coarse_pick<32>(mass0, nch, lane, s_u2[acc], chunk, rel, Z);
+      if (lane == 0) {
+        s_cchunk[acc] = chunk;
+        s_crel[acc] = rel;
+        s_cmode[acc] = (unsigned char)md;
       }
     }
-    __syncthreads();
-    if (warp == 0) {  // lane-contiguous ranges of chunks, scanned in column order
-      const int per = (nch + 31) / 32;
-      const int lo = min(nch, lane * per), hi = min(nch, lo + per);
-      double loc = 0.0;
-      int last = -1;
-      for (int c = lo; c < hi; ++c) {
-        loc += s_R[c];
-        if (s_R[c] > 0.0) last = c;
-      }
-      double incl = loc;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const double n = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += n;
-      }
-      const double prev = __shfl_up_sync(0xffffffffu, incl, 1);
-      const double excl = lane == 0 ? 0.0 : prev;
-      const double Z = __shfl_sync(0xffffffffu, incl, 31);
-      int last_all = last;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) last_all = max(last_all, __shfl_xor_sync(0xffffffffu, last_all, o));
-      if (!(Z > 0.0) && mode != 0) {
-        if (lane == 0) s_chunk = -2;  // degenerate residual
-      } else {
-        const double th = u2 * Z;
-        int found = -1;
-        double rel = INFINITY;
-        if (excl <= th && th < incl) {
-          double cum = excl;
-          for (int c = lo; c < hi; ++c) {
-            if (th < cum + s_R[c]) {
-              found = c;
-              rel = th - cum;
-              break;
-            }
-            cum += s_R[c];
-          }
-          if (found < 0) found = last;  // rounding inside the range: its last chunk with mass
-        }
-        const unsigned hit = __ballot_sync(0xffffffffu, found >= 0);
-        if (hit) {
-          const int src = __ffs(hit) - 1;
-          const int fc = __shfl_sync(0xffffffffu, found, src);
-          const double fr = __shfl_sync(0xffffffffu, rel, src);
-          if (lane == 0) {
-            s_chunk = fc;
-            s_theta = fr;
-          }
-        } else if (lane == 0) {  // theta at the very top: the last chunk with mass
-          s_chunk = last_all < 0 ? 0 : last_all;
-          s_theta = INFINITY;
-        }
-      }
-    }
-    __syncthreads();
-    if (s_chunk != -2) break;
-    mode = 0;  // fall back to the row itself
     __syncthreads();
   }
-  const int chunk = s_chunk;
-  const double theta = s_theta;
+  const int chunk = s_cchunk[acc];
+  const F2 rel = s_crel[acc];
+  const int mode = s_cmode[acc];
 
   // ------------------------------------------ fine level: one chunk re-read
   constexpr int kPer = kChunk / kDecThreads;  // 4 consecutive columns per thread
@@ -441,7 +551,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
 #pragma unroll
     for (int q = 0; q < kPer; ++q) r[q] = x0 + q < V ? load_dt(trow, a.dt_t, x0 + q) : 0.f;
   }
-  float run = 0.f;
+  F2 run = {0.f, 0.f};
   int last_pos = -1;
 #pragma unroll
   for (int q = 0; q < kPer; ++q) {
@@ -449,37 +559,42 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(DecideArgs a) {
     const float v = x < V ? r_of(x, r[q], mode) : 0.f;
     if (v > 0.f) last_pos = x;
     r[q] = v;
-    run += v;
+    run = f2_add(run, F2{v, 0.f});
   }
-  // block prefix: fp64 scan within each warp, warp totals scanned by warp 0
-  double incl = double(run);
+  // block prefix in pairs: scan within each warp, warp totals scanned by
+  // warp 0; a warp's last interval ends where the next warp's first begins
+  F2 incl = run;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const double n = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += n;
+    const F2 n = shfl_up_f2(incl, o, 32);
+    if (lane >= o) incl = f2_add(n, incl);
   }
-  const double prev = __shfl_up_sync(0xffffffffu, incl, 1);
-  double excl = lane == 0 ? 0.0 : prev;
+  const F2 prev = shfl_up_f2(incl, 1, 32);
+  F2 excl = lane == 0 ? F2{0.f, 0.f} : prev;
   if (lane == 31) s_wtot[warp] = incl;
   __syncthreads();
-  if (tid == 0) {  // warp bases in order, so that the intervals tile exactly
-    double acc_w = 0.0;
-    for (int w = 0; w < kWarps; ++w) {
-      s_wpre[w] = acc_w;
-      acc_w += s_wtot[w];
+  if (warp == 0) {
+    const F2 t = lane < kWarps ? s_wtot[lane] : F2{0.f, 0.f};
+    F2 wi = t;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const F2 n = shfl_up_f2(wi, o, 32);
+      if (lane >= o) wi = f2_add(n, wi);
     }
+    const F2 wp = shfl_up_f2(wi, 1, 32);
+    if (lane <= kWarps) s_wpre[lane] = lane == 0 ? F2{0.f, 0.f} : wp;
   }
   __syncthreads();
-  const double base = s_wpre[warp];
-  incl += base;
-  excl += base;
-  if (excl <= theta && theta < incl) {
-    double c = excl;
+  const F2 base = s_wpre[warp];
+  incl = lane == 31 ? s_wpre[warp + 1] : f2_add(base, incl);
+  excl = f2_add(base, excl);
+  if (f2_le(excl, rel) && f2_lt(rel, incl)) {
+    F2 c = excl;
     int pick = last_pos;
 #pragma unroll
     for (int q = 0; q < kPer; ++q) {
-      c += double(r[q]);
-      if (c > theta && r[q] > 0.f) {
+      c = f2_add(c, F2{r[q], 0.f});
+      if (r[q] > 0.f && f2_lt(rel, c)) {
         pick = x0 + q;
         break;
       }
@@ -561,6 +676,8 @@ __global__ void __launch_bounds__(kDecThreads) transfer_kernel(DecideArgs a) {
 // Needed-draft-row flags from an alignment map.
 __global__ void prep_kernel(PrepArgs a) {
   const int b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (a.work && blockIdx.x == 0 && threadIdx.x < kWorkShards)
+    a.work[threadIdx.x * kWorkStride] = 0ull;  // read after this grid ends
   if (b >= a.B) return;
   if (a.need && csr_ok(a.draft_off, b, a.n_draft) && csr_ok(a.target_off, b, a.n_target)) {
     const int d0 = a.draft_off[b], k = a.draft_off[b + 1] - d0;

@@ -28,13 +28,17 @@ constexpr int kConsumerWarps = 8;
 constexpr int kThreads = (kConsumerWarps + 1) * 32;
 constexpr int kRingBytes = 64 * 1024;  // three CTAs per SM fit
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
+constexpr int kGrabMinBytes = 16 * 1024;   // smallest draw from the work counter
+constexpr int kGrabMaxBytes = 128 * 1024;  // largest draw
 
+// One stage holds one unit: cps consecutive chunks of one row (cps = 1 for
+// fp32 rows, 2 for bf16 rows, so that every stage is one 8 KB bulk copy).
 struct Desc {
   int64_t row;    // < 0: no more work for this consumer warp
-  int32_t chunk;
-  int32_t n;      // columns in the chunk
+  int32_t chunk;  // first chunk of the unit
+  int32_t n;      // columns in the unit
   int32_t n_smem; // leading columns delivered by the bulk copy (rest read directly)
-  int32_t excl;   // column (within the row) left out of the sum, -1 = none
+  int32_t excl;   // column (within the unit) left out of the sum, -1 = none
   int32_t set;    // 0 draft rows, 1 target rows
   int32_t pad;
 };
@@ -44,11 +48,14 @@ struct Desc {
 // mbarrier parity wait cannot tell phase n from phase n + 2.
 template <int DTD, int DTT>
 struct Ring {
-  static constexpr int kEsz = (DTD == TT_F32 || DTT == TT_F32) ? 4 : 2;
-  static constexpr int kStageBytes = kChunk * kEsz;
+  static constexpr int kStageBytes = kChunk * 4;  // one fp32 chunk or two bf16 chunks
+  static constexpr int kCpsD = DTD == TT_F32 ? 1 : 2;  // chunks per stage, draft rows
+  static constexpr int kCpsT = DTT == TT_F32 ? 1 : 2;  // chunks per stage, target rows
   static constexpr int kStages = kRingBytes / kStageBytes;
   static constexpr size_t kSmem = size_t(kRingBytes) + kStages * (2 * sizeof(uint64_t) + sizeof(Desc));
   static_assert(kStages % kConsumerWarps == 0, "each stage belongs to one consumer warp");
+  static constexpr int kGrabMin = kGrabMinBytes / kStageBytes > 0 ? kGrabMinBytes / kStageBytes : 1;
+  static constexpr int kGrabMax = kGrabMaxBytes / kStageBytes;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -214,54 +221,59 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
   if (warp == kConsumerWarps) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
-      // this CTA's share: a block of target items, then a block of draft items
       const int64_t G = gridDim.x, g = blockIdx.x;
-      const int64_t t_lo = a.items_t * g / G, t_hi = a.items_t * (g + 1) / G;
-      const int64_t d_lo = a.items_d * g / G, d_hi = a.items_d * (g + 1) / G;
-      bool ok = true, waited = false;
+      // units (stages) per row and in all of each family
+      const int upr_t = (a.t.nch + R::kCpsT - 1) / R::kCpsT;
+      const int upr_d = (a.d.nch + R::kCpsD - 1) / R::kCpsD;
+      const int64_t items_t = a.rows_t * upr_t, items_d = a.rows_d * upr_d;
+      bool ok = true;
       int it = 0;
-      int64_t cached_row = -1;
+      int64_t cached_row = -1, cached_drow = -1;
       int cached_excl = -1;
-      for (int64_t item = t_lo; ok && item < t_hi + (d_hi - d_lo); ++item) {
+      bool cached_need = true;
+      // Queues chunk `chunk` of row `row` (tgt: a target row, else a draft
+      // row) on the next stage; false once a wait has run out.
+      bool late = false;  // past the grid-dependency wait
+      auto issue = [&](bool tgt, int64_t row, int unit) -> bool {
         Desc d;
         const RowSet* S;
-        int esz;
-        if (item < t_hi) {
+        int esz, cps;
+        d.row = row;
+        if (tgt) {
           S = &a.t;
           esz = DTT == TT_F32 ? 4 : 2;
-          d.row = item / a.t.nch;
-          d.chunk = int(item - d.row * a.t.nch);
+          cps = R::kCpsT;
           d.set = 1;
-          if (d.row != cached_row) {
-            cached_row = d.row;
-            cached_excl = a.excl ? a.excl[d.row] : target_excl(a, d.row);
+          if (row != cached_row) {
+            cached_row = row;
+            cached_excl = a.excl                ? a.excl[row]
+                          : (late && a.excl_late) ? a.excl_late[row]
+                                                  : target_excl(a, row);
           }
-          const int ex = cached_excl - d.chunk * kChunk;
-          d.excl = (cached_excl >= 0 && ex >= 0 && ex < kChunk) ? ex : -1;
+          const int ex = cached_excl - unit * cps * kChunk;
+          d.excl = (cached_excl >= 0 && ex >= 0 && ex < cps * kChunk) ? ex : -1;
         } else {
-          if (!waited) {  // draft rows need the alignment's flags
-            grid_dependency_wait();
-            waited = true;
-          }
-          const int64_t di = d_lo + (item - t_hi);
           S = &a.d;
           esz = DTD == TT_F32 ? 4 : 2;
-          d.row = di / a.d.nch;
-          d.chunk = int(di - d.row * a.d.nch);
+          cps = R::kCpsD;
           d.set = 0;
           d.excl = -1;
-          if (a.d.need && !a.d.need[d.row]) continue;
+          if (row != cached_drow) {
+            cached_drow = row;
+            cached_need = !a.d.need || a.d.need[row] != 0;
+          }
+          if (!cached_need) return true;  // no target position maps to this row
         }
+        d.chunk = unit * cps;
         const int c0 = d.chunk * kChunk;
-        d.n = min(kChunk, S->V - c0);
+        d.n = min(cps * kChunk, S->V - c0);
         const uint32_t bytes = uint32_t(d.n * esz) & ~15u;  // bulk copies move 16-byte units
         d.n_smem = int(bytes) / esz;
         const int s = it % R::kStages;
         const uint32_t par = ((it / R::kStages) & 1) ^ 1;
         if (!mbar_wait(&empty[s], par)) {
           report_error(a.err, a.epoch, TT_REQ_TIMEOUT);
-          ok = false;
-          break;
+          return false;
         }
         // every bulk copy is checked against the tensor before it is issued
         const char* src = S->data + d.row * S->stride_bytes + size_t(c0) * esz;
@@ -281,8 +293,71 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
           mbar_arrive(&full[s]);
         }
         ++it;
+        return true;
+      };
+      // Queues items [i0, i1) of a family (item = row * units per row + unit),
+      // walking rows and units without a division per item.
+      auto walk = [&](bool tgt, int64_t i0, int64_t i1) {
+        if (i0 >= i1) return;
+        const int upr = tgt ? upr_t : upr_d;
+        int64_t row = i0 / upr;
+        int unit = int(i0 - row * upr);
+        for (int64_t i = i0; ok && i < i1; ++i) {
+          ok = issue(tgt, row, unit);
+          if (++unit == upr) {
+            unit = 0;
+            ++row;
+          }
+        }
+      };
+
+      if (!a.work) {
+        // fixed shares only: a block of target items, then a block of draft items
+        const int64_t t_lo = items_t * g / G, t_hi = items_t * (g + 1) / G;
+        const int64_t d_lo = items_d * g / G, d_hi = items_d * (g + 1) / G;
+        walk(true, t_lo, t_hi);
+        grid_dependency_wait();  // draft rows need the alignment's flags
+        walk(false, d_lo, d_hi);
+      } else {
+        // A fixed block of the first half of the target items, streamed while
+        // the alignment may still run; then batches of the rest (target items,
+        // then draft items) from the work counter, so that CTAs that started
+        // late or drew less bandwidth take fewer and all finish together.
+        const int64_t per = items_t / 2 / G;
+        walk(true, g * per, (g + 1) * per);
+        grid_dependency_wait();  // the counters, flags and scored columns are ready
+        late = true;
+        const int64_t t_rest = G * per, n_rest_t = items_t - t_rest;
+        const int64_t pool = n_rest_t + items_d;
+        // Guided self-scheduling over kWorkShards sub-pools: CTA g starts on
+        // shard g mod kWorkShards; a draw takes 1/(4 * its CTAs) of what is
+        // left there (within [kGrabMin, kGrabMax] items), so draws are larger
+        // early and small only at the end. A CTA whose shard runs dry moves
+        // on to the next one. The next draw is made while the current batch
+        // is queued, so the counter's round trip never stalls the ring.
+        const int64_t ctas = max(int64_t(1), G / kWorkShards);
+        auto draw_size = [&](int64_t left) -> int64_t {
+          return max(int64_t(R::kGrabMin), min(int64_t(R::kGrabMax), left / (4 * ctas)));
+        };
+        for (int v = 0; ok && v < kWorkShards; ++v) {
+          const int sh = int((g + v) % kWorkShards);
+          const int64_t lo = pool * sh / kWorkShards, n = pool * (sh + 1) / kWorkShards - lo;
+          unsigned long long* ctr = a.work + sh * kWorkStride;
+          int64_t size = v == 0 ? draw_size(n / 2) : int64_t(R::kGrabMin);
+          int64_t base = int64_t(atomicAdd(ctr, (unsigned long long)size));
+          while (ok && base < n) {
+            const int64_t size_next = draw_size(n - base - size);
+            const int64_t next = int64_t(atomicAdd(ctr, (unsigned long long)size_next));
+            const int64_t x0 = lo + base, x1 = lo + min(n, base + size);
+            walk(true, t_rest + x0, t_rest + min(x1, n_rest_t));  // pool: target items first
+            walk(false, max(x0, n_rest_t) - n_rest_t, x1 - n_rest_t);
+            base = next;
+            size = size_next;
+          }
+        }
       }
-      if (!waited) grid_dependency_wait();  // this grid ends after the one before it
+      // nothing left to hand out: the next grid may start as CTAs retire
+      grid_launch_dependents();
       // one end marker per consumer warp
       for (int w = 0; ok && w < kConsumerWarps; ++w) {
         const int s = it % R::kStages;
@@ -296,7 +371,6 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
         mbar_arrive(&full[s]);
         ++it;
       }
-      grid_launch_dependents();
     }
     return;
   }
@@ -312,18 +386,34 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
     const Desc d = desc[s];
     if (d.row < 0) break;
     const char* stage = stages + size_t(s) * R::kStageBytes;
-    float m, sum;
-    if (d.set) {
-      reduce_chunk<DTT>(stage, d, a.t, lane, m, sum);
-    } else {
-      reduce_chunk<DTD>(stage, d, a.d, lane, m, sum);
+    const int cps = d.set ? R::kCpsT : R::kCpsD;
+    const int esz = (d.set ? DTT : DTD) == TT_F32 ? 4 : 2;
+    float m[2], sum[2];
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {  // the unit's chunks, each reduced on its own
+      m[c] = -INFINITY;
+      sum[c] = 0.f;
+      const int lo = c * kChunk;
+      if (c >= cps || lo >= d.n) continue;
+      Desc e = d;
+      e.chunk = d.chunk + c;
+      e.n = min(kChunk, d.n - lo);
+      e.n_smem = max(0, min(kChunk, d.n_smem - lo));
+      e.excl = (d.excl >= lo && d.excl < lo + kChunk) ? d.excl - lo : -1;
+      if (d.set) {
+        reduce_chunk<DTT>(stage + size_t(lo) * esz, e, a.t, lane, m[c], sum[c]);
+      } else {
+        reduce_chunk<DTD>(stage + size_t(lo) * esz, e, a.d, lane, m[c], sum[c]);
+      }
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[s]);  // the stage's bytes are consumed
-    warp_merge_ms(m, sum);
-    if (lane == 0) {
-      const RowSet& S = d.set ? a.t : a.d;
-      S.part[d.row * S.nch + d.chunk] = Partial{m, sum};
+    const RowSet& S = d.set ? a.t : a.d;
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {
+      if (c >= cps || c * kChunk >= d.n) continue;
+      warp_merge_ms(m[c], sum[c]);
+      if (lane == 0) S.part[d.row * S.nch + d.chunk + c] = Partial{m[c], sum[c]};
     }
   }
 }
@@ -353,7 +443,8 @@ cudaError_t launch_rowpass_t(const RowPassArgs& a, cudaStream_t stream, int sm_c
   using R = Ring<DTD, DTT>;
   const int per_sm = resident_per_sm<DTD, DTT>();
   if (per_sm == 0) return cudaErrorNotReady;  // preload_rowpass() was not called
-  const int64_t total = a.items_t + a.items_d;
+  const int64_t total = a.rows_t * ((a.t.nch + R::kCpsT - 1) / R::kCpsT) +
+                        a.rows_d * ((a.d.nch + R::kCpsD - 1) / R::kCpsD);
   if (total == 0) return cudaSuccess;
   const int64_t grid = std::min<int64_t>(total, int64_t(sm_count) * per_sm);
   cudaLaunchConfig_t cfg = {};

@@ -26,6 +26,11 @@ struct Partial {
   float s;
 };
 
+// The row pass hands out work from kWorkShards counters, each on its own
+// 256-byte line, so that no single L2 address serialises every CTA's draws.
+constexpr int kWorkShards = 8;
+constexpr int kWorkStride = 32;  // in 8-byte words
+
 struct Workspace {
   Partial* part_d;   // [n_draft * nch_d]
   Partial* part_t;   // [(n_target + B) * nch_t]
@@ -35,6 +40,8 @@ struct Workspace {
   int32_t* status;   // [B] per-request status between kernels
   int32_t* excl;     // [n_target + B] scored column of each target row (-1: bonus row)
   int32_t* err;      // two words: epoch of a call whose row pass failed, and why
+  unsigned long long* work;  // row-pass work counters (kWorkShards, kWorkStride apart), zeroed
+                             // by the kernel before the row pass
   size_t bytes;
 };
 
@@ -57,6 +64,7 @@ __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_d
   w.status = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * size_t(B)));
   w.excl = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (size_t(n_target) + B)));
   w.err = reinterpret_cast<int32_t*>(take(2 * sizeof(int32_t)));
+  w.work = reinterpret_cast<unsigned long long*>(take(kWorkShards * kWorkStride * sizeof(unsigned long long)));
   w.bytes = off;
   return w;
 }

@@ -28,6 +28,10 @@ struct AlignArgs {
   int32_t* map;
   int32_t* status;
   uint8_t* need;               // needed draft rows (may be NULL)
+  unsigned long long* work;    // row-pass work counters to zero (may be NULL)
+  const int32_t* target_cols;  // scored column of each target position
+  int32_t* excl;               // [n_target + B] written: scored column of each target row
+                               // (-1 for the bonus row), may be NULL
   int warps_per_block, tile_w;
   size_t smem_per_warp;
 };
@@ -46,7 +50,7 @@ struct RowSet {
 
 struct RowPassArgs {
   RowSet d, t;
-  int64_t items_d, items_t;  // rows * chunks of each family (0 = family absent)
+  int64_t rows_d, rows_t;    // rows of each family to stream (0 = family absent)
   const int32_t* excl;       // [target rows] column left out of the sum, or NULL: found
                              // from target_off / target_cols
   int B, n_target;
@@ -54,6 +58,12 @@ struct RowPassArgs {
   const int32_t* target_cols;
   int32_t* err;              // err[0] = epoch of a failed call, err[1] = its TT_REQ_* bits
   int32_t epoch;             // identifies this call
+  const int32_t* excl_late;  // as excl, but written by the grid this one depends on: read
+                             // only after the grid-dependency wait (may be NULL)
+  // Work counter for the items past each CTA's fixed share, zeroed by the grid
+  // this one depends on and read only after the grid-dependency wait; NULL:
+  // every item belongs to a fixed share.
+  unsigned long long* work;
 };
 
 struct DecideArgs {
@@ -85,6 +95,7 @@ struct PrepArgs {
   const int32_t* target_off;
   const int32_t* map;
   uint8_t* need;   // needed-draft-row flags, written from map
+  unsigned long long* work;  // row-pass work counter to zero (may be NULL)
 };
 
 size_t align_smem_per_warp(int max_k, int max_m, int tile_w);
