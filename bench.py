@@ -46,6 +46,9 @@ def parse_args(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["mine", "reference"], default="mine")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--batch", type=int, default=None,
+                    help="requests per GPU (default: the workload's own batch); smaller "
+                         "batches are for profiler captures, not bench lines")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -266,7 +269,7 @@ def run_mine(args):
     name = args.workload
     K = args.steps if args.steps is not None else default_steps(name)
     Wm = max(3, args.warmup)
-    wl = W.make_workload(name, seed=rank, device=str(dev))
+    wl = W.make_workload(name, B=args.batch, seed=rank, device=str(dev))
     inp = tt.device_inputs(wl, dev)
     prm = inp["params"]
     prm.request_base = request_base(rank, wl.B)
@@ -438,7 +441,7 @@ def run_reference(args):
     name = args.workload
     K = args.steps if args.steps is not None else 5
     Wm = max(3, args.warmup)
-    wl = W.make_workload(name, seed=0, device="cpu")
+    wl = W.make_workload(name, B=args.batch, seed=0, device="cpu")
     per_step = {"b1_g4_v32k": 1, "b64_g8_v152k": 4, "b256_g16_v152k_bf16": 2,
                 "dtw_4096x64": 16, "b1024_g8_v201k_bf16": 2}.get(name, 2)
     subs = []

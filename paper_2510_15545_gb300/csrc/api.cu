@@ -188,6 +188,7 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   d.B = batch->B;
   d.n_draft = batch->n_draft;
   d.n_target = batch->n_target;
+  d.max_k = batch->max_k;
   d.max_m = batch->max_m;
   d.mode_transfer_only = 1;
   d.draft_off = batch->draft_off;
@@ -296,6 +297,7 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   d.B = batch->B;
   d.n_draft = batch->n_draft;
   d.n_target = batch->n_target;
+  d.max_k = batch->max_k;
   d.max_m = batch->max_m;
   d.full_q = full_q ? 1 : 0;
   d.draft_off = batch->draft_off;
@@ -393,6 +395,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   d.B = batch->B;
   d.n_draft = batch->n_draft;
   d.n_target = batch->n_target;
+  d.max_k = batch->max_k;
   d.max_m = batch->max_m;
   d.full_q = full_q ? 1 : 0;
   d.draft_off = batch->draft_off;
@@ -417,6 +420,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   d.lse = out->lse;
   d.err = ws.err;
   d.epoch = r.epoch;
+  d.warm_ctas = sm_count_current();  // the first CTA on each SM
   if ((e = launch_decide(d, s, pdl)) != cudaSuccess) return cuda_fail(e);
   record(prm, 3, s);
   return TT_OK;

@@ -143,6 +143,39 @@ __device__ __forceinline__ float lane_elem(const uint4& v, int q) {
   }
 }
 
+__device__ __forceinline__ uint32_t max_bf16x2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+// Largest raw logit of one lane's share of a whole chunk. The scale is
+// positive and rounding is monotonic, so max(z * scale) = max(z) * scale
+// exactly: the maximum is taken on the raw values (bf16 two at a time).
+template <int DT>
+__device__ __forceinline__ float raw_max_plain(const uint4* sv, int lane) {
+  constexpr int VEC = DT == TT_F32 ? 4 : 8;
+  constexpr int NV = kChunk / (VEC * 32);
+  if constexpr (DT == TT_F32) {
+    float m = -INFINITY;
+#pragma unroll 4
+    for (int v = 0; v < NV; ++v) {
+      const uint4 w = sv[v * 32 + lane];
+      m = fmaxf(m, fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)),
+                         fmaxf(__uint_as_float(w.z), __uint_as_float(w.w))));
+    }
+    return m;
+  } else {
+    uint32_t m2 = 0xff80ff80u;  // two bf16 -inf
+#pragma unroll 4
+    for (int v = 0; v < NV; ++v) {
+      const uint4 w = sv[v * 32 + lane];
+      m2 = max_bf16x2(m2, max_bf16x2(max_bf16x2(w.x, w.y), max_bf16x2(w.z, w.w)));
+    }
+    return fmaxf(__uint_as_float(m2 << 16), __uint_as_float(m2 & 0xffff0000u));
+  }
+}
+
 // One consumer warp reduces one chunk held in shared memory (plus a ragged
 // tail of fewer than 16 bytes read directly) to (max, sum of 2^(s - max)).
 // The stage is read twice (max, then sum) rather than held in registers.
@@ -151,13 +184,17 @@ __device__ __forceinline__ void reduce_stage(const uint4* sv, const Desc& d, flo
                                              int lane, float& mx, float& sum) {
   constexpr int VEC = DT == TT_F32 ? 4 : 8;  // elements per 16 bytes
   constexpr int NV = kChunk / (VEC * 32);    // 16-byte vectors per lane
+  if constexpr (PLAIN) {
+    mx = fmaxf(mx, raw_max_plain<DT>(sv, lane) * scale);
+  } else {
 #pragma unroll 4
-  for (int v = 0; v < NV; ++v) {
-    const uint4 w = sv[v * 32 + lane];
+    for (int v = 0; v < NV; ++v) {
+      const uint4 w = sv[v * 32 + lane];
 #pragma unroll
-    for (int q = 0; q < VEC; ++q) {
-      const int e = (v * 32 + lane) * VEC + q;
-      if (PLAIN || (e < d.n_smem && e != d.excl)) mx = fmaxf(mx, lane_elem<DT>(w, q) * scale);
+      for (int q = 0; q < VEC; ++q) {
+        const int e = (v * 32 + lane) * VEC + q;
+        if (e < d.n_smem && e != d.excl) mx = fmaxf(mx, lane_elem<DT>(w, q) * scale);
+      }
     }
   }
   if (mx == -INFINITY) return;
@@ -317,6 +354,9 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
         const int64_t d_lo = items_d * g / G, d_hi = items_d * (g + 1) / G;
         walk(true, t_lo, t_hi);
         grid_dependency_wait();  // draft rows need the alignment's flags
+        // the next grid may start now (the alignment grid is complete): its CTAs
+        // are small enough to sit beside these and wait there for this grid's end
+        grid_launch_dependents();
         walk(false, d_lo, d_hi);
       } else {
         // A fixed block of the first half of the target items, streamed while
@@ -327,6 +367,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
         walk(true, g * per, (g + 1) * per);
         grid_dependency_wait();  // the counters, flags and scored columns are ready
         late = true;
+        grid_launch_dependents();  // as above
         const int64_t t_rest = G * per, n_rest_t = items_t - t_rest;
         const int64_t pool = n_rest_t + items_d;
         // Guided self-scheduling over kWorkShards sub-pools: CTA g starts on
@@ -356,8 +397,6 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
           }
         }
       }
-      // nothing left to hand out: the next grid may start as CTAs retire
-      grid_launch_dependents();
       // one end marker per consumer warp
       for (int w = 0; ok && w < kConsumerWarps; ++w) {
         const int s = it % R::kStages;
@@ -376,6 +415,9 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
   }
 
   // -------------------------------------------------------------- consumers
+  // (one thread's launch_dependents counts for its whole CTA: only the
+  // producer lane gives it, after its grid-dependency wait, because the next
+  // grid reads the alignment's outputs before its own wait)
   for (int it = warp;; it += kConsumerWarps) {
     const int s = it % R::kStages;
     const uint32_t par = (it / R::kStages) & 1;
@@ -429,6 +471,9 @@ cudaError_t preload_t() {
   using R = Ring<DTD, DTT>;
   cudaError_t e = cudaFuncSetAttribute(rowpass_kernel<DTD, DTT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, int(R::kSmem));
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(rowpass_kernel<DTD, DTT>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           int(cudaSharedmemCarveoutMaxShared));
   if (e != cudaSuccess) return e;
   int per_sm = 0;
   e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rowpass_kernel<DTD, DTT>, kThreads,

@@ -67,7 +67,7 @@ struct RowPassArgs {
 };
 
 struct DecideArgs {
-  int B, n_draft, n_target, max_m, full_q, mode_transfer_only;
+  int B, n_draft, n_target, max_k, max_m, full_q, mode_transfer_only;
   const int32_t* draft_off;
   const int32_t* draft_cols;
   const int32_t* target_off;
@@ -87,6 +87,7 @@ struct DecideArgs {
   float* q_hat_out;
   float* p_hat;
   float* lse;
+  int warm_ctas;  // CTAs b < warm_ctas run a warming pass before the wait (see decide.cu)
 };
 
 struct PrepArgs {
