@@ -24,6 +24,7 @@ _lib = None
 
 # Status bits (shared meaning with the CUDA library, defined independently).
 ST_ID_RANGE, ST_TOO_LONG, ST_EMPTY, ST_BAD_OFFSETS = 1, 2, 4, 8
+ST_NO_MATCH, ST_INCONSISTENT = 128, 256
 
 
 def build(force: bool = False) -> str:
@@ -65,6 +66,12 @@ def lib():
         L.tto_verify.argtypes = [i32, P, P, P, P, i32, i64, i32, f64, P, P, P, i32, i64, i32,
                                  f64, i32, u64, u64, P, P, P, P, P, P]
         L.tto_verify.restype = None
+        L.tto_encode.argtypes = [i32, P, P, P, P, i32, P, P, i32, i32, i32, i32, P, P, P]
+        L.tto_encode.restype = None
+        L.tto_consistency.argtypes = [i32, P, P, P, P, P, P, i32, P, P, i32, i32, i32, P]
+        L.tto_consistency.restype = None
+        L.tto_dpos_hist.argtypes = [i32, P, P, P, P, P, i32, i32, P]
+        L.tto_dpos_hist.restype = None
         _lib = L
     return _lib
 
@@ -227,4 +234,53 @@ def step(wl, *, window: Optional[int] = None, temp_draft: Optional[float] = None
     bad = status != 0
     out["accepted"] = np.where(bad, 0, out["accepted"]).astype(np.int32)
     out["next_token"] = np.where(bad, -1, out["next_token"]).astype(np.int32)
+    return out
+
+
+def encode(draft_off, draft_ids, vd_blob, vd_off, vt_blob, vt_off, max_m: int,
+           max_bytes: int = 2048, capacity: Optional[int] = None) -> dict:
+    """Re-encoding T = encode_t(decode_d(D)) by greedy longest match (tto_encode)."""
+    draft_off, draft_ids = _i32(draft_off), _i32(draft_ids)
+    vd_blob = np.ascontiguousarray(vd_blob, dtype=np.uint8)
+    vt_blob = np.ascontiguousarray(vt_blob, dtype=np.uint8)
+    vd_off = np.ascontiguousarray(vd_off, dtype=np.int64)
+    vt_off = np.ascontiguousarray(vt_off, dtype=np.int64)
+    B = len(draft_off) - 1
+    if capacity is None:
+        capacity = B * max_m
+    target_off = np.zeros(B + 1, np.int32)
+    target_ids = np.full(max(capacity, 1), -1, np.int32)
+    status = np.zeros(max(B, 1), np.int32)
+    lib().tto_encode(B, _p(draft_off), _p(draft_ids), _p(vd_blob), _p(vd_off), len(vd_off) - 1,
+                     _p(vt_blob), _p(vt_off), len(vt_off) - 1, int(max_m), int(max_bytes),
+                     int(capacity), _p(target_off), _p(target_ids), _p(status))
+    return dict(target_off=target_off, target_ids=target_ids[:target_off[-1]], status=status[:B])
+
+
+def consistency(draft_off, draft_ids, target_off, target_ids, vd_blob, vd_off, vt_blob, vt_off,
+                max_k: int, max_m: int) -> np.ndarray:
+    """Lemma 1 as a check: status per request (tto_consistency)."""
+    draft_off, draft_ids = _i32(draft_off), _i32(draft_ids)
+    target_off, target_ids = _i32(target_off), _i32(target_ids)
+    vd_blob = np.ascontiguousarray(vd_blob, dtype=np.uint8)
+    vt_blob = np.ascontiguousarray(vt_blob, dtype=np.uint8)
+    vd_off = np.ascontiguousarray(vd_off, dtype=np.int64)
+    vt_off = np.ascontiguousarray(vt_off, dtype=np.int64)
+    B = len(draft_off) - 1
+    status = np.zeros(max(B, 1), np.int32)
+    lib().tto_consistency(B, _p(draft_off), _p(draft_ids), _p(target_off), _p(target_ids),
+                          _p(vd_blob), _p(vd_off), len(vd_off) - 1, _p(vt_blob), _p(vt_off),
+                          len(vt_off) - 1, int(max_k), int(max_m), _p(status))
+    return status[:B]
+
+
+def dpos_hist(draft_off, target_off, path, path_len, mp, mode: int, n_bins: int,
+              hist=None) -> np.ndarray:
+    """Delta-pos histogram of the DTW paths (mode 0) or of the map (mode 1)."""
+    draft_off, target_off = _i32(draft_off), _i32(target_off)
+    path = _i32(np.asarray(path).reshape(-1))
+    path_len, mp = _i32(path_len), _i32(mp if len(mp) else np.zeros(1, np.int32))
+    out = np.zeros(n_bins, np.int64) if hist is None else np.ascontiguousarray(hist, np.int64)
+    lib().tto_dpos_hist(len(draft_off) - 1, _p(draft_off), _p(target_off), _p(path),
+                        _p(path_len), _p(mp), int(mode), int(n_bins), _p(out))
     return out

@@ -34,6 +34,8 @@
 #define ST_TOO_LONG 2
 #define ST_EMPTY 4
 #define ST_BAD_OFFSETS 8
+#define ST_NO_MATCH 128
+#define ST_INCONSISTENT 256
 #define MAX_K 256
 #define MAX_M 512
 #define MAX_TOKEN_BYTES 256
@@ -400,4 +402,181 @@ void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols
   free(p);
   free(q);
   free(r);
+}
+
+/* ------------------------------------------------------------ re-encoding */
+
+/* The target vocabulary sorted by (byte string, id), so that a string's
+ * smallest id is the first of its run. The sort's comparator reads the table
+ * through these file-level pointers (the oracle is single-threaded). */
+static const uint8_t* g_sort_bytes;
+static const int64_t* g_sort_off;
+
+static int cmp_bytes(const uint8_t* a, int64_t na, const uint8_t* b, int64_t nb) {
+  int64_t n = na < nb ? na : nb;
+  int c = n > 0 ? memcmp(a, b, (size_t)n) : 0;
+  if (c != 0) return c;
+  return na < nb ? -1 : (na > nb ? 1 : 0);
+}
+
+static int cmp_token_ids(const void* x, const void* y) {
+  int32_t a = *(const int32_t*)x, b = *(const int32_t*)y;
+  int c = cmp_bytes(g_sort_bytes + g_sort_off[a], g_sort_off[a + 1] - g_sort_off[a],
+                    g_sort_bytes + g_sort_off[b], g_sort_off[b + 1] - g_sort_off[b]);
+  if (c != 0) return c;
+  return a < b ? -1 : (a > b ? 1 : 0);
+}
+
+/* Smallest id of vt spelling s[0..n), or -1 (binary search over the sorted ids). */
+static int32_t find_token(const int32_t* sorted, int32_t Vt, const uint8_t* vt_bytes,
+                          const int64_t* vt_off, const uint8_t* s, int64_t n) {
+  int32_t lo = 0, hi = Vt;  /* first position whose string is >= s */
+  while (lo < hi) {
+    int32_t mid = lo + (hi - lo) / 2;
+    int32_t v = sorted[mid];
+    if (cmp_bytes(vt_bytes + vt_off[v], vt_off[v + 1] - vt_off[v], s, n) < 0) lo = mid + 1;
+    else hi = mid;
+  }
+  if (lo < Vt) {
+    int32_t v = sorted[lo];
+    if (cmp_bytes(vt_bytes + vt_off[v], vt_off[v + 1] - vt_off[v], s, n) == 0) return v;
+  }
+  return -1;
+}
+
+void tto_encode(int32_t B, const int32_t* draft_off, const int32_t* draft_ids,
+                const uint8_t* vd_bytes, const int64_t* vd_off, int32_t Vd,
+                const uint8_t* vt_bytes, const int64_t* vt_off, int32_t Vt,
+                int32_t max_m, int32_t max_bytes, int32_t capacity,
+                int32_t* target_off, int32_t* target_ids, int32_t* status) {
+  int32_t* sorted = (int32_t*)malloc(sizeof(int32_t) * (size_t)(Vt > 0 ? Vt : 1));
+  int64_t longest = 0;
+  for (int32_t v = 0; v < Vt; ++v) {
+    sorted[v] = v;
+    if (vt_off[v + 1] - vt_off[v] > longest) longest = vt_off[v + 1] - vt_off[v];
+  }
+  g_sort_bytes = vt_bytes;
+  g_sort_off = vt_off;
+  qsort(sorted, (size_t)Vt, sizeof(int32_t), cmp_token_ids);
+
+  uint8_t* text = (uint8_t*)malloc((size_t)(max_bytes > 0 ? max_bytes : 1));
+  int32_t* toks = (int32_t*)malloc(sizeof(int32_t) * (size_t)(max_m > 0 ? max_m : 1));
+  int64_t end_all = 0; /* tokens of every earlier request, written or not */
+  target_off[0] = 0;
+  for (int32_t b = 0; b < B; ++b) {
+    int32_t st = 0, m = 0;
+    if (!offsets_ok(draft_off, b)) {
+      st = ST_BAD_OFFSETS;
+    } else {
+      int32_t d0 = draft_off[b], k = draft_off[b + 1] - d0;
+      int64_t n = 0;
+      if (k == 0) st |= ST_EMPTY;
+      for (int32_t i = 0; i < k; ++i) {
+        int32_t id = draft_ids[d0 + i];
+        if (id < 0 || id >= Vd) { st |= ST_ID_RANGE; continue; }
+        n += vd_off[id + 1] - vd_off[id];
+      }
+      if (st == 0 && n > max_bytes) st |= ST_TOO_LONG;
+      if (st == 0) {
+        /* decode_d: concatenate the draft tokens' bytes */
+        int64_t at = 0;
+        for (int32_t i = 0; i < k; ++i) {
+          int32_t id = draft_ids[d0 + i];
+          int64_t len = vd_off[id + 1] - vd_off[id];
+          if (len > 0) memcpy(text + at, vd_bytes + vd_off[id], (size_t)len);
+          at += len;
+        }
+        /* encode_t: greedy longest match */
+        int64_t p = 0;
+        while (p < n && st == 0) {
+          int64_t L = n - p < longest ? n - p : longest;
+          int32_t v = -1;
+          for (; L >= 1; --L) {
+            v = find_token(sorted, Vt, vt_bytes, vt_off, text + p, L);
+            if (v >= 0) break;
+          }
+          if (v < 0) { st |= ST_NO_MATCH; break; }
+          if (m >= max_m) { st |= ST_TOO_LONG; break; }
+          toks[m++] = v;
+          p += L;
+        }
+      }
+    }
+    if (st != 0) m = 0;
+    end_all += m;
+    if (st == 0 && end_all > capacity) { st |= ST_TOO_LONG; m = 0; }
+    for (int32_t j = 0; j < m; ++j) target_ids[target_off[b] + j] = toks[j];
+    target_off[b + 1] = target_off[b] + m;
+    status[b] = st;
+  }
+  free(text);
+  free(toks);
+  free(sorted);
+}
+
+void tto_consistency(int32_t B, const int32_t* draft_off, const int32_t* draft_ids,
+                     const int32_t* target_off, const int32_t* target_ids,
+                     const uint8_t* vd_bytes, const int64_t* vd_off, int32_t Vd,
+                     const uint8_t* vt_bytes, const int64_t* vt_off, int32_t Vt,
+                     int32_t max_k, int32_t max_m, int32_t* status) {
+  for (int32_t b = 0; b < B; ++b) {
+    if (!offsets_ok(draft_off, b) || !offsets_ok(target_off, b)) {
+      status[b] = ST_BAD_OFFSETS;
+      continue;
+    }
+    int32_t d0 = draft_off[b], k = draft_off[b + 1] - d0;
+    int32_t t0 = target_off[b], m = target_off[b + 1] - t0;
+    int32_t st = 0;
+    if (k > max_k || m > max_m) st |= ST_TOO_LONG;
+    for (int32_t i = 0; i < k; ++i)
+      if (draft_ids[d0 + i] < 0 || draft_ids[d0 + i] >= Vd) st |= ST_ID_RANGE;
+    for (int32_t j = 0; j < m; ++j)
+      if (target_ids[t0 + j] < 0 || target_ids[t0 + j] >= Vt) st |= ST_ID_RANGE;
+    if (st == 0) {
+      /* walk both byte streams side by side */
+      int32_t i = 0, j = 0;
+      int64_t pi = 0, pj = 0; /* position inside token i / token j */
+      for (;;) {
+        while (i < k && pi == vd_off[draft_ids[d0 + i] + 1] - vd_off[draft_ids[d0 + i]]) {
+          ++i;
+          pi = 0;
+        }
+        while (j < m && pj == vt_off[target_ids[t0 + j] + 1] - vt_off[target_ids[t0 + j]]) {
+          ++j;
+          pj = 0;
+        }
+        if (i == k || j == m) {
+          if (i != k || j != m) st |= ST_INCONSISTENT; /* one string is longer */
+          break;
+        }
+        if (vd_bytes[vd_off[draft_ids[d0 + i]] + pi] != vt_bytes[vt_off[target_ids[t0 + j]] + pj]) {
+          st |= ST_INCONSISTENT;
+          break;
+        }
+        ++pi;
+        ++pj;
+      }
+    }
+    status[b] = st;
+  }
+}
+
+void tto_dpos_hist(int32_t B, const int32_t* draft_off, const int32_t* target_off,
+                   const int32_t* path, const int32_t* path_len, const int32_t* map,
+                   int32_t mode, int32_t n_bins, int64_t* hist) {
+  for (int32_t b = 0; b < B; ++b) {
+    if (path_len[b] <= 0) continue;
+    if (mode == 0) {
+      const int32_t* pp = path + 2 * ((int64_t)draft_off[b] + target_off[b]);
+      for (int32_t x = 0; x < path_len[b]; ++x) {
+        int32_t d = abs(pp[2 * x] - pp[2 * x + 1]);
+        hist[d < n_bins - 1 ? d : n_bins - 1] += 1;
+      }
+    } else {
+      for (int32_t j = 0; j < target_off[b + 1] - target_off[b]; ++j) {
+        int32_t d = abs(map[target_off[b] + j] - j);
+        hist[d < n_bins - 1 ? d : n_bins - 1] += 1;
+      }
+    }
+  }
 }

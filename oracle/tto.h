@@ -75,6 +75,43 @@ void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols
                 int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
                 int32_t* status, int32_t* boundary);
 
+/* ------------------------------------------------------------ re-encoding */
+
+/* Re-encoding (§4.2; App. A.1, Lemma 1): T_b = encode_t(decode_d(D_b)).
+ * decode_d concatenates the byte strings of the draft tokens; encode_t is
+ * greedy longest match over vt: at each position the longest token of vt that
+ * spells the next bytes (the smallest id among tokens with equal strings;
+ * empty tokens never match). Per request: status 8 bad draft offsets, 1 a
+ * draft id out of range, 4 no draft token, 2 decoded string longer than
+ * max_bytes or more than max_m target tokens, 128 some position that no token
+ * of vt spells. A request that fails writes no tokens. Requests are laid out in
+ * order in target_ids; a request whose tokens would end past `capacity`
+ * (counting every earlier request's tokens, written or not) is not written and
+ * gets status 2. target_off[b+1] = target_off[b] + (tokens written for b). */
+void tto_encode(int32_t B, const int32_t* draft_off, const int32_t* draft_ids,
+                const uint8_t* vd_bytes, const int64_t* vd_off, int32_t Vd,
+                const uint8_t* vt_bytes, const int64_t* vt_off, int32_t Vt,
+                int32_t max_m, int32_t max_bytes, int32_t capacity,
+                int32_t* target_off, int32_t* target_ids, int32_t* status);
+
+/* Lemma 1 (App. A.1) as a check: decode_t(T_b) == decode_d(D_b) byte for byte.
+ * Status bits: 8 bad offsets, 1 id out of range, 2 k > max_k or m > max_m,
+ * 256 the two byte strings differ. */
+void tto_consistency(int32_t B, const int32_t* draft_off, const int32_t* draft_ids,
+                     const int32_t* target_off, const int32_t* target_ids,
+                     const uint8_t* vd_bytes, const int64_t* vd_off, int32_t Vd,
+                     const uint8_t* vt_bytes, const int64_t* vt_off, int32_t Vt,
+                     int32_t max_k, int32_t max_m, int32_t* status);
+
+/* Delta-pos (§4.1, App. G): the position deviation |i - j| of matched tokens,
+ * counted into hist[min(|i - j|, n_bins - 1)] (hist is added to, not cleared).
+ * mode 0: every (i, j) on each request's DTW path; mode 1: every target
+ * position j with its mapped draft index map[j]. Requests with path_len[b] == 0
+ * (failed alignments) add nothing. */
+void tto_dpos_hist(int32_t B, const int32_t* draft_off, const int32_t* target_off,
+                   const int32_t* path, const int32_t* path_len, const int32_t* map,
+                   int32_t mode, int32_t n_bins, int64_t* hist);
+
 #ifdef __cplusplus
 }
 #endif
