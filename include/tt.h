@@ -72,6 +72,12 @@ typedef enum {
                                     the step's results are not valid */
 #define TT_REQ_INTERNAL 64       /* an internal bounds check in a kernel failed (the access
                                     was skipped); the step's results are not valid */
+#define TT_REQ_NO_MATCH 128      /* tt_encode: some position of the decoded draft string is
+                                    spelled by no token of the target vocabulary */
+#define TT_REQ_INCONSISTENT 256  /* tt_consistency: decode_t(T) != decode_d(D) (Lemma 1) */
+
+#define TT_MAX_ENCODE_BYTES 2048 /* longest decoded draft string tt_encode takes per request */
+#define TT_MAX_DPOS_BINS 4096    /* most bins of tt_dpos_hist */
 
 typedef enum { TT_F32 = 0, TT_BF16 = 1 } tt_dtype;
 
@@ -223,6 +229,67 @@ tt_status tt_step_noalloc(const tt_batch* batch, const tt_vocab* vd, const tt_vo
                           const tt_step_out* out, void* stream);
 
 /* Static text for a tt_status. */
+/* ------------------------------------------------------------------------
+ * Re-encoding and its checks (§4.2; App. A.1, Lemma 1; §4.1 and App. G).
+ * ---------------------------------------------------------------------- */
+
+/* Size of the re-encoding index of a vocabulary with n_tokens tokens and
+ * n_bytes bytes of strings (an open-addressing table of every prefix of every
+ * token, 16 bytes per slot, at most half full). */
+size_t tt_vocab_index_bytes(int32_t n_tokens, int64_t n_bytes);
+
+/* Builds the re-encoding index of a target vocabulary. HOST pointers in and
+ * out: `bytes`/`offsets` as in tt_vocab, `index` a host buffer of
+ * tt_vocab_index_bytes() bytes; the caller copies it to the device once (it
+ * is position-independent) and passes the device copy to tt_encode. Among
+ * tokens with equal strings the smallest id is kept; empty tokens are left
+ * out. TT_ERR_UNSUPPORTED for a token longer than TT_MAX_TOKEN_BYTES, or in
+ * the (never observed) event of two different prefixes longer than 8 bytes
+ * with equal 64-bit fingerprints. Synchronous, deterministic. */
+tt_status tt_vocab_index_build(const uint8_t* bytes, const int64_t* offsets, int32_t n_tokens,
+                               void* index, size_t index_bytes);
+
+/* Scratch of tt_encode for B requests of at most max_m target tokens. */
+size_t tt_encode_workspace_bytes(int32_t B, int32_t max_m);
+
+/* T_b = encode_t(decode_d(D_b)) for every request (§4.2, App. A.1): the draft
+ * tokens' byte strings (in vd) concatenated, then greedy longest match over
+ * the target vocabulary (vt, with its index vt_index from
+ * tt_vocab_index_build): at each position the longest target token spelling
+ * the next bytes, the smallest id among equal strings. This is the tokenizer
+ * of the synthetic workloads; a learned tokenizer's merges are not modelled.
+ * Inputs: B, n_draft (= draft_off[B]), draft_off [B+1], draft_ids [n_draft]
+ * (device). Outputs (device):
+ * target_off [B+1], target_ids [capacity], status [B]. Status bits: BAD_OFFSETS,
+ * ID_OUT_OF_RANGE (a draft id), EMPTY (k = 0), TOO_LONG (decoded string longer
+ * than TT_MAX_ENCODE_BYTES, more than max_m tokens, or the request's tokens
+ * would end past `capacity` counting every earlier request's tokens, written
+ * or not), NO_MATCH. A failed request writes no tokens:
+ * target_off[b+1] = target_off[b] + (tokens written for b). */
+tt_status tt_encode(int32_t B, int32_t n_draft, const int32_t* draft_off, const int32_t* draft_ids,
+                    const tt_vocab* vd, const tt_vocab* vt, const void* vt_index,
+                    int32_t max_m, int32_t capacity, int32_t* target_off,
+                    int32_t* target_ids, int32_t* status, void* workspace,
+                    size_t workspace_bytes, void* stream);
+
+/* Lemma 1 (App. A.1) as a check on any (D, T), e.g. a T re-encoded by the
+ * caller's own tokenizer: status[b] = 0 when the bytes of T_b are those of
+ * D_b, TT_REQ_INCONSISTENT when they differ, BAD_OFFSETS / ID_OUT_OF_RANGE /
+ * TOO_LONG (k > max_k or m > max_m) otherwise. Uses ids, not cols. */
+tt_status tt_consistency(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
+                         int32_t* status, void* stream);
+
+/* Delta-pos (§4.1, App. G), the position deviation of DTW-matched tokens,
+ * counted into hist[min(delta, n_bins - 1)] (int64, device, ADDED to: zero it
+ * before the first call; many steps can be accumulated). mode 0: delta = |i - j|
+ * for every pair on each request's path (tt_align's path / path_len); mode 1:
+ * delta = |map[j] - j| for every target position. Requests with path_len[b] <= 0
+ * add nothing. n_bins in [1, TT_MAX_DPOS_BINS]. The paper chooses w where the
+ * cumulative distribution of delta (taken with no band) reaches 0.9. */
+tt_status tt_dpos_hist(const tt_batch* batch, const int32_t* path, const int32_t* path_len,
+                       const int32_t* map, int32_t mode, int32_t n_bins, int64_t* hist,
+                       void* stream);
+
 const char* tt_status_string(tt_status s);
 
 /* cudaError_t of the last failed launch in this process (0 if none). */

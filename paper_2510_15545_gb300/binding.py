@@ -20,6 +20,8 @@ c_i32, c_i64, c_u64, c_f32, c_p = (ctypes.c_int32, ctypes.c_int64, ctypes.c_uint
 TT_OK, TT_ERR_INVALID_ARG, TT_ERR_UNSUPPORTED, TT_ERR_CUDA = 0, 1, 2, 3
 TT_REQ_ID_OUT_OF_RANGE, TT_REQ_TOO_LONG, TT_REQ_EMPTY, TT_REQ_BAD_OFFSETS, TT_REQ_NOT_FINITE = (
     1, 2, 4, 8, 16)
+TT_REQ_NO_MATCH, TT_REQ_INCONSISTENT = 128, 256
+TT_MAX_ENCODE_BYTES, TT_MAX_DPOS_BINS = 2048, 4096
 TT_F32, TT_BF16 = 0, 1
 TT_MAX_K, TT_MAX_M, TT_MAX_TOKEN_BYTES = 256, 512, 256
 
@@ -58,7 +60,9 @@ class _StepOut(ctypes.Structure):
 
 _lib = None
 EXPORTS = ("tt_workspace_bytes", "tt_align", "tt_transfer", "tt_verify", "tt_step",
-           "tt_step_noalloc", "tt_status_string", "tt_last_cuda_error", "tt_version")
+           "tt_step_noalloc", "tt_status_string", "tt_last_cuda_error", "tt_version",
+           "tt_vocab_index_bytes", "tt_vocab_index_build", "tt_encode_workspace_bytes",
+           "tt_encode", "tt_consistency", "tt_dpos_hist")
 TT_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
@@ -102,6 +106,19 @@ def load(build_if_missing: bool = False):
     L.tt_last_cuda_error.restype = c_i32
     L.tt_version.argtypes = []
     L.tt_version.restype = c_i32
+    L.tt_vocab_index_bytes.argtypes = [c_i32, c_i64]
+    L.tt_vocab_index_bytes.restype = ctypes.c_size_t
+    L.tt_vocab_index_build.argtypes = [c_p, c_p, c_i32, c_p, ctypes.c_size_t]
+    L.tt_vocab_index_build.restype = c_i32
+    L.tt_encode_workspace_bytes.argtypes = [c_i32, c_i32]
+    L.tt_encode_workspace_bytes.restype = ctypes.c_size_t
+    L.tt_encode.argtypes = [c_i32, c_i32, c_p, c_p, P(_Vocab), P(_Vocab), c_p, c_i32, c_i32,
+                            c_p, c_p, c_p, c_p, ctypes.c_size_t, c_p]
+    L.tt_encode.restype = c_i32
+    L.tt_consistency.argtypes = [P(_Batch), P(_Vocab), P(_Vocab), c_p, c_p]
+    L.tt_consistency.restype = c_i32
+    L.tt_dpos_hist.argtypes = [P(_Batch), c_p, c_p, c_p, c_i32, c_i32, c_p, c_p]
+    L.tt_dpos_hist.restype = c_i32
     _lib = L
     return L
 
@@ -412,3 +429,73 @@ def device_inputs(wl, device="cuda") -> dict:
                 draft_logits=wl.draft_logits.to(device), target_logits=wl.target_logits.to(device),
                 params=Params(window=wl.spec.window, temp_draft=wl.spec.temp_draft,
                               temp_target=wl.spec.temp_target, seed=wl.spec.seed))
+
+
+# ------------------------------------------------ re-encoding and its checks
+
+def vocab_index(blob, offsets, device="cuda") -> torch.Tensor:
+    """Re-encoding index of a target vocabulary (tt_vocab_index_build on host
+    arrays), copied to the device once; pass it to tt_encode."""
+    import numpy as np
+    blob = np.ascontiguousarray(np.asarray(blob, dtype=np.uint8))
+    offsets = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    n_tokens = len(offsets) - 1
+    L = load()
+    nbytes = int(L.tt_vocab_index_bytes(n_tokens, int(offsets[-1]) if n_tokens > 0 else 0))
+    host = np.zeros(nbytes, np.uint8)
+    code = L.tt_vocab_index_build(blob.ctypes.data if blob.size else None, offsets.ctypes.data,
+                                  n_tokens, host.ctypes.data, nbytes)
+    _check("tt_vocab_index_build", code)
+    return torch.from_numpy(host).to(device)
+
+
+def tt_encode_workspace_bytes(B: int, max_m: int) -> int:
+    return int(load().tt_encode_workspace_bytes(int(B), int(max_m)))
+
+
+def tt_encode(draft_off: torch.Tensor, draft_ids: torch.Tensor, vd: VocabTable, vt: VocabTable,
+              vt_index: torch.Tensor, max_m: int, *, capacity: Optional[int] = None, out=None,
+              ws=None, stream=None) -> dict:
+    """T_b = encode_t(decode_d(D_b)) on the device; returns target_off, target_ids
+    (capacity long) and status."""
+    dev = draft_off.device
+    B = draft_off.numel() - 1
+    n_draft = draft_ids.numel()
+    if capacity is None:
+        capacity = B * int(max_m)
+    o = dict(out or {})
+    o.setdefault("target_off", _empty(B + 1, torch.int32, dev))
+    o.setdefault("target_ids", _empty(capacity, torch.int32, dev))
+    o.setdefault("status", _empty(B, torch.int32, dev))
+    if ws is None:
+        ws = torch.empty(max(tt_encode_workspace_bytes(B, max_m), 256), dtype=torch.uint8,
+                         device=dev)
+    code = load().tt_encode(B, n_draft, _ptr(draft_off), _ptr(draft_ids), ctypes.byref(vd._c()),
+                            ctypes.byref(vt._c()), _ptr(vt_index), int(max_m), int(capacity),
+                            _ptr(o["target_off"]), _ptr(o["target_ids"]), _ptr(o["status"]),
+                            _ptr(ws), ws.numel(), _stream(stream))
+    _check("tt_encode", code)
+    return o
+
+
+def tt_consistency(batch: Batch, vd: VocabTable, vt: VocabTable, *, status=None,
+                   stream=None) -> torch.Tensor:
+    """Lemma-1 byte check of (D, T) per request."""
+    st = status if status is not None else _empty(batch.B, torch.int32, batch.draft_off.device)
+    code = load().tt_consistency(ctypes.byref(batch._c()), ctypes.byref(vd._c()),
+                                 ctypes.byref(vt._c()), _ptr(st), _stream(stream))
+    _check("tt_consistency", code)
+    return st
+
+
+def tt_dpos_hist(batch: Batch, path: torch.Tensor, path_len: torch.Tensor,
+                 map: Optional[torch.Tensor], mode: int, n_bins: int, *,
+                 hist: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Delta-pos histogram of the alignment paths (mode 0) or the map (mode 1),
+    added to `hist` (a zeroed int64 tensor is made when none is given)."""
+    dev = batch.draft_off.device
+    h = hist if hist is not None else torch.zeros(int(n_bins), dtype=torch.int64, device=dev)
+    code = load().tt_dpos_hist(ctypes.byref(batch._c()), _ptr(path), _ptr(path_len), _ptr(map),
+                               int(mode), int(n_bins), _ptr(h), _stream(stream))
+    _check("tt_dpos_hist", code)
+    return h

@@ -135,6 +135,10 @@ tt_status fill_align_args(const tt_batch* bt, const tt_vocab* vd, const tt_vocab
 
 }  // namespace
 
+namespace tt {
+tt_status record_cuda_error(cudaError_t e) { return cuda_fail(e); }
+}  // namespace tt
+
 extern "C" {
 
 size_t tt_workspace_bytes(const tt_batch* batch, int32_t V_d, int32_t V_t) {

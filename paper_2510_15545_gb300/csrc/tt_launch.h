@@ -113,4 +113,7 @@ cudaError_t preload_align();
 cudaError_t preload_rowpass();
 cudaError_t preload_decide();
 
+// Records a failed CUDA call for tt_last_cuda_error() and returns TT_ERR_CUDA.
+tt_status record_cuda_error(cudaError_t e);
+
 }  // namespace tt
