@@ -51,6 +51,8 @@ def parse_args(argv=None):
                          "batches are for profiler captures, not bench lines")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-reencode", action="store_true",
+                    help="skip timing the re-encoding, Lemma-1 check and delta-pos histogram")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU work budget of the oracle baseline sample")
     return ap.parse_args(argv)
@@ -339,6 +341,8 @@ def run_mine(args):
     if not args.no_e2e:
         e2e = run_e2e(tt, wl, inp, prm, dev, stream, K, ws)
 
+    reenc = None if args.no_reencode else run_reencode(tt, wl, inp, prm, dev, stream, rank, ws)
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         rate, sample, nreq, el = oracle_sample_rate(wl, args.cpu_seconds)
@@ -375,6 +379,8 @@ def run_mine(args):
     }
     if e2e is not None:
         line["e2e"] = e2e
+    if reenc is not None:
+        line["reencode"] = reenc
     if cpu is not None:
         line["cpu_baseline"] = cpu
     if rank == 0:
@@ -382,6 +388,74 @@ def run_mine(args):
     if ws > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def _time_calls(fn, stream, n, warm=3):
+    import torch
+    for _ in range(warm):
+        fn()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(n):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / n  # ms per call
+
+
+def run_reencode(tt, wl, inp, prm, dev, stream, rank, ws):
+    """The re-encoding of the batch's draft strings into target tokens on the
+    device (tt_encode), its Lemma-1 check (tt_consistency) and the delta-pos
+    histogram of the alignment paths (tt_dpos_hist), each timed alone with CUDA
+    events over repeated calls; and, on rank 0, the oracle's re-encoding of the
+    same batch on one host core. Outside the step's timed region: re-encoding
+    precedes the target model's forward, it is not part of a verification step."""
+    import time
+
+    import numpy as np
+    import torch
+    index = tt.vocab_index(wl.vt.blob, wl.vt.off, dev)
+    d_off, d_ids = inp["batch"].draft_off, inp["batch"].draft_ids
+    max_m = 512
+    ws_enc = torch.empty(max(tt.tt_encode_workspace_bytes(wl.B, max_m), 256), dtype=torch.uint8,
+                         device=dev)
+    out = {"target_off": torch.empty(wl.B + 1, dtype=torch.int32, device=dev),
+           "target_ids": torch.empty(wl.B * max_m, dtype=torch.int32, device=dev),
+           "status": torch.empty(wl.B, dtype=torch.int32, device=dev)}
+    enc = lambda: tt.tt_encode(d_off, d_ids, inp["vd"], inp["vt"], index, max_m, out=out,
+                               ws=ws_enc, stream=stream)
+    enc_ms = _time_calls(enc, stream, 200)
+    n_out = int(out["target_off"][-1])
+    ok = int((out["status"] == 0).sum())
+    cons_status = torch.empty(wl.B, dtype=torch.int32, device=dev)
+    cons_ms = _time_calls(lambda: tt.tt_consistency(inp["batch"], inp["vd"], inp["vt"],
+                                                    status=cons_status, stream=stream), stream, 200)
+    prm0 = tt.Params(window=-1, seed=prm.seed)
+    al = tt.tt_align(inp["batch"], inp["vd"], inp["vt"], prm0)
+    hist = torch.zeros(64, dtype=torch.int64, device=dev)
+    dpos_ms = _time_calls(lambda: tt.tt_dpos_hist(inp["batch"], al["path"], al["path_len"],
+                                                  al["map"], 0, 64, hist=hist, stream=stream),
+                          stream, 200)
+    h = tt.tt_dpos_hist(inp["batch"], al["path"], al["path_len"], al["map"], 0, 64).cpu().numpy()
+    cdf = np.cumsum(h) / max(1, h.sum())
+    r = {"draft_tokens": wl.n_draft, "target_tokens": n_out, "requests_ok": ok,
+         "encode_ms_per_batch": enc_ms,
+         "encode_draft_tokens_per_s": wl.n_draft / (enc_ms / 1e3),
+         "consistency_ms_per_batch": cons_ms, "dpos_hist_ms_per_batch": dpos_ms,
+         "dpos_cdf_0.9_at": int(np.searchsorted(cdf, 0.9)),
+         "bound": "latency (dependent L2 probes of the prefix index; a few KB per request)"}
+    if rank == 0 and ws == 1:
+        import oracle
+        oracle.build()
+        t0 = time.process_time()
+        oracle.encode(wl.draft_off, wl.draft_ids, wl.vd.blob, wl.vd.off, wl.vt.blob, wl.vt.off,
+                      max_m)
+        cpu_s = time.process_time() - t0
+        r["cpu_oracle_encode_ms_per_batch"] = cpu_s * 1e3
+        r["cpu_oracle_note"] = ("the oracle re-encodes the whole batch on one host core (its "
+                                "vocabulary sort included, as in one call)")
+    return r
 
 
 def run_e2e(tt, wl, inp, prm, dev, stream, K, ws):

@@ -8,7 +8,8 @@
 // Walking the prefixes of the text at position p one byte at a time, the walk
 // stops at the first prefix no token starts with, so a lookup costs about as
 // many probes as the match is long. One warp per request; a second kernel (one
-// CTA) turns the per-request counts into CSR offsets and compacts the tokens.
+// CTA) turns the per-request counts into CSR offsets, a third compacts the
+// tokens (one warp per request).
 #include <cstdint>
 #include <cstring>
 #include <vector>
@@ -255,7 +256,7 @@ __device__ int64_t block_scan(int64_t v, int64_t* s_warp, int64_t* total) {
   return v + before;
 }
 
-// One CTA: CSR offsets with the capacity rule, then the compaction.
+// One CTA: CSR offsets with the capacity rule.
 __global__ void __launch_bounds__(kFinThreads) encode_finish_kernel(FinArgs a) {
   __shared__ int64_t s_warp[kFinThreads / 32];
   int64_t carry_all = 0, carry_written = 0;
@@ -279,13 +280,17 @@ __global__ void __launch_bounds__(kFinThreads) encode_finish_kernel(FinArgs a) {
       a.target_off[b + 1] = int32_t(end_w);
     }
   }
-  __syncthreads();
-  // compaction: one warp per request
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int b = warp; b < a.B; b += kFinThreads / 32) {
-    const int o0 = a.target_off[b], n = a.target_off[b + 1] - o0;
-    for (int j = lane; j < n; j += 32) a.target_ids[o0 + j] = a.pad_ids[int64_t(b) * a.max_m + j];
-  }
+}
+
+constexpr int kCompactWarps = 8;
+
+// Compaction of the padded tokens into the CSR output: one warp per request.
+__global__ void __launch_bounds__(32 * kCompactWarps) encode_compact_kernel(FinArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.x * kCompactWarps + (threadIdx.x >> 5);
+  if (b >= a.B) return;
+  const int o0 = a.target_off[b], n = a.target_off[b + 1] - o0;
+  for (int j = lane; j < n; j += 32) a.target_ids[o0 + j] = a.pad_ids[int64_t(b) * a.max_m + j];
 }
 
 // ------------------------------------------------------- Lemma-1 byte check
@@ -539,6 +544,8 @@ extern "C" tt_status tt_encode(int32_t B, int32_t n_draft, const int32_t* draft_
   f.target_off = target_off;
   f.target_ids = target_ids;
   encode_finish_kernel<<<1, kFinThreads, 0, s>>>(f);
+  if ((e = cudaGetLastError()) != cudaSuccess) return record_cuda_error(e);
+  encode_compact_kernel<<<(B + kCompactWarps - 1) / kCompactWarps, 32 * kCompactWarps, 0, s>>>(f);
   e = cudaGetLastError();
   return e == cudaSuccess ? TT_OK : record_cuda_error(e);
 }
