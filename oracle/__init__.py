@@ -66,6 +66,13 @@ def lib():
         L.tto_verify.argtypes = [i32, P, P, P, P, i32, i64, i32, f64, P, P, P, i32, i64, i32,
                                  f64, i32, u64, u64, P, P, P, P, P, P]
         L.tto_verify.restype = None
+        L.tto_filtered_probs.argtypes = [P, i32, i64, f64, i32, f64, P, P]
+        L.tto_filtered_probs.restype = f64
+        L.tto_transfer2.argtypes = [i32, P, P, P, P, P, i32, i64, i32, P, f64, i32, f64, P, P, P]
+        L.tto_transfer2.restype = None
+        L.tto_verify2.argtypes = [i32, P, P, P, P, i32, i64, i32, f64, P, P, P, i32, i64, i32,
+                                  f64, i32, u64, u64, i32, f64, i32, f64, P, P, P, P, P, P]
+        L.tto_verify2.restype = None
         L.tto_encode.argtypes = [i32, P, P, P, P, i32, P, P, i32, i32, i32, i32, P, P, P]
         L.tto_encode.restype = None
         L.tto_consistency.argtypes = [i32, P, P, P, P, P, P, i32, P, P, i32, i32, i32, P]
@@ -163,8 +170,20 @@ def align(draft_off, draft_ids, target_off, target_ids, vd_blob, vd_off, vt_blob
                 map=mp[:nt], status=status)
 
 
+def filtered_probs(row, temp: float = 1.0, top_k: int = 0, top_p: float = 1.0):
+    """Temperature, top-k, top-p distribution of one row (tto_filtered_probs);
+    returns (probs over all columns, log-normaliser of the kept set, boundary bits)."""
+    buf, dt, stride, V = _logits(row if np.ndim(row) == 2 or not isinstance(row, np.ndarray)
+                                 else np.asarray(row, np.float32)[None, :])
+    out = np.zeros(V, np.float64)
+    bnd = np.zeros(1, np.int32)
+    lse = lib().tto_filtered_probs(_p(buf), dt, V, float(temp), int(top_k), float(top_p),
+                                   _p(out), _p(bnd))
+    return out, lse, int(bnd[0])
+
+
 def transfer(draft_off, draft_cols, target_off, mp, draft_logits, temp_draft: float = 1.0,
-             draft_probs=None) -> dict:
+             draft_probs=None, top_k: int = 0, top_p: float = 1.0) -> dict:
     draft_off, target_off, mp = _i32(draft_off), _i32(target_off), _i32(mp)
     draft_cols = _i32(draft_cols)
     B = len(draft_off) - 1
@@ -176,14 +195,17 @@ def transfer(draft_off, draft_cols, target_off, mp, draft_logits, temp_draft: fl
         buf, dt, stride, V = _logits(draft_logits)
     else:
         buf, dt, stride, V = None, 0, 0, 0
-    lib().tto_transfer(B, _p(draft_off), _p(draft_cols), _p(target_off), _p(mp), _p(buf), dt,
-                       stride, V, _p(probs), float(temp_draft), _p(q), _p(status))
-    return dict(q_hat=q[:nt], status=status)
+    bnd = np.zeros(max(B, 1), np.int32)
+    lib().tto_transfer2(B, _p(draft_off), _p(draft_cols), _p(target_off), _p(mp), _p(buf), dt,
+                        stride, V, _p(probs), float(temp_draft), int(top_k), float(top_p), _p(q),
+                        _p(status), _p(bnd))
+    return dict(q_hat=q[:nt], status=status, boundary=bnd[:B])
 
 
 def verify(target_off, target_cols, q_hat, target_logits, *, temp_target: float = 1.0,
            seed: int = 1234, request_base: int = 0, full_q: bool = False, draft_off=None,
-           mp=None, draft_logits=None, temp_draft: float = 1.0) -> dict:
+           mp=None, draft_logits=None, temp_draft: float = 1.0, top_k_target: int = 0,
+           top_p_target: float = 1.0, top_k_draft: int = 0, top_p_draft: float = 1.0) -> dict:
     target_off, target_cols = _i32(target_off), _i32(target_cols)
     q_hat = np.ascontiguousarray(q_hat, dtype=np.float64)
     B = len(target_off) - 1
@@ -200,18 +222,20 @@ def verify(target_off, target_cols, q_hat, target_logits, *, temp_target: float 
     lse = np.zeros(nt + B, np.float64)
     status = np.zeros(B, np.int32)
     bnd = np.zeros(B, np.int32)
-    lib().tto_verify(B, _p(target_off), _p(target_cols), _p(q_hat), _p(tbuf), tdt, tstride, Vt,
-                     float(temp_target), _p(draft_off) if full_q else None,
-                     _p(mp) if full_q else None, _p(dbuf), ddt, dstride, Vd, float(temp_draft),
-                     int(bool(full_q)), int(seed), int(request_base), _p(acc), _p(nxt),
-                     _p(p_hat), _p(lse), _p(status), _p(bnd))
+    lib().tto_verify2(B, _p(target_off), _p(target_cols), _p(q_hat), _p(tbuf), tdt, tstride, Vt,
+                      float(temp_target), _p(draft_off) if full_q else None,
+                      _p(mp) if full_q else None, _p(dbuf), ddt, dstride, Vd, float(temp_draft),
+                      int(bool(full_q)), int(seed), int(request_base), int(top_k_target),
+                      float(top_p_target), int(top_k_draft), float(top_p_draft), _p(acc),
+                      _p(nxt), _p(p_hat), _p(lse), _p(status), _p(bnd))
     return dict(accepted=acc, next_token=nxt, p_hat=p_hat[:nt], lse=lse, status=status,
                 boundary=bnd)
 
 
 def step(wl, *, window: Optional[int] = None, temp_draft: Optional[float] = None,
          temp_target: Optional[float] = None, seed: Optional[int] = None,
-         request_base: int = 0, full_q: bool = False, draft_probs=None) -> dict:
+         request_base: int = 0, full_q: bool = False, draft_probs=None, top_k_draft: int = 0,
+         top_p_draft: float = 1.0, top_k_target: int = 0, top_p_target: float = 1.0) -> dict:
     """The whole verification path for a workload (align -> transfer -> verify)."""
     spec = wl.spec
     window = spec.window if window is None else window
@@ -221,16 +245,18 @@ def step(wl, *, window: Optional[int] = None, temp_draft: Optional[float] = None
     al = align(wl.draft_off, wl.draft_ids, wl.target_off, wl.target_ids, wl.vd.blob, wl.vd.off,
                wl.vt.blob, wl.vt.off, window)
     tr = transfer(wl.draft_off, wl.draft_cols, wl.target_off, al["map"], wl.draft_logits,
-                  temp_draft, draft_probs)
+                  temp_draft, draft_probs, top_k=top_k_draft, top_p=top_p_draft)
     ve = verify(wl.target_off, wl.target_cols, tr["q_hat"], wl.target_logits,
                 temp_target=temp_target, seed=seed, request_base=request_base, full_q=full_q,
                 draft_off=wl.draft_off, mp=al["map"], draft_logits=wl.draft_logits,
-                temp_draft=temp_draft)
+                temp_draft=temp_draft, top_k_target=top_k_target, top_p_target=top_p_target,
+                top_k_draft=top_k_draft, top_p_draft=top_p_draft)
     # the fused step reports the alignment's problems first, else the later stages'
     status = np.where(al["status"] != 0, al["status"], tr["status"] | ve["status"])
     out = dict(al)
     out.update(q_hat=tr["q_hat"], p_hat=ve["p_hat"], lse=ve["lse"], accepted=ve["accepted"],
-               next_token=ve["next_token"], boundary=ve["boundary"], status=status)
+               next_token=ve["next_token"], boundary=ve["boundary"] | tr["boundary"],
+               status=status)
     bad = status != 0
     out["accepted"] = np.where(bad, 0, out["accepted"]).astype(np.int32)
     out["next_token"] = np.where(bad, -1, out["next_token"]).astype(np.int32)

@@ -202,6 +202,59 @@ void tto_softmax(const void* row, int32_t dtype, int64_t V, double T, double* p)
 
 /* ------------------------------------------------------------ batched align */
 
+/* ------------------------------------------------------- sampling filters */
+
+/* The generation filters of the paper's hyperparameter table, in the usual
+ * order: temperature, then top-k (keep the k largest logits; among equal
+ * logits the smaller column first), then top-p (after renormalising, keep
+ * tokens in decreasing probability while the mass before a token is below
+ * top_p, so the kept set is the smallest prefix reaching top_p). top_k <= 0 or
+ * top_k >= V: no top-k; top_p <= 0 or >= 1: no top-p. Writes the filtered
+ * distribution over all V columns (zeros outside the kept set) and returns the
+ * natural log of the kept set's normaliser sum exp(z/T). *boundary gets bit 4
+ * when the mass before some token lies within 1e-6 of top_p. */
+static const void* g_sort_row; /* the row the comparator reads (single-threaded) */
+static int32_t g_sort_dtype;
+static double sort_val(int64_t x) { return load_logit(g_sort_row, g_sort_dtype, x); }
+static int cmp_desc_logit(const void* pa, const void* pb) {
+  int64_t a = *(const int64_t*)pa, b = *(const int64_t*)pb;
+  double va = sort_val(a), vb = sort_val(b);
+  if (va > vb) return -1;
+  if (va < vb) return 1;
+  return a < b ? -1 : (a > b ? 1 : 0);
+}
+
+double tto_filtered_probs(const void* row, int32_t dtype, int64_t V, double T, int32_t top_k,
+                          double top_p, double* p, int32_t* boundary) {
+  int64_t* order = (int64_t*)malloc(sizeof(int64_t) * (size_t)V);
+  for (int64_t x = 0; x < V; ++x) order[x] = x;
+  g_sort_row = row;
+  g_sort_dtype = dtype;
+  qsort(order, (size_t)V, sizeof(int64_t), cmp_desc_logit);
+  int64_t K = (top_k <= 0 || top_k >= V) ? V : top_k;
+  /* softmax over the top-K (the maximum is the first) */
+  double mx = load_logit(row, dtype, order[0]) / T, sum = 0.0;
+  for (int64_t i = 0; i < K; ++i) sum += exp(load_logit(row, dtype, order[i]) / T - mx);
+  int64_t keep = K;
+  if (top_p > 0.0 && top_p < 1.0) {
+    double before = 0.0;
+    keep = 0;
+    while (keep < K) {
+      if (fabs(before - top_p) < 1e-6 && boundary) *boundary |= 4;
+      if (!(before < top_p)) break;
+      before += exp(load_logit(row, dtype, order[keep]) / T - mx) / sum;
+      ++keep;
+    }
+  }
+  double kept = 0.0;
+  for (int64_t i = 0; i < keep; ++i) kept += exp(load_logit(row, dtype, order[i]) / T - mx);
+  for (int64_t x = 0; x < V; ++x) p[x] = 0.0;
+  for (int64_t i = 0; i < keep; ++i)
+    p[order[i]] = exp(load_logit(row, dtype, order[i]) / T - mx) / kept;
+  free(order);
+  return mx + log(kept);
+}
+
 static int32_t offsets_ok(const int32_t* off, int32_t b) {
   return off[b] >= 0 && off[b + 1] >= off[b];
 }
@@ -266,11 +319,15 @@ void tto_align(int32_t B, const int32_t* draft_off, const int32_t* draft_ids,
 
 /* ---------------------------------------------------------------- transfer */
 
-void tto_transfer(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
-                  const int32_t* target_off, const int32_t* map,
-                  const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
-                  const float* draft_probs, double T_d, double* q_hat, int32_t* status) {
+void tto_transfer2(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                   const int32_t* target_off, const int32_t* map,
+                   const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                   const float* draft_probs, double T_d, int32_t top_k, double top_p,
+                   double* q_hat, int32_t* status, int32_t* boundary) {
+  const int filtered = top_k > 0 || (top_p > 0.0 && top_p < 1.0);
+  double* qf = filtered ? (double*)malloc(sizeof(double) * (size_t)(V > 0 ? V : 1)) : NULL;
   for (int32_t b = 0; b < B; ++b) {
+    if (boundary) boundary[b] = 0;
     if (!offsets_ok(draft_off, b) || !offsets_ok(target_off, b)) {
       status[b] = ST_BAD_OFFSETS;
       continue;
@@ -287,10 +344,18 @@ void tto_transfer(int32_t B, const int32_t* draft_off, const int32_t* draft_cols
     status[b] = st;
     for (int32_t j = 0; j < m; ++j) q_hat[t0 + j] = 0.0;
     if (st) continue;
+    int64_t have = -1; /* the draft row whose filtered distribution qf holds */
     for (int32_t j = 0; j < m; ++j) {
       int64_t r = (int64_t)d0 + map[t0 + j];
       if (draft_probs) {
         q_hat[t0 + j] = (double)draft_probs[r];
+      } else if (filtered) {
+        const void* row = row_ptr(draft_logits, dtype, row_stride, r);
+        if (r != have) {
+          tto_filtered_probs(row, dtype, V, T_d, top_k, top_p, qf, boundary ? &boundary[b] : NULL);
+          have = r;
+        }
+        q_hat[t0 + j] = qf[draft_cols[r]];
       } else {
         const void* row = row_ptr(draft_logits, dtype, row_stride, r);
         double lse = tto_logsumexp(row, dtype, V, T_d);
@@ -298,18 +363,31 @@ void tto_transfer(int32_t B, const int32_t* draft_off, const int32_t* draft_cols
       }
     }
   }
+  free(qf);
+}
+
+void tto_transfer(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                  const int32_t* target_off, const int32_t* map,
+                  const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                  const float* draft_probs, double T_d, double* q_hat, int32_t* status) {
+  tto_transfer2(B, draft_off, draft_cols, target_off, map, draft_logits, dtype, row_stride, V,
+                draft_probs, T_d, 0, 1.0, q_hat, status, NULL);
 }
 
 /* ------------------------------------------------------------------ verify */
 
-void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols,
-                const double* q_hat, const void* target_logits, int32_t dtype_t,
-                int64_t stride_t, int32_t V_t, double T_t,
-                const int32_t* draft_off, const int32_t* map, const void* draft_logits,
-                int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
-                int32_t full_q, uint64_t seed, uint64_t request_base,
-                int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
-                int32_t* status, int32_t* boundary) {
+void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                 const double* q_hat, const void* target_logits, int32_t dtype_t,
+                 int64_t stride_t, int32_t V_t, double T_t,
+                 const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                 int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                 int32_t full_q, uint64_t seed, uint64_t request_base,
+                 int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
+                 int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
+                 int32_t* status, int32_t* boundary) {
+  const int filt_t = top_k_t > 0 || (top_p_t > 0.0 && top_p_t < 1.0);
+  const int filt_d = top_k_d > 0 || (top_p_d > 0.0 && top_p_d < 1.0);
+  double* pf = filt_t ? (double*)malloc(sizeof(double) * (size_t)V_t) : NULL;
   double* p = (double*)malloc(sizeof(double) * (size_t)V_t);
   double* q = full_q ? (double*)malloc(sizeof(double) * (size_t)V_d) : NULL;
   double* r = (double*)malloc(sizeof(double) * (size_t)V_t);
@@ -342,12 +420,20 @@ void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols
     status[b] = st;
     if (st) continue;
 
-    /* p_hat_j = p_j(t_j) for every target position; lse of all m+1 rows */
+    /* p_hat_j = p_j(t_j) for every target position; lse of all m+1 rows
+       (with filters: of the kept set) */
     for (int32_t j = 0; j <= m; ++j) {
       const void* row = row_ptr(target_logits, dtype_t, stride_t, row0 + j);
-      double l = tto_logsumexp(row, dtype_t, V_t, T_t);
-      if (lse) lse[row0 + j] = l;
-      if (j < m) p_hat[t0 + j] = exp(load_logit(row, dtype_t, target_cols[t0 + j]) / T_t - l);
+      if (filt_t) {
+        double l = tto_filtered_probs(row, dtype_t, V_t, T_t, top_k_t, top_p_t, pf,
+                                      &boundary[b]);
+        if (lse) lse[row0 + j] = l;
+        if (j < m) p_hat[t0 + j] = pf[target_cols[t0 + j]];
+      } else {
+        double l = tto_logsumexp(row, dtype_t, V_t, T_t);
+        if (lse) lse[row0 + j] = l;
+        if (j < m) p_hat[t0 + j] = exp(load_logit(row, dtype_t, target_cols[t0 + j]) / T_t - l);
+      }
     }
 
     /* sequential accept, stop at the first rejection */
@@ -365,12 +451,14 @@ void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols
 
     /* the residual (or bonus) row a */
     const void* prow = row_ptr(target_logits, dtype_t, stride_t, row0 + a);
-    tto_softmax(prow, dtype_t, V_t, T_t, p);
+    if (filt_t) tto_filtered_probs(prow, dtype_t, V_t, T_t, top_k_t, top_p_t, p, &boundary[b]);
+    else tto_softmax(prow, dtype_t, V_t, T_t, p);
     if (a < m) {
       if (full_q) {
         const void* qrow = row_ptr(draft_logits, dtype_d, stride_d,
                                    (int64_t)draft_off[b] + map[t0 + a]);
-        tto_softmax(qrow, dtype_d, V_d, T_d, q);
+        if (filt_d) tto_filtered_probs(qrow, dtype_d, V_d, T_d, top_k_d, top_p_d, q, &boundary[b]);
+        else tto_softmax(qrow, dtype_d, V_d, T_d, q);
         for (int32_t x = 0; x < V_t; ++x) r[x] = p[x] > q[x] ? p[x] - q[x] : 0.0;
       } else {
         int32_t t = target_cols[t0 + a];
@@ -402,6 +490,20 @@ void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols
   free(p);
   free(q);
   free(r);
+  free(pf);
+}
+
+void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                const double* q_hat, const void* target_logits, int32_t dtype_t,
+                int64_t stride_t, int32_t V_t, double T_t,
+                const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                int32_t full_q, uint64_t seed, uint64_t request_base,
+                int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
+                int32_t* status, int32_t* boundary) {
+  tto_verify2(B, target_off, target_cols, q_hat, target_logits, dtype_t, stride_t, V_t, T_t,
+              draft_off, map, draft_logits, dtype_d, stride_d, V_d, T_d, full_q, seed,
+              request_base, 0, 1.0, 0, 1.0, accepted, next_token, p_hat, lse, status, boundary);
 }
 
 /* ------------------------------------------------------------ re-encoding */

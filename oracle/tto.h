@@ -75,6 +75,37 @@ void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols
                 int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
                 int32_t* status, int32_t* boundary);
 
+/* ------------------------------------------------------- sampling filters */
+
+/* Temperature, then top-k (keep the k largest logits, smaller column first
+ * among equal ones; k <= 0 or k >= V: none), then top-p (keep tokens in
+ * decreasing probability while the mass before a token is below top_p; top_p
+ * <= 0 or >= 1: none), as in the paper's generation hyperparameters. Writes the
+ * filtered distribution over all V columns and returns the log of the kept
+ * set's normaliser. *boundary (may be NULL) gets bit 4 when the mass before
+ * some token lies within 1e-6 of top_p. */
+double tto_filtered_probs(const void* row, int32_t dtype, int64_t V, double T, int32_t top_k,
+                          double top_p, double* p, int32_t* boundary);
+
+/* tto_transfer with the draft rows' filters (boundary: bit 4 as above, may be NULL). */
+void tto_transfer2(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                   const int32_t* target_off, const int32_t* map,
+                   const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                   const float* draft_probs, double T_d, int32_t top_k, double top_p,
+                   double* q_hat, int32_t* status, int32_t* boundary);
+
+/* tto_verify with filters on the target rows (p) and, in full-q mode, on the
+ * draft rows (q); lse is then the log-normaliser of each target row's kept set. */
+void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                 const double* q_hat, const void* target_logits, int32_t dtype_t,
+                 int64_t stride_t, int32_t V_t, double T_t,
+                 const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                 int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                 int32_t full_q, uint64_t seed, uint64_t request_base,
+                 int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
+                 int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
+                 int32_t* status, int32_t* boundary);
+
 /* ------------------------------------------------------------ re-encoding */
 
 /* Re-encoding (§4.2; App. A.1, Lemma 1): T_b = encode_t(decode_d(D_b)).
