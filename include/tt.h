@@ -77,6 +77,7 @@ typedef enum {
 #define TT_REQ_INCONSISTENT 256  /* tt_consistency: decode_t(T) != decode_d(D) (Lemma 1) */
 
 #define TT_MAX_ENCODE_BYTES 2048 /* longest decoded draft string tt_encode takes per request */
+#define TT_MAX_TOP_K 32          /* largest top-k of the sampling filters */
 #define TT_MAX_DPOS_BINS 4096    /* most bins of tt_dpos_hist */
 
 typedef enum { TT_F32 = 0, TT_BF16 = 1 } tt_dtype;
@@ -115,6 +116,19 @@ typedef struct {
   void* const* events; /* host array of 4 cudaEvent_t or NULL: tt_step records
                           them before align, before the row pass, before the
                           decision kernel and after it (profiling only) */
+  /* Sampling filters of the paper's generation hyperparameters, per family,
+     after the temperature: keep the top_k largest logits of a row (0 = off,
+     at most TT_MAX_TOP_K; among equal logits the smaller column first), then
+     keep tokens in decreasing probability while the mass before a token is
+     below top_p (top_p >= 1 = off), and renormalise the kept set. Every
+     probability of the step is then the filtered one: q_hat, p_hat, the accept
+     ratio, the residual and the bonus row; lse is the log-normaliser of each
+     target row's kept set. top_p < 1 needs top_k >= 1 (TT_ERR_UNSUPPORTED
+     otherwise); in full-q mode either both families are filtered or neither. */
+  int32_t top_k_draft;
+  float top_p_draft;
+  int32_t top_k_target;
+  float top_p_target;
 } tt_params;
 
 typedef struct {
@@ -148,8 +162,14 @@ typedef struct {
 } tt_step_out;
 
 /* Bytes of scratch the transfer / verify / step calls need for this batch and
- * these row widths. 256-byte aligned sizes; pass a 256-byte aligned pointer. */
+ * these row widths, without sampling filters. 256-byte aligned sizes; pass a
+ * 256-byte aligned pointer. */
 size_t tt_workspace_bytes(const tt_batch* batch, int32_t V_d, int32_t V_t);
+
+/* The same with the sampling filters of `prm` (a filtered family keeps
+ * top_k candidates of 8 bytes per 2048-column chunk of each row). */
+size_t tt_workspace_bytes_for(const tt_batch* batch, int32_t V_d, int32_t V_t,
+                              const tt_params* prm);
 
 /* (a) DTW alignment (§4.1, Alg. 1; App. F token distance).
  * Per request: local cost d(i,j) = Levenshtein distance between the byte

@@ -43,7 +43,9 @@ class _Logits(ctypes.Structure):
 
 class _Params(ctypes.Structure):
     _fields_ = [("window", c_i32), ("temp_draft", c_f32), ("temp_target", c_f32),
-                ("full_q", c_i32), ("seed", c_u64), ("request_base", c_u64), ("events", c_p)]
+                ("full_q", c_i32), ("seed", c_u64), ("request_base", c_u64), ("events", c_p),
+                ("top_k_draft", c_i32), ("top_p_draft", c_f32), ("top_k_target", c_i32),
+                ("top_p_target", c_f32)]
 
 
 class _Batch(ctypes.Structure):
@@ -59,7 +61,7 @@ class _StepOut(ctypes.Structure):
 
 
 _lib = None
-EXPORTS = ("tt_workspace_bytes", "tt_align", "tt_transfer", "tt_verify", "tt_step",
+EXPORTS = ("tt_workspace_bytes", "tt_workspace_bytes_for", "tt_align", "tt_transfer", "tt_verify", "tt_step",
            "tt_step_noalloc", "tt_status_string", "tt_last_cuda_error", "tt_version",
            "tt_vocab_index_bytes", "tt_vocab_index_build", "tt_encode_workspace_bytes",
            "tt_encode", "tt_consistency", "tt_dpos_hist")
@@ -85,6 +87,8 @@ def load(build_if_missing: bool = False):
     P = ctypes.POINTER
     L.tt_workspace_bytes.argtypes = [P(_Batch), c_i32, c_i32]
     L.tt_workspace_bytes.restype = ctypes.c_size_t
+    L.tt_workspace_bytes_for.argtypes = [P(_Batch), c_i32, c_i32, P(_Params)]
+    L.tt_workspace_bytes_for.restype = ctypes.c_size_t
     L.tt_align.argtypes = [P(_Batch), P(_Vocab), P(_Vocab), P(_Params), c_p, c_p, c_p, c_p, c_p,
                            c_p]
     L.tt_align.restype = c_i32
@@ -202,6 +206,11 @@ class Params:
     seed: int = 1234
     request_base: int = 0
     events: Optional[Sequence] = None  # 4 torch.cuda.Event (tt_step stage timing)
+    # sampling filters (0 / 1.0 = off); top_p < 1 needs top_k >= 1
+    top_k_draft: int = 0
+    top_p_draft: float = 1.0
+    top_k_target: int = 0
+    top_p_target: float = 1.0
 
     def _c(self, keep: list) -> _Params:
         ev = None
@@ -210,7 +219,9 @@ class Params:
             keep.append(arr)
             ev = ctypes.cast(arr, c_p)
         return _Params(int(self.window), float(self.temp_draft), float(self.temp_target),
-                       int(bool(self.full_q)), int(self.seed), int(self.request_base), ev)
+                       int(bool(self.full_q)), int(self.seed), int(self.request_base), ev,
+                       int(self.top_k_draft), float(self.top_p_draft), int(self.top_k_target),
+                       float(self.top_p_target))
 
 
 def _logits(t: Optional[torch.Tensor]) -> Optional[_Logits]:
@@ -247,13 +258,19 @@ def _empty(n, dtype, device):
 
 # ----------------------------------------------------------- entry points
 
-def tt_workspace_bytes(batch: Batch, V_d: int, V_t: int) -> int:
-    return int(load().tt_workspace_bytes(ctypes.byref(batch._c()), int(V_d), int(V_t)))
+def tt_workspace_bytes(batch: Batch, V_d: int, V_t: int,
+                       params: Optional["Params"] = None) -> int:
+    if params is None:
+        return int(load().tt_workspace_bytes(ctypes.byref(batch._c()), int(V_d), int(V_t)))
+    return int(load().tt_workspace_bytes_for(ctypes.byref(batch._c()), int(V_d), int(V_t),
+                                             ctypes.byref(params._c([]))))
 
 
-def workspace(batch: Batch, V_d: int, V_t: int, device="cuda") -> torch.Tensor:
-    """Scratch for transfer / verify / step (the caching allocator aligns to 512 bytes)."""
-    return torch.empty(max(tt_workspace_bytes(batch, V_d, V_t), 256), dtype=torch.uint8,
+def workspace(batch: Batch, V_d: int, V_t: int, device="cuda",
+              params: Optional["Params"] = None) -> torch.Tensor:
+    """Scratch for transfer / verify / step (the caching allocator aligns to 512 bytes);
+    pass the call's params when it uses sampling filters."""
+    return torch.empty(max(tt_workspace_bytes(batch, V_d, V_t, params), 256), dtype=torch.uint8,
                        device=device)
 
 
@@ -281,7 +298,7 @@ def tt_transfer(batch: Batch, map: torch.Tensor, params: Params, *, draft_logits
     o.setdefault("q_hat", _empty(batch.n_target, torch.float32, dev))
     o.setdefault("status", _empty(batch.B, torch.int32, dev))
     if ws is None and draft_logits is not None:
-        ws = workspace(batch, draft_logits.shape[1], 0, dev)
+        ws = workspace(batch, draft_logits.shape[1], 0, dev, params)
     keep = []
     L = _logits(draft_logits)
     code = load().tt_transfer(ctypes.byref(batch._c()), _ptr(map),
@@ -304,7 +321,7 @@ def tt_verify(batch: Batch, q_hat: torch.Tensor, target_logits: torch.Tensor, pa
     o.setdefault("lse", _empty(batch.n_target + batch.B, torch.float32, dev))
     if ws is None:
         Vd = draft_logits.shape[1] if (params.full_q and draft_logits is not None) else 0
-        ws = workspace(batch, Vd, target_logits.shape[1], dev)
+        ws = workspace(batch, Vd, target_logits.shape[1], dev, params)
     keep = []
     Lt, Ld = _logits(target_logits), _logits(draft_logits)
     code = load().tt_verify(ctypes.byref(batch._c()), _ptr(q_hat), ctypes.byref(Lt),
@@ -346,7 +363,7 @@ class StepCall:
         self.out = out if out is not None else step_outputs(batch, dev)
         if ws is None:
             Vd = draft_logits.shape[1] if draft_logits is not None else 0
-            ws = workspace(batch, Vd, target_logits.shape[1], dev)
+            ws = workspace(batch, Vd, target_logits.shape[1], dev, params)
         self._keep = [batch, vd, vt, draft_logits, target_logits, draft_probs, ws, self.out]
         self._b = batch._c()
         self._vd = vd._c()

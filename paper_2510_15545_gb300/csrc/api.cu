@@ -76,8 +76,23 @@ bool params_ok(const tt_params* p) {
   if (!(p->temp_draft > 0.f) || !std::isfinite(p->temp_draft)) return false;
   if (!(p->temp_target > 0.f) || !std::isfinite(p->temp_target)) return false;
   if (p->full_q != 0 && p->full_q != 1) return false;
+  if (p->top_k_draft < 0 || p->top_k_draft > TT_MAX_TOP_K) return false;
+  if (p->top_k_target < 0 || p->top_k_target > TT_MAX_TOP_K) return false;
+  if (!(p->top_p_draft > 0.f) || std::isnan(p->top_p_draft)) return false;
+  if (!(p->top_p_target > 0.f) || std::isnan(p->top_p_target)) return false;
   return true;
 }
+
+// Filters the kernels take: top-p only after a top-k (a nucleus over the whole
+// vocabulary is not built).
+bool filters_supported(const tt_params* p) {
+  if (p->top_p_draft < 1.f && p->top_k_draft == 0) return false;
+  if (p->top_p_target < 1.f && p->top_k_target == 0) return false;
+  return true;
+}
+
+int k_draft(const tt_params* p) { return p->top_k_draft; }
+int k_target(const tt_params* p) { return p->top_k_target; }
 
 bool vocab_ok(const tt_vocab* v) {
   return v && v->bytes && v->offsets && v->n_tokens >= 1 && v->n_bytes >= 0;
@@ -95,6 +110,8 @@ RowSet rowset(const tt_logits* L, Partial* part, const uint8_t* need, float T) {
   r.n_rows = L->n_rows;
   r.part = part;
   r.need = need;
+  r.top_k = 0;
+  r.cand = nullptr;
   return r;
 }
 
@@ -141,6 +158,16 @@ tt_status record_cuda_error(cudaError_t e) { return cuda_fail(e); }
 
 extern "C" {
 
+size_t tt_workspace_bytes_for(const tt_batch* batch, int32_t V_d, int32_t V_t,
+                              const tt_params* prm) {
+  if (!batch || batch->B < 0 || batch->n_draft < 0 || batch->n_target < 0) return 0;
+  const int kd = prm ? prm->top_k_draft : 0, kt = prm ? prm->top_k_target : 0;
+  if (kd < 0 || kd > TT_MAX_TOP_K || kt < 0 || kt > TT_MAX_TOP_K) return 0;
+  return workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d < 0 ? 0 : V_d,
+                          V_t < 0 ? 0 : V_t, kd, kt)
+      .bytes;
+}
+
 size_t tt_workspace_bytes(const tt_batch* batch, int32_t V_d, int32_t V_t) {
   if (!batch || batch->B < 0 || batch->n_draft < 0 || batch->n_target < 0) return 0;
   return workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d < 0 ? 0 : V_d,
@@ -179,13 +206,17 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   if (from_logits && !logits_ok(draft, batch->n_draft)) return TT_ERR_INVALID_ARG;
   const int32_t* cols = batch->draft_cols ? batch->draft_cols : batch->draft_ids;
   if (from_logits && batch->n_draft > 0 && !cols) return TT_ERR_INVALID_ARG;
+  if (!filters_supported(prm)) return TT_ERR_UNSUPPORTED;
+  const int kd = from_logits ? k_draft(prm) : 0;  // given probabilities are taken as they are
   const int V_d = from_logits ? draft->n_cols : 0;
-  const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d, 0).bytes;
+  const size_t need =
+      workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d, 0, kd, 0).bytes;
   if (from_logits && (!workspace || workspace_bytes < need ||
                       (reinterpret_cast<uintptr_t>(workspace) & 255) != 0))
     return TT_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d, 0);
+  Workspace ws =
+      workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d, 0, kd, 0);
 
   DecideArgs d;
   std::memset(&d, 0, sizeof d);
@@ -201,6 +232,9 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   d.map = map;
   d.draft_probs = draft_probs;
   d.d = from_logits ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
+  d.d.top_k = kd;
+  d.d.cand = ws.cand_d;
+  d.top_p_d = prm->top_p_draft;
   d.t = no_rows();
   d.dt_d = from_logits ? draft->dtype : TT_F32;
   d.status = status;
@@ -233,7 +267,11 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
     if ((e = launch_rowpass(r, draft->dtype, TT_F32, s, sm_count_current(), true)) != cudaSuccess)
       return cuda_fail(e);
   }
-  if ((e = launch_decide(d, s, from_logits)) != cudaSuccess) return cuda_fail(e);
+  if (kd > 0) {
+    if ((e = launch_filter_q(d, s, true)) != cudaSuccess) return cuda_fail(e);
+  } else if ((e = launch_decide(d, s, from_logits)) != cudaSuccess) {
+    return cuda_fail(e);
+  }
   return TT_OK;
 }
 
@@ -254,14 +292,18 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
     if (!logits_ok(draft, batch->n_draft) || draft->n_cols != target->n_cols) return TT_ERR_INVALID_ARG;
     if (batch->n_target > 0 && !map) return TT_ERR_INVALID_ARG;
   }
+  if (!filters_supported(prm)) return TT_ERR_UNSUPPORTED;
+  // q_hat is given; the draft rows' filter matters only to the full-q residual
+  const int kt = k_target(prm), kd = full_q ? k_draft(prm) : 0;
+  if (full_q && (kd > 0) != (kt > 0)) return TT_ERR_UNSUPPORTED;
   const int V_d = full_q ? draft->n_cols : 0;
   const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d,
-                                       target->n_cols).bytes;
+                                       target->n_cols, kd, kt).bytes;
   if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
     return TT_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d,
-                                  target->n_cols);
+                                  target->n_cols, kd, kt);
   cudaError_t e = ensure_loaded();
   if (e != cudaSuccess) return cuda_fail(e);
   if (full_q) {  // the residual needs the mapped draft rows' normalisers
@@ -280,8 +322,12 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   RowPassArgs r;
   std::memset(&r, 0, sizeof r);
   r.t = rowset(target, ws.part_t, nullptr, prm->temp_target);
+  r.t.top_k = kt;
+  r.t.cand = ws.cand_t;
   r.rows_t = int64_t(batch->n_target) + batch->B;
   r.d = full_q ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
+  r.d.top_k = kd;
+  r.d.cand = ws.cand_d;
   r.rows_d = full_q ? batch->n_draft : 0;
   r.B = batch->B;
   r.n_target = batch->n_target;
@@ -322,7 +368,13 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   d.lse = lse;
   d.err = ws.err;
   d.epoch = r.epoch;
-  if ((e = launch_decide(d, s, true)) != cudaSuccess) return cuda_fail(e);
+  d.top_p_d = prm->top_p_draft;
+  d.top_p_t = prm->top_p_target;
+  if (kt > 0) {
+    if ((e = launch_decide_filtered(d, s, true)) != cudaSuccess) return cuda_fail(e);
+  } else if ((e = launch_decide(d, s, true)) != cudaSuccess) {
+    return cuda_fail(e);
+  }
   return TT_OK;
 }
 
@@ -341,9 +393,14 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   if (!logits_ok(target, int64_t(batch->n_target) + batch->B)) return TT_ERR_INVALID_ARG;
   if (from_logits && !logits_ok(draft, batch->n_draft)) return TT_ERR_INVALID_ARG;
   if (full_q && draft->n_cols != target->n_cols) return TT_ERR_INVALID_ARG;
+  if (!filters_supported(prm)) return TT_ERR_UNSUPPORTED;
+  // given draft probabilities are taken as they are (no draft filter)
+  const int kd = from_logits ? k_draft(prm) : 0, kt = k_target(prm);
+  if (full_q && (kd > 0) != (kt > 0)) return TT_ERR_UNSUPPORTED;
+  const bool filtered = kd > 0 || kt > 0;
   const int V_d = from_logits ? draft->n_cols : 0;
   const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d,
-                                       target->n_cols).bytes;
+                                       target->n_cols, kd, kt).bytes;
   if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
     return TT_ERR_INVALID_ARG;
   const int32_t* dcols = batch->draft_cols ? batch->draft_cols : batch->draft_ids;
@@ -354,7 +411,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d,
-                                  target->n_cols);
+                                  target->n_cols, kd, kt);
   int32_t* map = out->map ? out->map : ws.map;
   a.path = out->path;
   a.path_len = out->path_len;
@@ -378,6 +435,10 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   r.rows_t = int64_t(batch->n_target) + batch->B;
   r.d = from_logits ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
   r.rows_d = from_logits ? batch->n_draft : 0;
+  r.t.top_k = kt;
+  r.t.cand = ws.cand_t;
+  r.d.top_k = kd;
+  r.d.cand = ws.cand_d;
   r.B = batch->B;
   r.n_target = batch->n_target;
   r.target_off = batch->target_off;
@@ -424,8 +485,38 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   d.lse = out->lse;
   d.err = ws.err;
   d.epoch = r.epoch;
-  d.warm_ctas = sm_count_current();  // the first CTA on each SM
-  if ((e = launch_decide(d, s, pdl)) != cudaSuccess) return cuda_fail(e);
+  d.top_p_d = prm->top_p_draft;
+  d.top_p_t = prm->top_p_target;
+  if (!filtered) {
+    d.warm_ctas = sm_count_current();  // the first CTA on each SM
+    if ((e = launch_decide(d, s, pdl)) != cudaSuccess) return cuda_fail(e);
+    record(prm, 3, s);
+    return TT_OK;
+  }
+  // Filtered: q_hat first (from the draft rows' top-k lists, or as without
+  // filters), into out->q_hat or the workspace with its own status; then the
+  // decision over the target rows (their top-k lists, or the partials).
+  float* qbuf = out->q_hat ? out->q_hat : ws.q_hat;
+  DecideArgs q = d;
+  q.mode_transfer_only = 1;
+  q.status = ws.status;
+  q.q_hat_out = qbuf;
+  q.draft_probs = full_q ? nullptr : draft_probs;
+  if (kd > 0) {
+    if ((e = launch_filter_q(q, s, pdl)) != cudaSuccess) return cuda_fail(e);
+  } else if ((e = launch_decide(q, s, pdl)) != cudaSuccess) {
+    return cuda_fail(e);
+  }
+  d.q_hat_in = qbuf;
+  d.q_hat_out = nullptr;
+  d.draft_probs = nullptr;
+  d.status_q = ws.status;
+  if (kt > 0) {
+    if ((e = launch_decide_filtered(d, s, pdl)) != cudaSuccess) return cuda_fail(e);
+  } else if ((e = launch_decide(d, s, false)) != cudaSuccess) {
+    // (this decision kernel reads q_hat before its grid-dependency wait)
+    return cuda_fail(e);
+  }
   record(prm, 3, s);
   return TT_OK;
 }
@@ -442,6 +533,6 @@ const char* tt_status_string(tt_status s) {
 
 int32_t tt_last_cuda_error(void) { return g_last_cuda_error; }
 
-int32_t tt_version(void) { return 100; }
+int32_t tt_version(void) { return 110; }
 
 }  // extern "C"

@@ -365,9 +365,12 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
       }
   }
   const int s_in = a.status_in ? __ldcg(a.status_in + b) : 0;
+  // (status_q, when given, comes from a kernel that ended before this grid started)
+  const int s_q = a.status_q ? __ldcg(a.status_q + b) : 0;
   if (bad) atomicOr(&s_bad, bad);
   __syncthreads();
   if (st == 0 && (s_bad & 1)) st |= TT_REQ_ID_OUT_OF_RANGE;
+  if (st == 0 && s_q != 0) st = s_q;  // the transfer's verdict
   if (s_in != 0) st = s_in;  // the alignment's verdict comes first
   if (st == 0 && (s_bad & 2)) st |= TT_REQ_ID_OUT_OF_RANGE;
 

@@ -1,0 +1,493 @@
+// filter.cu -- verification under the sampling filters of the paper's
+// generation hyperparameters (temperature, top-k, top-p), for the families
+// whose rows the row pass reduced to top-k lists (one sorted list of k
+// candidates per 2048-column chunk).
+//
+// A filtered row's distribution is fixed by its top k logits: the row's top-k
+// is merged from its chunk lists (the k-th largest chunk head bounds the row's
+// k-th largest from below, so only list entries at or above it are read),
+// then softmax at temperature, the top-p cut and renormalisation give the kept
+// set. filter_q_kernel turns the mapped draft rows into q_hat (§4.2, App. A.2
+// with the filtered draft distribution); decide_filtered_kernel takes p_hat
+// from the target rows' kept sets, runs the accept test (Alg. 2 / Alg. 4) and
+// draws the next token from the residual (or the bonus row) over the kept set,
+// in column order.
+#include <cstdint>
+
+#include "tt_device.cuh"
+#include "tt_launch.h"
+
+namespace tt {
+
+namespace {
+
+constexpr int kFThreads = 256;
+constexpr int kFWarps = kFThreads / 32;
+constexpr int kRowCap = 256;  // merge candidates of one row a warp keeps in shared memory
+
+struct F2 {  // unevaluated sum hi + lo
+  float hi, lo;
+};
+
+__device__ __forceinline__ F2 two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  return {s, __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb))};
+}
+
+__device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
+  const F2 s = two_sum(a.hi, b.hi);
+  const float lo = __fadd_rn(s.lo, __fadd_rn(a.lo, b.lo));
+  const float hi = __fadd_rn(s.hi, lo);
+  return {hi, __fsub_rn(lo, __fsub_rn(hi, s.hi))};
+}
+
+// a * b as a normalised pair.
+__device__ __forceinline__ F2 f2_mul_f(F2 a, float b) {
+  const float p = __fmul_rn(a.hi, b);
+  const float e = fmaf(a.hi, b, -p);
+  const float lo = fmaf(a.lo, b, e);
+  const float hi = __fadd_rn(p, lo);
+  return {hi, __fsub_rn(lo, __fsub_rn(hi, p))};
+}
+
+__device__ __forceinline__ bool f2_lt(F2 a, F2 b) {
+  return a.hi < b.hi || (a.hi == b.hi && a.lo < b.lo);
+}
+
+__device__ __forceinline__ F2 shfl_up_f2(F2 v, int o) {
+  return {__shfl_up_sync(0xffffffffu, v.hi, o), __shfl_up_sync(0xffffffffu, v.lo, o)};
+}
+
+// Inclusive prefix in pairs over the warp's lanes.
+__device__ __forceinline__ F2 warp_scan_f2(F2 v, int lane) {
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const F2 n = shfl_up_f2(v, o);
+    if (lane >= o) v = f2_add(n, v);
+  }
+  return v;
+}
+
+// 2^(z * scale - M) with the exponent split exactly (TwoProd, TwoSum, rint);
+// only 2^f, |f| <= 1/2, comes from the SFU.
+__device__ __forceinline__ float exp2_scaled(float z, float scale, float M) {
+  const float xh = __fmul_rn(z, scale);
+  const float xl = fmaf(z, scale, -xh);
+  const F2 d = two_sum(xh, -M);
+  const float n = rintf(d.hi);
+  const float f = __fadd_rn(__fsub_rn(d.hi, n), __fadd_rn(d.lo, xl));
+  if (!(n > -126.f)) return 0.f;
+  return ex2_approx(f) * __int_as_float((int(n) + 127) << 23);
+}
+
+__device__ __forceinline__ bool cand_before(float v1, int c1, float v2, int c2) {
+  return v1 > v2 || (v1 == v2 && c1 < c2);
+}
+
+// Warp-wide best element after (pv, pc) in candidate order; f = found.
+__device__ __forceinline__ void warp_best(float& bv, int& bc, bool& f) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+    const int oc = __shfl_xor_sync(0xffffffffu, bc, o);
+    const bool of = __shfl_xor_sync(0xffffffffu, int(f), o) != 0;
+    if (of && (!f || cand_before(ov, oc, bv, bc))) {
+      bv = ov;
+      bc = oc;
+      f = true;
+    }
+  }
+}
+
+// The top-K of one filtered row (its nch chunk lists of K entries merged),
+// ordered by cand_before, padded with (-inf, -1). One warp; `scr` holds
+// kRowCap candidates, `top` K entries (shared memory).
+__device__ void row_topk(const Cand* lists, int nch, int K, int lane, Cand* scr, Cand* top) {
+  // tau: the K-th best chunk head (fewer than K heads: every entry counts)
+  float tau = -INFINITY;
+  {
+    float pv = INFINITY;
+    int pc = -1;
+    for (int r = 0; r < K; ++r) {
+      float bv = -INFINITY;
+      int bc = 0x7fffffff;
+      bool f = false;
+      for (int c = lane; c < nch; c += 32) {
+        const Cand h = lists[int64_t(c) * K];
+        if (h.c >= 0 && cand_before(pv, pc, h.v, h.c) && (!f || cand_before(h.v, h.c, bv, bc))) {
+          bv = h.v;
+          bc = h.c;
+          f = true;
+        }
+      }
+      warp_best(bv, bc, f);
+      if (!f) {
+        tau = -INFINITY;
+        break;
+      }
+      pv = bv;
+      pc = bc;
+      if (r == K - 1) tau = bv;
+    }
+  }
+  // candidates: every list entry at or above tau (lists are ordered)
+  int cnt = 0;
+  for (int c = lane; c < nch; c += 32)
+    for (int i = 0; i < K; ++i) {
+      const Cand x = lists[int64_t(c) * K + i];
+      if (x.c < 0 || x.v < tau) break;
+      ++cnt;
+    }
+  int incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int n = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += n;
+  }
+  const int C = __shfl_sync(0xffffffffu, incl, 31);
+  if (C <= kRowCap) {
+    int pos = incl - cnt;
+    for (int c = lane; c < nch; c += 32)
+      for (int i = 0; i < K; ++i) {
+        const Cand x = lists[int64_t(c) * K + i];
+        if (x.c < 0 || x.v < tau) break;
+        scr[pos++] = x;
+      }
+    __syncwarp();
+    for (int i = lane; i < C; i += 32) {
+      const Cand ci = scr[i];
+      int r = 0;
+      for (int j = 0; j < C; ++j) r += cand_before(scr[j].v, scr[j].c, ci.v, ci.c);
+      if (r < K) top[r] = ci;
+    }
+    for (int r = C + lane; r < K; r += 32) top[r] = Cand{-INFINITY, -1};
+  } else {
+    // exact extraction over every list entry
+    float pv = INFINITY;
+    int pc = -1;
+    for (int r = 0; r < K; ++r) {
+      float bv = -INFINITY;
+      int bc = 0x7fffffff;
+      bool f = false;
+      for (int c = lane; c < nch; c += 32)
+        for (int i = 0; i < K; ++i) {
+          const Cand x = lists[int64_t(c) * K + i];
+          if (x.c < 0) break;
+          if (cand_before(pv, pc, x.v, x.c) && (!f || cand_before(x.v, x.c, bv, bc))) {
+            bv = x.v;
+            bc = x.c;
+            f = true;
+          }
+        }
+      warp_best(bv, bc, f);
+      if (lane == 0) top[r] = f ? Cand{bv, bc} : Cand{-INFINITY, -1};
+      if (f) {
+        pv = bv;
+        pc = bc;
+      } else {
+        pv = -INFINITY;
+        pc = 0x7fffffff;
+      }
+    }
+  }
+  __syncwarp();
+}
+
+// The kept set of a filtered row from its top-K (in shared memory): lane i < n
+// holds kept entry i (column, probability); returns n (0: no finite logit).
+// lse = natural log of the kept set's normaliser sum exp(z / T).
+__device__ int kept_set(const Cand* top, int K, float scale, float top_p, int lane, int& col,
+                        float& prob, float& lse) {
+  const Cand me = lane < K ? top[lane] : Cand{-INFINITY, -1};
+  const float v0 = top[0].v;
+  if (!(v0 > -INFINITY) || isnan(v0) || top[0].c < 0) {
+    col = -1;
+    prob = 0.f;
+    lse = NAN;
+    return 0;
+  }
+  const float M = __fmul_rn(v0, scale);
+  const bool valid = lane < K && me.c >= 0;
+  const float e = valid ? exp2_scaled(me.v, scale, M) : 0.f;
+  const F2 incl = warp_scan_f2(F2{e, 0.f}, lane);
+  const F2 all = {__shfl_sync(0xffffffffu, incl.hi, 31), __shfl_sync(0xffffffffu, incl.lo, 31)};
+  const F2 prev = shfl_up_f2(incl, 1);
+  const F2 before = lane == 0 ? F2{0.f, 0.f} : prev;
+  // top-p: keep while the mass before the token is below top_p
+  const bool keep = valid && (!(top_p < 1.f) || f2_lt(before, f2_mul_f(all, top_p)));
+  const unsigned km = __ballot_sync(0xffffffffu, keep);
+  const int n = __popc(km);  // a prefix of the lanes
+  const F2 kept_incl = warp_scan_f2(F2{keep ? e : 0.f, 0.f}, lane);
+  const float S = __shfl_sync(0xffffffffu, __fadd_rn(kept_incl.hi, kept_incl.lo), 31);
+  col = keep ? me.c : -1;
+  prob = keep ? e * __frcp_rn(S) : 0.f;
+  lse = (M + lg2_approx(S)) * 0.6931471805599453f;
+  return n;
+}
+
+// Probability of column c in the kept set held by the warp's lanes (0 if absent).
+__device__ __forceinline__ float kept_prob(int col, float prob, int c) {
+  const unsigned hit = __ballot_sync(0xffffffffu, col >= 0 && col == c);
+  return hit ? __shfl_sync(0xffffffffu, prob, __ffs(hit) - 1) : 0.f;
+}
+
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// ------------------------------------------------------- q_hat, filtered
+
+__global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
+  __shared__ int s_map[TT_MAX_M];
+  __shared__ float s_q[TT_MAX_M];
+  __shared__ Cand s_scr[kFWarps][kRowCap];
+  __shared__ Cand s_top[kFWarps][TT_MAX_TOP_K];
+  const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int K = a.d.top_k;
+  int st = 0, t0 = 0, m = 0, d0 = 0, k = 0;
+  if (!csr_ok(a.target_off, b, a.n_target) || !csr_ok(a.draft_off, b, a.n_draft)) {
+    st = TT_REQ_BAD_OFFSETS;
+  } else {
+    t0 = a.target_off[b];
+    m = a.target_off[b + 1] - t0;
+    d0 = a.draft_off[b];
+    k = a.draft_off[b + 1] - d0;
+    if (m == 0 || k == 0) st = TT_REQ_EMPTY;
+    if (m > TT_MAX_M) st |= TT_REQ_TOO_LONG;
+  }
+  int bad = 0;
+  if (st == 0)
+    for (int i = tid; i < k; i += kFThreads) {
+      const int col = a.draft_cols[d0 + i];
+      if (col < 0 || col >= a.d.V) bad = 1;
+    }
+  grid_dependency_wait();
+  if (st == 0)
+    for (int j = tid; j < m; j += kFThreads) {
+      const int i = a.map[t0 + j];
+      s_map[j] = i;
+      if (i < 0 || i >= k) bad = 1;
+    }
+  if (__syncthreads_or(bad)) st |= TT_REQ_ID_OUT_OF_RANGE;
+  if (st == 0 && a.err && a.err[0] == a.epoch) st = a.err[1];
+  if (st != 0) {
+    if (!(st & (TT_REQ_BAD_OFFSETS | TT_REQ_TOO_LONG)))
+      for (int j = tid; j < m; j += kFThreads) a.q_hat_out[t0 + j] = 0.f;
+    if (tid == 0) a.status[b] = st;
+    return;
+  }
+  // one warp per run of equal map entries (the copy rule reuses its q)
+  int nonfinite = 0;
+  for (int j = warp; j < m; j += kFWarps) {
+    if (j > 0 && s_map[j] == s_map[j - 1]) continue;
+    const int64_t row = int64_t(d0) + s_map[j];
+    row_topk(a.d.cand + row * a.d.nch * K, a.d.nch, K, lane, s_scr[warp], s_top[warp]);
+    int col;
+    float prob, lse;
+    const int n = kept_set(s_top[warp], K, a.d.scale, a.top_p_d, lane, col, prob, lse);
+    if (n == 0) nonfinite = 1;
+    const float q = kept_prob(col, prob, a.draft_cols[row]);
+    if (lane == 0) s_q[j] = q;
+  }
+  const int nf = __syncthreads_or(nonfinite);
+  for (int j = tid; j < m; j += kFThreads) {
+    int f = j;
+    while (f > 0 && s_map[f - 1] == s_map[j]) --f;
+    a.q_hat_out[t0 + j] = s_q[f];
+  }
+  if (tid == 0) a.status[b] = nf ? TT_REQ_NOT_FINITE : 0;
+}
+
+// ------------------------------------------------ decision, filtered target
+
+__global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a) {
+  __shared__ float s_p[TT_MAX_M];
+  __shared__ Cand s_scr[kFWarps][kRowCap];
+  __shared__ Cand s_top[kFWarps][TT_MAX_TOP_K];
+  __shared__ int s_a, s_nf, s_pick;
+  const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int K = a.t.top_k;
+  int st = 0, t0 = 0, m = 0, d0 = 0, k = 0;
+  if (!csr_ok(a.target_off, b, a.n_target) ||
+      (a.full_q && !csr_ok(a.draft_off, b, a.n_draft))) {
+    st = TT_REQ_BAD_OFFSETS;
+  } else {
+    t0 = a.target_off[b];
+    m = a.target_off[b + 1] - t0;
+    if (a.full_q) {
+      d0 = a.draft_off[b];
+      k = a.draft_off[b + 1] - d0;
+    }
+    if (m == 0 || (a.full_q && k == 0)) st |= TT_REQ_EMPTY;
+    if (m > a.max_m || m > TT_MAX_M) st |= TT_REQ_TOO_LONG;
+  }
+  if (tid == 0) {
+    s_a = m;
+    s_nf = 0;
+    s_pick = -1;
+  }
+  int bad = 0;
+  if (st == 0)
+    for (int j = tid; j < m; j += kFThreads) {
+      const int col = a.target_cols[t0 + j];
+      if (col < 0 || col >= a.t.V) bad = 1;
+    }
+  if (__syncthreads_or(bad)) st |= TT_REQ_ID_OUT_OF_RANGE;
+  grid_dependency_wait();
+  if (a.status_in) {
+    const int s_in = a.status_in[b];
+    if (s_in != 0) st = s_in;  // the alignment's verdict comes first
+  }
+  if (st == 0 && a.status_q) st = a.status_q[b];  // then the transfer's
+  if (a.err && a.err[0] == a.epoch) st = a.err[1];  // the row pass failed
+  bad = 0;
+  if (st == 0 && a.full_q)
+    for (int j = tid; j < m; j += kFThreads) {
+      const int i = a.map[t0 + j];
+      if (i < 0 || i >= k) bad = 1;
+    }
+  if (__syncthreads_or(bad)) st |= TT_REQ_ID_OUT_OF_RANGE;
+  if (st != 0) {
+    if (tid == 0) {
+      a.accepted[b] = 0;
+      a.next_token[b] = -1;
+      a.status[b] = st;
+    }
+    return;
+  }
+  // target rows 0..m: kept sets, p_hat, lse; one warp per row
+  for (int j = warp; j <= m; j += kFWarps) {
+    const int64_t row = int64_t(t0) + b + j;
+    row_topk(a.t.cand + row * a.t.nch * K, a.t.nch, K, lane, s_scr[warp], s_top[warp]);
+    int col;
+    float prob, lse;
+    const int n = kept_set(s_top[warp], K, a.t.scale, a.top_p_t, lane, col, prob, lse);
+    if (n == 0 && lane == 0) s_nf = 1;
+    if (j < m) {
+      const float p = kept_prob(col, prob, a.target_cols[t0 + j]);
+      if (lane == 0) {
+        s_p[j] = p;
+        if (a.p_hat) a.p_hat[t0 + j] = p;
+      }
+    }
+    if (lane == 0 && a.lse) a.lse[row] = lse;
+  }
+  __syncthreads();
+  if (s_nf) {
+    if (tid == 0) {
+      a.accepted[b] = 0;
+      a.next_token[b] = -1;
+      a.status[b] = TT_REQ_NOT_FINITE;
+    }
+    return;
+  }
+  // accept while u_j q_j < p_j (u < 1 exactly)
+  const uint64_t req = a.request_base + uint64_t(b);
+  for (int j = tid; j < m; j += kFThreads) {
+    const float u = float(philox_uniform(a.seed, uint64_t(j), 0, req));
+    if (!(u * a.q_hat_in[t0 + j] < s_p[j])) atomicMin(&s_a, j);
+  }
+  __syncthreads();
+  const int acc = s_a;
+  // the residual (or bonus) row acc over its kept set, in column order; warp 0
+  if (warp == 0) {
+    const int64_t row = int64_t(t0) + b + acc;
+    row_topk(a.t.cand + row * a.t.nch * K, a.t.nch, K, lane, s_scr[0], s_top[0]);
+    int col;
+    float prob, lse;
+    kept_set(s_top[0], K, a.t.scale, a.top_p_t, lane, col, prob, lse);
+    float qx = 0.f;  // what the residual takes away at this column
+    if (acc < m) {
+      if (a.full_q) {  // max(0, p - q) with the filtered draft row map[acc]
+        const int64_t rd = int64_t(d0) + a.map[t0 + acc];
+        row_topk(a.d.cand + rd * a.d.nch * a.d.top_k, a.d.nch, a.d.top_k, lane, s_scr[0],
+                 s_top[1]);
+        int dcol;
+        float dprob, dlse;
+        kept_set(s_top[1], a.d.top_k, a.d.scale, a.top_p_d, lane, dcol, dprob, dlse);
+        // this lane's column in the draft's kept set (lanes hold distinct columns)
+        float found = 0.f;
+        for (int l = 0; l < 32; ++l) {
+          const int c = __shfl_sync(0xffffffffu, dcol, l);
+          const float pr = __shfl_sync(0xffffffffu, dprob, l);
+          if (c >= 0 && c == col) found = pr;
+        }
+        qx = found;
+      } else if (col >= 0 && col == a.target_cols[t0 + acc]) {
+        qx = a.q_hat_in[t0 + acc];  // one-hot q
+      }
+    }
+    float r = col >= 0 ? fmaxf(0.f, prob - qx) : 0.f;
+    // total (pairs); no mass left: the row itself
+    F2 z = warp_scan_f2(F2{r, 0.f}, lane);
+    if (!(__shfl_sync(0xffffffffu, z.hi, 31) > 0.f)) r = col >= 0 ? prob : 0.f;
+    // column order: this lane's rank among the kept columns
+    int rank = 0;
+    for (int l = 0; l < 32; ++l) {
+      const int c = __shfl_sync(0xffffffffu, col, l);
+      rank += c >= 0 && col >= 0 && c < col;
+    }
+    // gather the masses in column order: lane i takes the entry of rank i
+    float rs = 0.f;
+    int cs = -1;
+    for (int l = 0; l < 32; ++l) {
+      const int rk = __shfl_sync(0xffffffffu, rank, l);
+      const int c = __shfl_sync(0xffffffffu, col, l);
+      const float x = __shfl_sync(0xffffffffu, r, l);
+      if (c >= 0 && rk == lane) {
+        rs = x;
+        cs = c;
+      }
+    }
+    const F2 incl = warp_scan_f2(F2{rs, 0.f}, lane);
+    const F2 Z = {__shfl_sync(0xffffffffu, incl.hi, 31), __shfl_sync(0xffffffffu, incl.lo, 31)};
+    const float u2 = float(philox_uniform(a.seed, uint64_t(acc), 1, req));
+    const F2 th = f2_mul_f(Z, u2);
+    const F2 prev = shfl_up_f2(incl, 1);
+    const F2 excl = lane == 0 ? F2{0.f, 0.f} : prev;
+    // the first column whose running mass exceeds theta; rounding past the
+    // end: the last column with mass
+    const bool hit = cs >= 0 && rs > 0.f && !f2_lt(th, excl) && f2_lt(th, incl);
+    const unsigned hm = __ballot_sync(0xffffffffu, hit);
+    const unsigned pm = __ballot_sync(0xffffffffu, cs >= 0 && rs > 0.f);
+    int pick = -1;
+    if (hm) pick = __shfl_sync(0xffffffffu, cs, __ffs(hm) - 1);
+    else if (pm) pick = __shfl_sync(0xffffffffu, cs, 31 - __clz(pm));
+    if (lane == 0) s_pick = pick;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    a.accepted[b] = acc;
+    a.next_token[b] = s_pick;
+    a.status[b] = s_pick >= 0 ? 0 : TT_REQ_NOT_FINITE;
+  }
+}
+
+template <typename Kern>
+cudaError_t launch_f(Kern kernel, const DecideArgs& args, cudaStream_t stream, bool pdl) {
+  if (args.B == 0) return cudaSuccess;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(args.B));
+  cfg.blockDim = dim3(kFThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args);
+}
+
+}  // namespace
+
+cudaError_t launch_filter_q(const DecideArgs& args, cudaStream_t stream, bool pdl) {
+  return launch_f(filter_q_kernel, args, stream, pdl);
+}
+
+cudaError_t launch_decide_filtered(const DecideArgs& args, cudaStream_t stream, bool pdl) {
+  return launch_f(decide_filtered_kernel, args, stream, pdl);
+}
+
+}  // namespace tt

@@ -36,7 +36,7 @@ extern "C" tt_status tt_step_noalloc(const tt_batch* batch, const tt_vocab* vd,
   const bool from_logits = draft_probs == nullptr || prm->full_q != 0;
   if (from_logits && !draft) return TT_ERR_INVALID_ARG;
   const int V_d = from_logits ? draft->n_cols : 0;
-  const size_t need = tt_workspace_bytes(batch, V_d, target->n_cols);
+  const size_t need = tt_workspace_bytes_for(batch, V_d, target->n_cols, prm);
   if (need > size_t(TT_NOALLOC_SCRATCH_BYTES)) return TT_ERR_UNSUPPORTED;
   if (batch->B == 0) return TT_OK;
 

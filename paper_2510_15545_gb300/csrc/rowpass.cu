@@ -46,13 +46,17 @@ struct Desc {
 // Stage s is always refilled for the same consumer warp (s mod kConsumerWarps),
 // so a warp never waits on a stage more than one phase ahead of it: an
 // mbarrier parity wait cannot tell phase n from phase n + 2.
-template <int DTD, int DTT>
+constexpr int kCandCap = 128;  // top-k candidates of one chunk a warp keeps in shared memory
+
+template <int DTD, int DTT, bool SEL>
 struct Ring {
   static constexpr int kStageBytes = kChunk * 4;  // one fp32 chunk or two bf16 chunks
   static constexpr int kCpsD = DTD == TT_F32 ? 1 : 2;  // chunks per stage, draft rows
   static constexpr int kCpsT = DTT == TT_F32 ? 1 : 2;  // chunks per stage, target rows
   static constexpr int kStages = kRingBytes / kStageBytes;
-  static constexpr size_t kSmem = size_t(kRingBytes) + kStages * (2 * sizeof(uint64_t) + sizeof(Desc));
+  static constexpr size_t kScratch = SEL ? size_t(kConsumerWarps) * kCandCap * sizeof(Cand) : 0;
+  static constexpr size_t kSmem =
+      size_t(kRingBytes) + kStages * (2 * sizeof(uint64_t) + sizeof(Desc)) + kScratch;
   static_assert(kStages % kConsumerWarps == 0, "each stage belongs to one consumer warp");
   static constexpr int kGrabMin = kGrabMinBytes / kStageBytes > 0 ? kGrabMinBytes / kStageBytes : 1;
   static constexpr int kGrabMax = kGrabMaxBytes / kStageBytes;
@@ -236,15 +240,157 @@ __device__ __forceinline__ void reduce_chunk(const char* stage, const Desc& d, c
   s_out = sum;
 }
 
-template <int DTD, int DTT>
+// Candidate order of the top-k: larger logit first, then smaller column.
+__device__ __forceinline__ bool cand_before(float v1, int c1, float v2, int c2) {
+  return v1 > v2 || (v1 == v2 && c1 < c2);
+}
+
+// One consumer warp writes the top-K (value, column) list of one chunk held in
+// shared memory (plus its ragged tail) to `out`, ordered by cand_before. The
+// K-th largest of the 32 lane maxima bounds the chunk's K-th largest from
+// below, so the elements at or above it are the candidates; they usually
+// number about K and are ranked by counting. More than kCandCap candidates
+// (ties, rows of equal logits) take K rounds of a warp-wide extraction.
+template <int DT>
+__device__ void select_chunk(const char* stage, const Desc& e, const RowSet& S, int lane, int K,
+                             Cand* scratch, Cand* out) {
+  constexpr int VEC = DT == TT_F32 ? 4 : 8;
+  constexpr int NV = kChunk / (VEC * 32);
+  const uint4* sv = reinterpret_cast<const uint4*>(stage);
+  const int col0 = e.chunk * kChunk;
+  float ztail = -INFINITY;
+  bool has_tail = false;
+  if (lane < e.n - e.n_smem) {
+    const char* row = S.data + e.row * S.stride_bytes;
+    ztail = load_logit<DT>(row, int64_t(col0) + e.n_smem + lane);
+    has_tail = true;
+  }
+  // lane maxima
+  float lmx = has_tail ? ztail : -INFINITY;
+  bool any = has_tail;
+#pragma unroll 4
+  for (int v = 0; v < NV; ++v) {
+    const uint4 w = sv[v * 32 + lane];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) {
+      const int el = (v * 32 + lane) * VEC + q;
+      if (el < e.n_smem) {
+        lmx = fmaxf(lmx, lane_elem<DT>(w, q));
+        any = true;
+      }
+    }
+  }
+  if (!any) lmx = -INFINITY;
+  // tau = the K-th largest lane maximum (ranks by value, then lane)
+  int rank = 0;
+#pragma unroll 8
+  for (int l = 0; l < 32; ++l) {
+    const float o = __shfl_sync(0xffffffffu, lmx, l);
+    rank += (o > lmx) || (o == lmx && l < lane);
+  }
+  const unsigned sel = __ballot_sync(0xffffffffu, rank == K - 1);
+  const float tau = __shfl_sync(0xffffffffu, lmx, __ffs(sel) - 1);
+  // candidates: valid elements >= tau
+  int cnt = (has_tail && ztail >= tau) ? 1 : 0;
+#pragma unroll 4
+  for (int v = 0; v < NV; ++v) {
+    const uint4 w = sv[v * 32 + lane];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) {
+      const int el = (v * 32 + lane) * VEC + q;
+      if (el < e.n_smem && lane_elem<DT>(w, q) >= tau) ++cnt;
+    }
+  }
+  int incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int x = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += x;
+  }
+  const int C = __shfl_sync(0xffffffffu, incl, 31);
+  if (C <= kCandCap) {
+    int pos = incl - cnt;
+    if (has_tail && ztail >= tau) scratch[pos++] = Cand{ztail, e.n_smem + lane};
+#pragma unroll 4
+    for (int v = 0; v < NV; ++v) {
+      const uint4 w = sv[v * 32 + lane];
+#pragma unroll
+      for (int q = 0; q < VEC; ++q) {
+        const int el = (v * 32 + lane) * VEC + q;
+        const float x = lane_elem<DT>(w, q);
+        if (el < e.n_smem && x >= tau) scratch[pos++] = Cand{x, el};
+      }
+    }
+    __syncwarp();
+    for (int i = lane; i < C; i += 32) {
+      const Cand ci = scratch[i];
+      int r = 0;
+      for (int j = 0; j < C; ++j) {
+        const Cand cj = scratch[j];
+        r += cand_before(cj.v, cj.c, ci.v, ci.c);
+      }
+      if (r < K) out[r] = Cand{ci.v, col0 + ci.c};
+    }
+    for (int r = C + lane; r < K; r += 32) out[r] = Cand{-INFINITY, -1};
+    __syncwarp();  // the scratch is free for the next chunk
+  } else {
+    // exact extraction: round r takes the best element after round r-1's pick
+    float pv = INFINITY;
+    int pc = -1;
+    for (int r = 0; r < K; ++r) {
+      float bv = -INFINITY;
+      int bc = 0x7fffffff;
+      bool f = false;
+      auto consider = [&](float x, int c) {
+        if (cand_before(pv, pc, x, c) && (!f || cand_before(x, c, bv, bc))) {
+          bv = x;
+          bc = c;
+          f = true;
+        }
+      };
+      if (has_tail) consider(ztail, e.n_smem + lane);
+      for (int v = 0; v < NV; ++v) {
+        const uint4 w = sv[v * 32 + lane];
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) {
+          const int el = (v * 32 + lane) * VEC + q;
+          if (el < e.n_smem) consider(lane_elem<DT>(w, q), el);
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+        const int oc = __shfl_xor_sync(0xffffffffu, bc, o);
+        const bool of = __shfl_xor_sync(0xffffffffu, int(f), o) != 0;
+        if (of && (!f || cand_before(ov, oc, bv, bc))) {
+          bv = ov;
+          bc = oc;
+          f = true;
+        }
+      }
+      if (lane == 0) out[r] = f ? Cand{bv, col0 + bc} : Cand{-INFINITY, -1};
+      if (f) {
+        pv = bv;
+        pc = bc;
+      } else {
+        pv = -INFINITY;  // nothing left: pad the rest
+        pc = 0x7fffffff;
+      }
+    }
+  }
+}
+
+template <int DTD, int DTT, bool SEL>
 __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
-  using R = Ring<DTD, DTT>;
+  using R = Ring<DTD, DTT, SEL>;
   extern __shared__ __align__(128) char smem[];
   char* stages = smem;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + kRingBytes);
   uint64_t* empty = full + R::kStages;
   Desc* desc = reinterpret_cast<Desc*>(empty + R::kStages);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // a consumer warp's candidate scratch (filtered rows only)
+  Cand* scratch = reinterpret_cast<Cand*>(desc + R::kStages) + (SEL ? warp * kCandCap : 0);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < R::kStages; ++s) {
@@ -442,7 +588,15 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       e.n = min(kChunk, d.n - lo);
       e.n_smem = max(0, min(kChunk, d.n_smem - lo));
       e.excl = (d.excl >= lo && d.excl < lo + kChunk) ? d.excl - lo : -1;
-      if (d.set) {
+      const RowSet& S = d.set ? a.t : a.d;
+      if (SEL && S.top_k > 0) {  // filtered rows: the chunk's top-k list
+        Cand* out = S.cand + (d.row * S.nch + e.chunk) * S.top_k;
+        if (d.set) {
+          select_chunk<DTT>(stage + size_t(lo) * esz, e, a.t, lane, S.top_k, scratch, out);
+        } else {
+          select_chunk<DTD>(stage + size_t(lo) * esz, e, a.d, lane, S.top_k, scratch, out);
+        }
+      } else if (d.set) {
         reduce_chunk<DTT>(stage + size_t(lo) * esz, e, a.t, lane, m[c], sum[c]);
       } else {
         reduce_chunk<DTD>(stage + size_t(lo) * esz, e, a.d, lane, m[c], sum[c]);
@@ -451,6 +605,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[s]);  // the stage's bytes are consumed
     const RowSet& S = d.set ? a.t : a.d;
+    if (SEL && S.top_k > 0) continue;
 #pragma unroll
     for (int c = 0; c < 2; ++c) {
       if (c >= cps || c * kChunk >= d.n) continue;
@@ -460,33 +615,34 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
   }
 }
 
-template <int DTD, int DTT>
+template <int DTD, int DTT, bool SEL>
 int& resident_per_sm() {
   static int per_sm = 0;
   return per_sm;
 }
 
-template <int DTD, int DTT>
+template <int DTD, int DTT, bool SEL>
 cudaError_t preload_t() {
-  using R = Ring<DTD, DTT>;
-  cudaError_t e = cudaFuncSetAttribute(rowpass_kernel<DTD, DTT>,
+  using R = Ring<DTD, DTT, SEL>;
+  cudaError_t e = cudaFuncSetAttribute(rowpass_kernel<DTD, DTT, SEL>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, int(R::kSmem));
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(rowpass_kernel<DTD, DTT>, cudaFuncAttributePreferredSharedMemoryCarveout,
+  e = cudaFuncSetAttribute(rowpass_kernel<DTD, DTT, SEL>,
+                           cudaFuncAttributePreferredSharedMemoryCarveout,
                            int(cudaSharedmemCarveoutMaxShared));
   if (e != cudaSuccess) return e;
   int per_sm = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rowpass_kernel<DTD, DTT>, kThreads,
-                                                    R::kSmem);
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rowpass_kernel<DTD, DTT, SEL>,
+                                                    kThreads, R::kSmem);
   if (e != cudaSuccess) return e;
-  resident_per_sm<DTD, DTT>() = per_sm < 1 ? 1 : per_sm;
+  resident_per_sm<DTD, DTT, SEL>() = per_sm < 1 ? 1 : per_sm;
   return cudaSuccess;
 }
 
-template <int DTD, int DTT>
+template <int DTD, int DTT, bool SEL>
 cudaError_t launch_rowpass_t(const RowPassArgs& a, cudaStream_t stream, int sm_count, bool pdl) {
-  using R = Ring<DTD, DTT>;
-  const int per_sm = resident_per_sm<DTD, DTT>();
+  using R = Ring<DTD, DTT, SEL>;
+  const int per_sm = resident_per_sm<DTD, DTT, SEL>();
   if (per_sm == 0) return cudaErrorNotReady;  // preload_rowpass() was not called
   const int64_t total = a.rows_t * ((a.t.nch + R::kCpsT - 1) / R::kCpsT) +
                         a.rows_d * ((a.d.nch + R::kCpsD - 1) / R::kCpsD);
@@ -502,25 +658,37 @@ cudaError_t launch_rowpass_t(const RowPassArgs& a, cudaStream_t stream, int sm_c
   attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, rowpass_kernel<DTD, DTT>, a);
+  return cudaLaunchKernelEx(&cfg, rowpass_kernel<DTD, DTT, SEL>, a);
+}
+
+template <int DTD, int DTT>
+cudaError_t preload_pair() {
+  cudaError_t e = preload_t<DTD, DTT, false>();
+  return e != cudaSuccess ? e : preload_t<DTD, DTT, true>();
+}
+
+template <int DTD, int DTT>
+cudaError_t launch_pair(const RowPassArgs& a, cudaStream_t stream, int sm_count, bool pdl) {
+  if (a.d.top_k > 0 || a.t.top_k > 0) return launch_rowpass_t<DTD, DTT, true>(a, stream, sm_count, pdl);
+  return launch_rowpass_t<DTD, DTT, false>(a, stream, sm_count, pdl);
 }
 
 }  // namespace
 
 cudaError_t preload_rowpass() {
   cudaError_t e;
-  if ((e = preload_t<TT_F32, TT_F32>()) != cudaSuccess) return e;
-  if ((e = preload_t<TT_F32, TT_BF16>()) != cudaSuccess) return e;
-  if ((e = preload_t<TT_BF16, TT_F32>()) != cudaSuccess) return e;
-  return preload_t<TT_BF16, TT_BF16>();
+  if ((e = preload_pair<TT_F32, TT_F32>()) != cudaSuccess) return e;
+  if ((e = preload_pair<TT_F32, TT_BF16>()) != cudaSuccess) return e;
+  if ((e = preload_pair<TT_BF16, TT_F32>()) != cudaSuccess) return e;
+  return preload_pair<TT_BF16, TT_BF16>();
 }
 
 cudaError_t launch_rowpass(const RowPassArgs& a, int dt_d, int dt_t, cudaStream_t stream,
                            int sm_count, bool pdl) {
-  if (dt_d == TT_F32 && dt_t == TT_F32) return launch_rowpass_t<TT_F32, TT_F32>(a, stream, sm_count, pdl);
-  if (dt_d == TT_F32 && dt_t == TT_BF16) return launch_rowpass_t<TT_F32, TT_BF16>(a, stream, sm_count, pdl);
-  if (dt_d == TT_BF16 && dt_t == TT_F32) return launch_rowpass_t<TT_BF16, TT_F32>(a, stream, sm_count, pdl);
-  return launch_rowpass_t<TT_BF16, TT_BF16>(a, stream, sm_count, pdl);
+  if (dt_d == TT_F32 && dt_t == TT_F32) return launch_pair<TT_F32, TT_F32>(a, stream, sm_count, pdl);
+  if (dt_d == TT_F32 && dt_t == TT_BF16) return launch_pair<TT_F32, TT_BF16>(a, stream, sm_count, pdl);
+  if (dt_d == TT_BF16 && dt_t == TT_F32) return launch_pair<TT_BF16, TT_F32>(a, stream, sm_count, pdl);
+  return launch_pair<TT_BF16, TT_BF16>(a, stream, sm_count, pdl);
 }
 
 }  // namespace tt

@@ -26,6 +26,14 @@ struct Partial {
   float s;
 };
 
+// A top-k candidate of a filtered row: the raw logit and its column; a chunk's
+// list holds its k best in order (larger logit first, then smaller column),
+// padded with (-inf, -1) when the chunk has fewer than k columns.
+struct Cand {
+  float v;
+  int32_t c;
+};
+
 // The row pass hands out work from kWorkShards counters, each on its own
 // 256-byte line, so that no single L2 address serialises every CTA's draws.
 constexpr int kWorkShards = 8;
@@ -42,11 +50,14 @@ struct Workspace {
   int32_t* err;      // two words: epoch of a call whose row pass failed, and why
   unsigned long long* work;  // row-pass work counters (kWorkShards, kWorkStride apart), zeroed
                              // by the kernel before the row pass
+  Cand* cand_d;      // [n_draft * nch_d * k_d] top-k lists of filtered draft rows
+  Cand* cand_t;      // [(n_target + B) * nch_t * k_t] top-k lists of filtered target rows
   size_t bytes;
 };
 
 __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_draft, int n_target,
-                                                      int V_d, int V_t) {
+                                                      int V_d, int V_t, int k_d = 0,
+                                                      int k_t = 0) {
   Workspace w;
   char* p = static_cast<char*>(base);
   size_t off = 0;
@@ -65,6 +76,10 @@ __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_d
   w.excl = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (size_t(n_target) + B)));
   w.err = reinterpret_cast<int32_t*>(take(2 * sizeof(int32_t)));
   w.work = reinterpret_cast<unsigned long long*>(take(kWorkShards * kWorkStride * sizeof(unsigned long long)));
+  w.cand_d = reinterpret_cast<Cand*>(
+      take(sizeof(Cand) * size_t(n_draft) * n_chunks(V_d) * size_t(k_d > 0 ? k_d : 0)));
+  w.cand_t = reinterpret_cast<Cand*>(
+      take(sizeof(Cand) * size_t(n_target + B) * n_chunks(V_t) * size_t(k_t > 0 ? k_t : 0)));
   w.bytes = off;
   return w;
 }

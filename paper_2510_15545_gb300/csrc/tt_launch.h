@@ -46,6 +46,8 @@ struct RowSet {
   int64_t n_rows;
   Partial* part;
   const uint8_t* need;  // rows to visit (NULL = all)
+  int top_k;            // > 0: filtered rows, the row pass writes top-k lists to cand
+  Cand* cand;
 };
 
 struct RowPassArgs {
@@ -88,6 +90,8 @@ struct DecideArgs {
   float* p_hat;
   float* lse;
   int warm_ctas;  // CTAs b < warm_ctas run a warming pass before the wait (see decide.cu)
+  float top_p_d, top_p_t;    // top-p of filtered families (d.top_k / t.top_k > 0)
+  const int32_t* status_q;   // status of the kernel that produced q_hat_in, or NULL
 };
 
 struct PrepArgs {
@@ -106,6 +110,12 @@ cudaError_t launch_rowpass(const RowPassArgs& args, int dt_d, int dt_t, cudaStre
                            int sm_count, bool pdl);
 cudaError_t launch_decide(const DecideArgs& args, cudaStream_t stream, bool pdl);
 cudaError_t launch_prep(const PrepArgs& args, cudaStream_t stream);
+
+// Filtered families (filter.cu): q_hat of every target position from the
+// top-k lists of the mapped draft rows, and the decision over filtered target
+// rows (args.t.top_k > 0) with q_hat_in given.
+cudaError_t launch_filter_q(const DecideArgs& args, cudaStream_t stream, bool pdl);
+cudaError_t launch_decide_filtered(const DecideArgs& args, cudaStream_t stream, bool pdl);
 
 // Loads every kernel of the library on the current device and sets its launch
 // attributes, so that no module is loaded lazily inside a dependent-launch chain.
