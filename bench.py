@@ -51,6 +51,12 @@ def parse_args(argv=None):
                          "batches are for profiler captures, not bench lines")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--temp", type=float, default=None,
+                    help="temperature of draft and target rows (default: the workload's)")
+    ap.add_argument("--top-k", type=int, default=0,
+                    help="top-k filter of draft and target rows (0 = off)")
+    ap.add_argument("--top-p", type=float, default=1.0,
+                    help="top-p filter after the top-k (1 = off)")
     ap.add_argument("--no-reencode", action="store_true",
                     help="skip timing the re-encoding, Lemma-1 check and delta-pos histogram")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -326,6 +332,11 @@ def run_mine(args):
     inp = tt.device_inputs(wl, dev)
     prm = inp["params"]
     prm.request_base = request_base(rank, wl.B)
+    if args.temp is not None:
+        prm.temp_draft = prm.temp_target = args.temp
+    prm.top_k_draft = prm.top_k_target = args.top_k
+    prm.top_p_draft = prm.top_p_target = args.top_p
+    filtered = args.top_k > 0
     batch, vd, vt = inp["batch"], inp["vd"], inp["vt"]
     dl, tl = inp["draft_logits"], inp["target_logits"]
     stream = torch.cuda.current_stream(dev)
@@ -386,7 +397,7 @@ def run_mine(args):
     peak, peak_kind = measured_hbm_peak()
     achieved = ab["total"] / (row_ms / 1e3) / 1e9
     step_gbs = ab["total"] / (sec / K) / 1e9
-    traffic = profiled_traffic(name)
+    traffic = profiled_traffic(name) if not filtered else None  # captured without filters
 
     e2e = None
     if not args.no_e2e:
@@ -412,6 +423,9 @@ def run_mine(args):
                    "V_d": wl.spec.V_d, "V_t": wl.spec.V_t,
                    "logits_cols": [int(dl.shape[1]), int(tl.shape[1])],
                    "target_tokens_per_gpu": wl.n_target, "window": prm.window,
+                   "temperature": [prm.temp_draft, prm.temp_target],
+                   "filters": ({"top_k": args.top_k, "top_p": args.top_p} if filtered
+                               else None),
                    "parallelism": "dp%d (independent requests per GPU)" % ws,
                    "l2": "inputs %.0f MB exceed the 129 MB L2; no flush between steps"
                          % ((dl.numel() * dl.element_size() + tl.numel() * tl.element_size()) / 1e6)
@@ -427,7 +441,7 @@ def run_mine(args):
                      "peak_kind": "%s copy bandwidth (hbm_gbs)" % peak_kind,
                      "traffic": traffic, "algorithmic_bytes": ab["total"],
                      "vs_nominal_8tbs": achieved / 8000.0},
-        "gpu_launches": 3 * K,
+        "gpu_launches": (4 if filtered else 3) * K,
         "clocks": clk,
     }
     if e2e is not None:

@@ -112,6 +112,7 @@ RowSet rowset(const tt_logits* L, Partial* part, const uint8_t* need, float T) {
   r.need = need;
   r.top_k = 0;
   r.cand = nullptr;
+  r.nlist = L->dtype == TT_F32 ? r.nch : (r.nch + 1) / 2;
   return r;
 }
 
@@ -119,6 +120,7 @@ RowSet no_rows() {
   RowSet r;
   std::memset(&r, 0, sizeof r);
   r.nch = 1;
+  r.nlist = 1;
   return r;
 }
 

@@ -1,10 +1,10 @@
 // filter.cu -- verification under the sampling filters of the paper's
 // generation hyperparameters (temperature, top-k, top-p), for the families
 // whose rows the row pass reduced to top-k lists (one sorted list of k
-// candidates per 2048-column chunk).
+// candidates per row unit: 2048 fp32 or 4096 bf16 columns).
 //
 // A filtered row's distribution is fixed by its top k logits: the row's top-k
-// is merged from its chunk lists (the k-th largest chunk head bounds the row's
+// is merged from its unit lists (the k-th largest list head bounds the row's
 // k-th largest from below, so only list entries at or above it are read),
 // then softmax at temperature, the top-p cut and renormalisation give the kept
 // set. filter_q_kernel turns the mapped draft rows into q_hat (§4.2, App. A.2
@@ -100,11 +100,61 @@ __device__ __forceinline__ void warp_best(float& bv, int& bc, bool& f) {
   }
 }
 
-// The top-K of one filtered row (its nch chunk lists of K entries merged),
+constexpr int kMergeLists = 4;  // lists a lane owns in the K-way merge (rows of <= 128 units)
+
+// The top-K of one filtered row by a K-way merge of its nch ordered unit
+// lists: lane l owns lists l, l + 32, ... and keeps each one's current and
+// next entry in registers; every round a warp-wide arg-best takes the winner
+// and its owner advances that list, loading the entry after next. Exact, no
+// candidate buffer. Rows of more than 32 * kMergeLists units use row_topk_wide.
+__device__ void row_topk_merge(const Cand* lists, int nch, int K, int lane, Cand* top) {
+  Cand cur[kMergeLists], nxt[kMergeLists];
+  int pos[kMergeLists];
+#pragma unroll
+  for (int i = 0; i < kMergeLists; ++i) {
+    const int c = lane + 32 * i;
+    const bool ok = c < nch;
+    cur[i] = ok ? lists[int64_t(c) * K] : Cand{-INFINITY, -1};
+    nxt[i] = ok && K > 1 ? lists[int64_t(c) * K + 1] : Cand{-INFINITY, -1};
+    pos[i] = 1;  // index of nxt in its list
+  }
+  for (int r = 0; r < K; ++r) {
+    // this lane's best current head
+    float bv = -INFINITY;
+    int bc = 0x7fffffff, bi = -1;
+#pragma unroll
+    for (int i = 0; i < kMergeLists; ++i)
+      if (cur[i].c >= 0 && (bi < 0 || cand_before(cur[i].v, cur[i].c, bv, bc))) {
+        bv = cur[i].v;
+        bc = cur[i].c;
+        bi = i;
+      }
+    bool f = bi >= 0;
+    float wv = bv;
+    int wc = bc;
+    warp_best(wv, wc, f);
+    if (lane == 0) top[r] = f ? Cand{wv, wc} : Cand{-INFINITY, -1};
+    if (!f) continue;
+    // the owner (columns are distinct) advances the winning list
+    if (bi >= 0 && bc == wc && bv == wv) {
+#pragma unroll
+      for (int i = 0; i < kMergeLists; ++i)
+        if (i == bi) {
+          cur[i] = nxt[i];
+          ++pos[i];
+          const int c = lane + 32 * i;
+          nxt[i] = pos[i] < K ? lists[int64_t(c) * K + pos[i]] : Cand{-INFINITY, -1};
+        }
+    }
+  }
+  __syncwarp();
+}
+
+// The top-K of one filtered row (its nch unit lists of K entries merged),
 // ordered by cand_before, padded with (-inf, -1). One warp; `scr` holds
-// kRowCap candidates, `top` K entries (shared memory).
-__device__ void row_topk(const Cand* lists, int nch, int K, int lane, Cand* scr, Cand* top) {
-  // tau: the K-th best chunk head (fewer than K heads: every entry counts)
+// kRowCap candidates, `top` K entries (shared memory). For rows of many units.
+__device__ void row_topk_wide(const Cand* lists, int nch, int K, int lane, Cand* scr, Cand* top) {
+  // tau: the K-th best list head (fewer than K heads: every entry counts)
   float tau = -INFINITY;
   {
     float pv = INFINITY;
@@ -192,6 +242,12 @@ __device__ void row_topk(const Cand* lists, int nch, int K, int lane, Cand* scr,
     }
   }
   __syncwarp();
+}
+
+__device__ __forceinline__ void row_topk(const Cand* lists, int nch, int K, int lane, Cand* scr,
+                                         Cand* top) {
+  if (nch <= 32 * kMergeLists) row_topk_merge(lists, nch, K, lane, top);
+  else row_topk_wide(lists, nch, K, lane, scr, top);
 }
 
 // The kept set of a filtered row from its top-K (in shared memory): lane i < n
@@ -282,7 +338,7 @@ __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
   for (int j = warp; j < m; j += kFWarps) {
     if (j > 0 && s_map[j] == s_map[j - 1]) continue;
     const int64_t row = int64_t(d0) + s_map[j];
-    row_topk(a.d.cand + row * a.d.nch * K, a.d.nch, K, lane, s_scr[warp], s_top[warp]);
+    row_topk(a.d.cand + row * a.d.nlist * K, a.d.nlist, K, lane, s_scr[warp], s_top[warp]);
     int col;
     float prob, lse;
     const int n = kept_set(s_top[warp], K, a.d.scale, a.top_p_d, lane, col, prob, lse);
@@ -359,7 +415,7 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
   // target rows 0..m: kept sets, p_hat, lse; one warp per row
   for (int j = warp; j <= m; j += kFWarps) {
     const int64_t row = int64_t(t0) + b + j;
-    row_topk(a.t.cand + row * a.t.nch * K, a.t.nch, K, lane, s_scr[warp], s_top[warp]);
+    row_topk(a.t.cand + row * a.t.nlist * K, a.t.nlist, K, lane, s_scr[warp], s_top[warp]);
     int col;
     float prob, lse;
     const int n = kept_set(s_top[warp], K, a.t.scale, a.top_p_t, lane, col, prob, lse);
@@ -393,7 +449,7 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
   // the residual (or bonus) row acc over its kept set, in column order; warp 0
   if (warp == 0) {
     const int64_t row = int64_t(t0) + b + acc;
-    row_topk(a.t.cand + row * a.t.nch * K, a.t.nch, K, lane, s_scr[0], s_top[0]);
+    row_topk(a.t.cand + row * a.t.nlist * K, a.t.nlist, K, lane, s_scr[0], s_top[0]);
     int col;
     float prob, lse;
     kept_set(s_top[0], K, a.t.scale, a.top_p_t, lane, col, prob, lse);
@@ -401,7 +457,7 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
     if (acc < m) {
       if (a.full_q) {  // max(0, p - q) with the filtered draft row map[acc]
         const int64_t rd = int64_t(d0) + a.map[t0 + acc];
-        row_topk(a.d.cand + rd * a.d.nch * a.d.top_k, a.d.nch, a.d.top_k, lane, s_scr[0],
+        row_topk(a.d.cand + rd * a.d.nlist * a.d.top_k, a.d.nlist, a.d.top_k, lane, s_scr[0],
                  s_top[1]);
         int dcol;
         float dprob, dlse;

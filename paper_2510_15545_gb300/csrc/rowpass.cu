@@ -46,7 +46,8 @@ struct Desc {
 // Stage s is always refilled for the same consumer warp (s mod kConsumerWarps),
 // so a warp never waits on a stage more than one phase ahead of it: an
 // mbarrier parity wait cannot tell phase n from phase n + 2.
-constexpr int kCandCap = 128;  // top-k candidates of one chunk a warp keeps in shared memory
+constexpr int kCandCap = 128;   // top-k candidates of one unit a warp keeps in shared memory
+constexpr int kLevel2Cap = 64;  // vector maxima ranked by counting (more: radix search)
 
 template <int DTD, int DTT, bool SEL>
 struct Ring {
@@ -54,7 +55,8 @@ struct Ring {
   static constexpr int kCpsD = DTD == TT_F32 ? 1 : 2;  // chunks per stage, draft rows
   static constexpr int kCpsT = DTT == TT_F32 ? 1 : 2;  // chunks per stage, target rows
   static constexpr int kStages = kRingBytes / kStageBytes;
-  static constexpr size_t kScratch = SEL ? size_t(kConsumerWarps) * kCandCap * sizeof(Cand) : 0;
+  static constexpr size_t kScratch =
+      SEL ? size_t(kConsumerWarps) * (kCandCap + 1) * sizeof(Cand) : 0;
   static constexpr size_t kSmem =
       size_t(kRingBytes) + kStages * (2 * sizeof(uint64_t) + sizeof(Desc)) + kScratch;
   static_assert(kStages % kConsumerWarps == 0, "each stage belongs to one consumer warp");
@@ -245,83 +247,156 @@ __device__ __forceinline__ bool cand_before(float v1, int c1, float v2, int c2) 
   return v1 > v2 || (v1 == v2 && c1 < c2);
 }
 
-// One consumer warp writes the top-K (value, column) list of one chunk held in
-// shared memory (plus its ragged tail) to `out`, ordered by cand_before. The
-// K-th largest of the 32 lane maxima bounds the chunk's K-th largest from
-// below, so the elements at or above it are the candidates; they usually
-// number about K and are ranked by counting. More than kCandCap candidates
-// (ties, rows of equal logits) take K rounds of a warp-wide extraction.
+// Largest logit of one 16-byte vector (4 fp32 or 8 bf16 logits).
 template <int DT>
-__device__ void select_chunk(const char* stage, const Desc& e, const RowSet& S, int lane, int K,
-                             Cand* scratch, Cand* out) {
-  constexpr int VEC = DT == TT_F32 ? 4 : 8;
-  constexpr int NV = kChunk / (VEC * 32);
+__device__ __forceinline__ float vec_max(const uint4& w) {
+  if constexpr (DT == TT_F32) {
+    return fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)),
+                 fmaxf(__uint_as_float(w.z), __uint_as_float(w.w)));
+  } else {
+    const uint32_t m = max_bf16x2(max_bf16x2(w.x, w.y), max_bf16x2(w.z, w.w));
+    return fmaxf(__uint_as_float(m << 16), __uint_as_float(m & 0xffff0000u));
+  }
+}
+
+// Bitonic sort of one value per lane across the warp, largest at lane 0.
+__device__ __forceinline__ float warp_sort_desc(float x, int lane) {
+#pragma unroll
+  for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      const float o = __shfl_xor_sync(0xffffffffu, x, j);
+      // lanes [i, i + k) form a run sorted descending when (i & k) == 0 (k = 32:
+      // the whole warp); the lower lane of a pair keeps the larger value there
+      const bool keep_max = ((lane & j) == 0) == (k == 32 || (lane & k) == 0);
+      x = keep_max ? fmaxf(x, o) : fminf(x, o);
+    }
+  }
+  return x;
+}
+
+// One consumer warp writes the top-K (value, column) list of one unit held in
+// shared memory (its whole 16-byte vectors) plus a ragged tail of fewer than
+// 16 bytes read directly, ordered by cand_before, padded with (-inf, -1);
+// columns are absolute. Each lane owns 16 vectors and keeps their maxima in
+// registers. Two thresholds bound the unit's K-th largest element from below:
+//   tau1, the K-th largest of the 32 lane maxima (a bitonic sort; K <= 32);
+//   tau2, the K-th largest vector maximum (K vectors reach it, so at least K
+//   elements do), found among the vectors that reach tau1: by counting when
+//   they are few, else by a radix search over the maxima in registers.
+// Only elements at or above tau2 can be in the list: about K of them, in
+// about K vectors, whatever the spread of the large logits over the lanes.
+// They are gathered in `scratch` and ranked by counting; more than kCandCap
+// (runs of equal logits) take K rounds of a warp-wide extraction over the
+// same vectors instead. The work per unit is thus nearly the same for every
+// unit, which keeps the stage ring from waiting on one slow warp.
+template <int DT>
+__device__ void select_unit(const char* stage, const Desc& d, const RowSet& S, int lane, int K,
+                            Cand* scratch, Cand* out) {
+  constexpr int VEC = DT == TT_F32 ? 4 : 8;  // logits per 16-byte vector
+  constexpr int NV = kChunk * 4 / (16 * 32);   // vectors per lane in one stage
+  constexpr uint32_t kTailBit = 1u << NV;      // flag of the lane's tail element
+  const float kNaN = __int_as_float(0x7fffffff);
   const uint4* sv = reinterpret_cast<const uint4*>(stage);
-  const int col0 = e.chunk * kChunk;
-  float ztail = -INFINITY;
-  bool has_tail = false;
-  if (lane < e.n - e.n_smem) {
-    const char* row = S.data + e.row * S.stride_bytes;
-    ztail = load_logit<DT>(row, int64_t(col0) + e.n_smem + lane);
-    has_tail = true;
+  const int col0 = d.chunk * kChunk;
+  const int nvec = d.n_smem / VEC;  // whole vectors delivered (the copy moves 16-byte units)
+  // the tail element, NaN where the lane has none (NaN never compares >= and
+  // fmaxf skips it)
+  float zt = kNaN;
+  if (lane < d.n - d.n_smem) {
+    const char* row = S.data + d.row * S.stride_bytes;
+    zt = load_logit<DT>(row, int64_t(col0) + d.n_smem + lane);
   }
-  // lane maxima
-  float lmx = has_tail ? ztail : -INFINITY;
-  bool any = has_tail;
-#pragma unroll 4
-  for (int v = 0; v < NV; ++v) {
-    const uint4 w = sv[v * 32 + lane];
+  float vm[NV];  // vector maxima; NaN for a vector past the copy
+  float m = -INFINITY;
 #pragma unroll
-    for (int q = 0; q < VEC; ++q) {
-      const int el = (v * 32 + lane) * VEC + q;
-      if (el < e.n_smem) {
-        lmx = fmaxf(lmx, lane_elem<DT>(w, q));
-        any = true;
-      }
-    }
-  }
-  if (!any) lmx = -INFINITY;
-  // tau = the K-th largest lane maximum (ranks by value, then lane)
-  int rank = 0;
-#pragma unroll 8
-  for (int l = 0; l < 32; ++l) {
-    const float o = __shfl_sync(0xffffffffu, lmx, l);
-    rank += (o > lmx) || (o == lmx && l < lane);
-  }
-  const unsigned sel = __ballot_sync(0xffffffffu, rank == K - 1);
-  const float tau = __shfl_sync(0xffffffffu, lmx, __ffs(sel) - 1);
-  // candidates: valid elements >= tau
-  int cnt = (has_tail && ztail >= tau) ? 1 : 0;
-#pragma unroll 4
   for (int v = 0; v < NV; ++v) {
-    const uint4 w = sv[v * 32 + lane];
-#pragma unroll
-    for (int q = 0; q < VEC; ++q) {
-      const int el = (v * 32 + lane) * VEC + q;
-      if (el < e.n_smem && lane_elem<DT>(w, q) >= tau) ++cnt;
-    }
+    const int vi = v * 32 + lane;
+    const float x = vec_max<DT>(sv[vi]);
+    vm[v] = vi < nvec ? x : kNaN;
+    m = fmaxf(m, vm[v]);
   }
-  int incl = cnt;
+  m = fmaxf(m, zt);
+  auto at_or_above = [&](float t) {
+    uint32_t f = zt >= t ? kTailBit : 0u;
+#pragma unroll
+    for (int v = 0; v < NV; ++v) f |= vm[v] >= t ? (1u << v) : 0u;
+    return f;
+  };
+  const float tau1 = __shfl_sync(0xffffffffu, warp_sort_desc(m, lane), K - 1);
+  uint32_t flags = at_or_above(tau1);
+
+  // tau2: the K-th largest maximum; every vector that reaches it reaches tau1
+  const int nf = __popc(flags);
+  int incl = nf;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
     const int x = __shfl_up_sync(0xffffffffu, incl, o);
     if (lane >= o) incl += x;
   }
-  const int C = __shfl_sync(0xffffffffu, incl, 31);
-  if (C <= kCandCap) {
-    int pos = incl - cnt;
-    if (has_tail && ztail >= tau) scratch[pos++] = Cand{ztail, e.n_smem + lane};
-#pragma unroll 4
-    for (int v = 0; v < NV; ++v) {
-      const uint4 w = sv[v * 32 + lane];
+  const int F1 = __shfl_sync(0xffffffffu, incl, 31);
+  float tau2;
+  if (F1 <= kLevel2Cap) {
+    float* vals = reinterpret_cast<float*>(scratch);
+    int p = incl - nf;
 #pragma unroll
-      for (int q = 0; q < VEC; ++q) {
-        const int el = (v * 32 + lane) * VEC + q;
-        const float x = lane_elem<DT>(w, q);
-        if (el < e.n_smem && x >= tau) scratch[pos++] = Cand{x, el};
-      }
-    }
+    for (int v = 0; v < NV; ++v)
+      if (flags & (1u << v)) vals[p++] = vm[v];
+    if (flags & kTailBit) vals[p] = zt;
     __syncwarp();
+    // the K-th largest w is the largest with #{values >= w} >= K (fewer than
+    // K values: none, -inf)
+    float best = -INFINITY;
+    for (int i = lane; i < F1; i += 32) {
+      const float w = vals[i];
+      int c = 0;
+#pragma unroll 4
+      for (int j = 0; j < F1; ++j) c += vals[j] >= w;
+      if (c >= K) best = fmaxf(best, w);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, o));
+    tau2 = best;
+    __syncwarp();  // the values are read before the scratch takes candidates
+  } else {
+    // radix search on order-preserving keys (x >= 0: bits | 2^31, else ~bits):
+    // the largest key t with #{maxima whose key >= t} >= K, one bit at a
+    // time. A probe's float is compared, so probes below the key of -inf
+    // (NaN floats) never pass: a K-th largest of -inf ends at t = 0.
+    uint32_t t = 0;
+    for (int b = 31; b >= 0; --b) {
+      const uint32_t probe = t | (1u << b);
+      const float pf = __uint_as_float((probe & 0x80000000u) ? (probe & 0x7fffffffu) : ~probe);
+      int c = zt >= pf;
+#pragma unroll
+      for (int v = 0; v < NV; ++v) c += vm[v] >= pf;
+      if (int(__reduce_add_sync(0xffffffffu, unsigned(c))) >= K) t = probe;
+    }
+    tau2 = t < 0x007fffffu ? -INFINITY
+                           : __uint_as_float((t & 0x80000000u) ? (t & 0x7fffffffu) : ~t);
+  }
+  flags = at_or_above(tau2);
+
+  int* count = reinterpret_cast<int*>(scratch + kCandCap);
+  if (lane == 0) *count = 0;
+  __syncwarp();
+  auto push = [&](float x, int c) {
+    const int p = atomicAdd(count, 1);
+    if (p < kCandCap) scratch[p] = Cand{x, c};
+  };
+  if (flags & kTailBit) push(zt, d.n_smem + lane);
+  for (uint32_t f = flags & (kTailBit - 1); f; f &= f - 1) {
+    const int v = __ffs(f) - 1;
+    const uint4 w = sv[v * 32 + lane];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) {
+      const float x = lane_elem<DT>(w, q);
+      if (x >= tau2) push(x, (v * 32 + lane) * VEC + q);
+    }
+  }
+  __syncwarp();
+  const int C = *reinterpret_cast<volatile int*>(count);
+  if (C <= kCandCap) {
     for (int i = lane; i < C; i += 32) {
       const Cand ci = scratch[i];
       int r = 0;
@@ -332,9 +407,9 @@ __device__ void select_chunk(const char* stage, const Desc& e, const RowSet& S, 
       if (r < K) out[r] = Cand{ci.v, col0 + ci.c};
     }
     for (int r = C + lane; r < K; r += 32) out[r] = Cand{-INFINITY, -1};
-    __syncwarp();  // the scratch is free for the next chunk
   } else {
-    // exact extraction: round r takes the best element after round r-1's pick
+    // exact extraction over the flagged vectors: round r takes the best
+    // element after round r-1's pick
     float pv = INFINITY;
     int pc = -1;
     for (int r = 0; r < K; ++r) {
@@ -348,14 +423,12 @@ __device__ void select_chunk(const char* stage, const Desc& e, const RowSet& S, 
           f = true;
         }
       };
-      if (has_tail) consider(ztail, e.n_smem + lane);
-      for (int v = 0; v < NV; ++v) {
+      if (flags & kTailBit) consider(zt, d.n_smem + lane);
+      for (uint32_t g = flags & (kTailBit - 1); g; g &= g - 1) {
+        const int v = __ffs(g) - 1;
         const uint4 w = sv[v * 32 + lane];
 #pragma unroll
-        for (int q = 0; q < VEC; ++q) {
-          const int el = (v * 32 + lane) * VEC + q;
-          if (el < e.n_smem) consider(lane_elem<DT>(w, q), el);
-        }
+        for (int q = 0; q < VEC; ++q) consider(lane_elem<DT>(w, q), (v * 32 + lane) * VEC + q);
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
@@ -378,6 +451,7 @@ __device__ void select_chunk(const char* stage, const Desc& e, const RowSet& S, 
       }
     }
   }
+  __syncwarp();  // the scratch is free for the next unit
 }
 
 template <int DTD, int DTT, bool SEL>
@@ -390,7 +464,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
   Desc* desc = reinterpret_cast<Desc*>(empty + R::kStages);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // a consumer warp's candidate scratch (filtered rows only)
-  Cand* scratch = reinterpret_cast<Cand*>(desc + R::kStages) + (SEL ? warp * kCandCap : 0);
+  Cand* scratch = reinterpret_cast<Cand*>(desc + R::kStages) + (SEL ? warp * (kCandCap + 1) : 0);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < R::kStages; ++s) {
@@ -576,6 +650,17 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
     const char* stage = stages + size_t(s) * R::kStageBytes;
     const int cps = d.set ? R::kCpsT : R::kCpsD;
     const int esz = (d.set ? DTT : DTD) == TT_F32 ? 4 : 2;
+    if (SEL && (d.set ? a.t : a.d).top_k > 0) {  // filtered rows: the unit's top-k list
+      const RowSet& S = d.set ? a.t : a.d;
+      Cand* out = S.cand + (d.row * S.nlist + d.chunk / cps) * S.top_k;
+      if (d.set) {
+        select_unit<DTT>(stage, d, a.t, lane, S.top_k, scratch, out);
+      } else {
+        select_unit<DTD>(stage, d, a.d, lane, S.top_k, scratch, out);
+      }
+      if (lane == 0) mbar_arrive(&empty[s]);  // the stage's bytes are consumed
+      continue;
+    }
     float m[2], sum[2];
 #pragma unroll
     for (int c = 0; c < 2; ++c) {  // the unit's chunks, each reduced on its own
@@ -588,15 +673,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       e.n = min(kChunk, d.n - lo);
       e.n_smem = max(0, min(kChunk, d.n_smem - lo));
       e.excl = (d.excl >= lo && d.excl < lo + kChunk) ? d.excl - lo : -1;
-      const RowSet& S = d.set ? a.t : a.d;
-      if (SEL && S.top_k > 0) {  // filtered rows: the chunk's top-k list
-        Cand* out = S.cand + (d.row * S.nch + e.chunk) * S.top_k;
-        if (d.set) {
-          select_chunk<DTT>(stage + size_t(lo) * esz, e, a.t, lane, S.top_k, scratch, out);
-        } else {
-          select_chunk<DTD>(stage + size_t(lo) * esz, e, a.d, lane, S.top_k, scratch, out);
-        }
-      } else if (d.set) {
+      if (d.set) {
         reduce_chunk<DTT>(stage + size_t(lo) * esz, e, a.t, lane, m[c], sum[c]);
       } else {
         reduce_chunk<DTD>(stage + size_t(lo) * esz, e, a.d, lane, m[c], sum[c]);
@@ -605,7 +682,6 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[s]);  // the stage's bytes are consumed
     const RowSet& S = d.set ? a.t : a.d;
-    if (SEL && S.top_k > 0) continue;
 #pragma unroll
     for (int c = 0; c < 2; ++c) {
       if (c >= cps || c * kChunk >= d.n) continue;

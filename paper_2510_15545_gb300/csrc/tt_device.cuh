@@ -26,9 +26,9 @@ struct Partial {
   float s;
 };
 
-// A top-k candidate of a filtered row: the raw logit and its column; a chunk's
-// list holds its k best in order (larger logit first, then smaller column),
-// padded with (-inf, -1) when the chunk has fewer than k columns.
+// A top-k candidate of a filtered row: the raw logit and its column; a row
+// unit's list holds its k best in order (larger logit first, then smaller
+// column), padded with (-inf, -1) when the unit has fewer than k columns.
 struct Cand {
   float v;
   int32_t c;

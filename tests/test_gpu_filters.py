@@ -80,6 +80,39 @@ def test_ties_and_candidate_overflow(k, p):
         compare(wl, g, o)
 
 
+def _padded(t: torch.Tensor) -> torch.Tensor:
+    """``t`` on the GPU as a view into rows padded to a 16-byte multiple plus
+    one more 16-byte vector, the padding NaN: a read past a row's end shows."""
+    R, V = t.shape
+    per16 = 16 // t.element_size()
+    buf = torch.full((R, (V + per16 - 1) // per16 * per16 + per16), float("nan"),
+                     dtype=t.dtype, device="cuda")
+    buf[:, :V] = t.to("cuda")
+    return buf[:, :V]
+
+
+# (V, dtype, k): a unit with a ragged tail only (4100 bf16, 2053 fp32), fewer
+# lanes' worth of columns than k (threshold -inf: 100 fp32 ranked, 150 bf16
+# past the candidate buffer), one short unit (37 bf16), several units (6001 bf16)
+@pytest.mark.parametrize("V,dtype,k", [(37, torch.bfloat16, 20), (150, torch.bfloat16, 20),
+                                       (100, torch.float32, 20), (4100, torch.bfloat16, 20),
+                                       (2053, torch.float32, 32), (6001, torch.bfloat16, 7)])
+def test_narrow_and_ragged_rows(V, dtype, k):
+    wl = W.homogeneous_workload(6, 4, V, seed=V, dtype=dtype)
+    f = dict(top_k_draft=k, top_p_draft=0.9, top_k_target=k, top_p_target=0.9)
+    inp = tt.device_inputs(wl, "cuda")
+    dl, tl = _padded(wl.draft_logits), _padded(wl.target_logits)
+    for full_q in (False, True):
+        prm = inp["params"]
+        prm.temp_draft = prm.temp_target = 0.8
+        prm.full_q = full_q
+        prm.top_k_draft, prm.top_p_draft = k, 0.9
+        prm.top_k_target, prm.top_p_target = k, 0.9
+        g = to_np(tt.tt_step(inp["batch"], inp["vd"], inp["vt"], dl, tl, prm))
+        o = oracle.step(wl, full_q=full_q, temp_draft=0.8, temp_target=0.8, **f)
+        compare(wl, g, o)
+
+
 def test_transfer_and_verify_alone_with_filters():
     wl = _wl("b64_g8_v152k", 16, seed=5)
     inp = tt.device_inputs(wl, "cuda")
