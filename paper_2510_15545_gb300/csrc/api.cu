@@ -33,6 +33,7 @@ cudaError_t ensure_loaded() {
   if ((e = preload_align()) != cudaSuccess) return e;
   if ((e = preload_rowpass()) != cudaSuccess) return e;
   if ((e = preload_decide()) != cudaSuccess) return e;
+  if ((e = preload_filter()) != cudaSuccess) return e;
   if (dev >= 0 && dev < 64) done[dev] = true;
   return cudaSuccess;
 }
@@ -122,6 +123,32 @@ RowSet no_rows() {
   r.nch = 1;
   r.nlist = 1;
   return r;
+}
+
+// Kept sets of the filtered families among d (rows_d rows) and t (rows_t).
+cudaError_t launch_kept_sets(const RowSet& d, int64_t rows_d, const RowSet& t, int64_t rows_t,
+                             const tt_params* prm, const Workspace& ws, cudaStream_t s,
+                             bool pdl) {
+  KeptArgs k;
+  std::memset(&k, 0, sizeof k);
+  k.d = d;
+  k.t = t;
+  k.rows_d = d.top_k > 0 ? rows_d : 0;
+  k.rows_t = t.top_k > 0 ? rows_t : 0;
+  k.top_p_d = prm->top_p_draft;
+  k.top_p_t = prm->top_p_target;
+  k.kept_d = ws.kept_d;
+  k.kept_t = ws.kept_t;
+  k.head_d = ws.head_d;
+  k.head_t = ws.head_t;
+  return launch_kept(k, s, sm_count_current(), pdl);
+}
+
+void attach_kept(DecideArgs& d, const Workspace& ws) {
+  d.kept_d = ws.kept_d;
+  d.kept_t = ws.kept_t;
+  d.head_d = ws.head_d;
+  d.head_t = ws.head_t;
 }
 
 void record(const tt_params* p, int i, cudaStream_t s) {
@@ -270,6 +297,9 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
       return cuda_fail(e);
   }
   if (kd > 0) {
+    attach_kept(d, ws);
+    if ((e = launch_kept_sets(d.d, batch->n_draft, no_rows(), 0, prm, ws, s, true)) != cudaSuccess)
+      return cuda_fail(e);
     if ((e = launch_filter_q(d, s, true)) != cudaSuccess) return cuda_fail(e);
   } else if ((e = launch_decide(d, s, from_logits)) != cudaSuccess) {
     return cuda_fail(e);
@@ -373,6 +403,9 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   d.top_p_d = prm->top_p_draft;
   d.top_p_t = prm->top_p_target;
   if (kt > 0) {
+    attach_kept(d, ws);
+    if ((e = launch_kept_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, s, true)) != cudaSuccess)
+      return cuda_fail(e);
     if ((e = launch_decide_filtered(d, s, true)) != cudaSuccess) return cuda_fail(e);
   } else if ((e = launch_decide(d, s, true)) != cudaSuccess) {
     return cuda_fail(e);
@@ -499,6 +532,9 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   // filters), into out->q_hat or the workspace with its own status; then the
   // decision over the target rows (their top-k lists, or the partials).
   float* qbuf = out->q_hat ? out->q_hat : ws.q_hat;
+  attach_kept(d, ws);
+  if ((e = launch_kept_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, s, pdl)) != cudaSuccess)
+    return cuda_fail(e);
   DecideArgs q = d;
   q.mode_transfer_only = 1;
   q.status = ws.status;

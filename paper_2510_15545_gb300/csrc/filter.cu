@@ -3,15 +3,16 @@
 // whose rows the row pass reduced to top-k lists (one sorted list of k
 // candidates per row unit: 2048 fp32 or 4096 bf16 columns).
 //
-// A filtered row's distribution is fixed by its top k logits: the row's top-k
-// is merged from its unit lists (the k-th largest list head bounds the row's
-// k-th largest from below, so only list entries at or above it are read),
-// then softmax at temperature, the top-p cut and renormalisation give the kept
-// set. filter_q_kernel turns the mapped draft rows into q_hat (§4.2, App. A.2
-// with the filtered draft distribution); decide_filtered_kernel takes p_hat
-// from the target rows' kept sets, runs the accept test (Alg. 2 / Alg. 4) and
-// draws the next token from the residual (or the bonus row) over the kept set,
-// in column order.
+// A filtered row's distribution is fixed by its top k logits: kept_kernel
+// merges the row's unit lists into its top-k (one warp per row, every
+// filtered row of the call at once), then softmax at temperature, the top-p
+// cut and renormalisation give the kept set, stored as k (probability,
+// column) entries. filter_q_kernel turns the mapped draft rows' kept sets
+// into q_hat (§4.2, App. A.2 with the filtered draft distribution);
+// decide_filtered_kernel takes p_hat from the target rows' kept sets, runs
+// the accept test (Alg. 2 / Alg. 4) and draws the next token from the
+// residual (or the bonus row) over the kept set, in column order.
+#include <algorithm>
 #include <cstdint>
 
 #include "tt_device.cuh"
@@ -292,13 +293,55 @@ __device__ __forceinline__ void grid_dependency_wait() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
+// ------------------------------------------------------------ kept sets
+
+// One warp per filtered row (draft rows first, then target rows; unneeded
+// draft rows skipped): the row's top-K from its unit lists, then its kept set
+// as K (probability, column) entries in value order, unused ones (0, -1),
+// and the header (lse, kept count).
+__global__ void __launch_bounds__(kFThreads) kept_kernel(KeptArgs a) {
+  __shared__ Cand s_scr[kFWarps][kRowCap];
+  __shared__ Cand s_top[kFWarps][TT_MAX_TOP_K];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t rows_d = a.d.top_k > 0 ? a.rows_d : 0, rows_t = a.t.top_k > 0 ? a.rows_t : 0;
+  const int64_t total = rows_d + rows_t;
+  const int64_t w0 = int64_t(blockIdx.x) * kFWarps + warp, stride = int64_t(gridDim.x) * kFWarps;
+  grid_dependency_wait();  // the lists (and the need flags) come from earlier kernels
+  // the next kernel reads only the caller's inputs before its own wait
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  for (int64_t w = w0; w < total; w += stride) {
+    const bool tgt = w >= rows_d;
+    const int64_t row = tgt ? w - rows_d : w;
+    const RowSet& S = tgt ? a.t : a.d;
+    if (!tgt && S.need && S.need[row] == 0) continue;
+    const int K = S.top_k;
+    row_topk(S.cand + row * S.nlist * K, S.nlist, K, lane, s_scr[warp], s_top[warp]);
+    int col;
+    float prob, lse;
+    const int n = kept_set(s_top[warp], K, S.scale, tgt ? a.top_p_t : a.top_p_d, lane, col,
+                           prob, lse);
+    Cand* out = (tgt ? a.kept_t : a.kept_d) + row * K;
+    if (lane < K) out[lane] = Cand{col >= 0 ? prob : 0.f, col};
+    if (lane == 0) (tgt ? a.head_t : a.head_d)[row] = KeptHead{lse, n};
+  }
+}
+
+// A row's kept set as kept_set leaves it: lane l < K holds entry l.
+__device__ __forceinline__ int load_kept(const Cand* kept, const KeptHead* head, int64_t row,
+                                         int K, int lane, int& col, float& prob, float& lse) {
+  const Cand e = lane < K ? kept[row * K + lane] : Cand{0.f, -1};
+  col = e.c;
+  prob = e.c >= 0 ? e.v : 0.f;
+  const KeptHead h = head[row];
+  lse = h.lse;
+  return h.n;
+}
+
 // ------------------------------------------------------- q_hat, filtered
 
 __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
   __shared__ int s_map[TT_MAX_M];
   __shared__ float s_q[TT_MAX_M];
-  __shared__ Cand s_scr[kFWarps][kRowCap];
-  __shared__ Cand s_top[kFWarps][TT_MAX_TOP_K];
   const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int K = a.d.top_k;
   int st = 0, t0 = 0, m = 0, d0 = 0, k = 0;
@@ -338,10 +381,9 @@ __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
   for (int j = warp; j < m; j += kFWarps) {
     if (j > 0 && s_map[j] == s_map[j - 1]) continue;
     const int64_t row = int64_t(d0) + s_map[j];
-    row_topk(a.d.cand + row * a.d.nlist * K, a.d.nlist, K, lane, s_scr[warp], s_top[warp]);
     int col;
     float prob, lse;
-    const int n = kept_set(s_top[warp], K, a.d.scale, a.top_p_d, lane, col, prob, lse);
+    const int n = load_kept(a.kept_d, a.head_d, row, K, lane, col, prob, lse);
     if (n == 0) nonfinite = 1;
     const float q = kept_prob(col, prob, a.draft_cols[row]);
     if (lane == 0) s_q[j] = q;
@@ -359,8 +401,6 @@ __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
 
 __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a) {
   __shared__ float s_p[TT_MAX_M];
-  __shared__ Cand s_scr[kFWarps][kRowCap];
-  __shared__ Cand s_top[kFWarps][TT_MAX_TOP_K];
   __shared__ int s_a, s_nf, s_pick;
   const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int K = a.t.top_k;
@@ -415,10 +455,9 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
   // target rows 0..m: kept sets, p_hat, lse; one warp per row
   for (int j = warp; j <= m; j += kFWarps) {
     const int64_t row = int64_t(t0) + b + j;
-    row_topk(a.t.cand + row * a.t.nlist * K, a.t.nlist, K, lane, s_scr[warp], s_top[warp]);
     int col;
     float prob, lse;
-    const int n = kept_set(s_top[warp], K, a.t.scale, a.top_p_t, lane, col, prob, lse);
+    const int n = load_kept(a.kept_t, a.head_t, row, K, lane, col, prob, lse);
     if (n == 0 && lane == 0) s_nf = 1;
     if (j < m) {
       const float p = kept_prob(col, prob, a.target_cols[t0 + j]);
@@ -449,19 +488,16 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
   // the residual (or bonus) row acc over its kept set, in column order; warp 0
   if (warp == 0) {
     const int64_t row = int64_t(t0) + b + acc;
-    row_topk(a.t.cand + row * a.t.nlist * K, a.t.nlist, K, lane, s_scr[0], s_top[0]);
     int col;
     float prob, lse;
-    kept_set(s_top[0], K, a.t.scale, a.top_p_t, lane, col, prob, lse);
+    load_kept(a.kept_t, a.head_t, row, K, lane, col, prob, lse);
     float qx = 0.f;  // what the residual takes away at this column
     if (acc < m) {
       if (a.full_q) {  // max(0, p - q) with the filtered draft row map[acc]
         const int64_t rd = int64_t(d0) + a.map[t0 + acc];
-        row_topk(a.d.cand + rd * a.d.nlist * a.d.top_k, a.d.nlist, a.d.top_k, lane, s_scr[0],
-                 s_top[1]);
         int dcol;
         float dprob, dlse;
-        kept_set(s_top[1], a.d.top_k, a.d.scale, a.top_p_d, lane, dcol, dprob, dlse);
+        load_kept(a.kept_d, a.head_d, rd, a.d.top_k, lane, dcol, dprob, dlse);
         // this lane's column in the draft's kept set (lanes hold distinct columns)
         float found = 0.f;
         for (int l = 0; l < 32; ++l) {
@@ -537,6 +573,31 @@ cudaError_t launch_f(Kern kernel, const DecideArgs& args, cudaStream_t stream, b
 }
 
 }  // namespace
+
+cudaError_t preload_filter() {
+  cudaFuncAttributes fa;
+  cudaError_t e;
+  if ((e = cudaFuncGetAttributes(&fa, kept_kernel)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, filter_q_kernel)) != cudaSuccess) return e;
+  return cudaFuncGetAttributes(&fa, decide_filtered_kernel);
+}
+
+cudaError_t launch_kept(const KeptArgs& args, cudaStream_t stream, int sm_count, bool pdl) {
+  const int64_t rows = (args.d.top_k > 0 ? args.rows_d : 0) + (args.t.top_k > 0 ? args.rows_t : 0);
+  if (rows == 0) return cudaSuccess;
+  const int64_t blocks = std::min<int64_t>((rows + kFWarps - 1) / kFWarps, int64_t(sm_count) * 8);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(blocks));
+  cfg.blockDim = dim3(kFThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kept_kernel, args);
+}
 
 cudaError_t launch_filter_q(const DecideArgs& args, cudaStream_t stream, bool pdl) {
   return launch_f(filter_q_kernel, args, stream, pdl);

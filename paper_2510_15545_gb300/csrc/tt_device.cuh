@@ -34,6 +34,14 @@ struct Cand {
   int32_t c;
 };
 
+// Header of a filtered row's kept set (the set itself is k Cand entries
+// holding (probability, column), larger logit first, unused entries (0, -1)):
+// natural log of the kept normaliser, and the kept count (0: not finite).
+struct KeptHead {
+  float lse;
+  int32_t n;
+};
+
 // The row pass hands out work from kWorkShards counters, each on its own
 // 256-byte line, so that no single L2 address serialises every CTA's draws.
 constexpr int kWorkShards = 8;
@@ -52,6 +60,10 @@ struct Workspace {
                              // by the kernel before the row pass
   Cand* cand_d;      // [n_draft * nch_d * k_d] top-k lists of filtered draft rows
   Cand* cand_t;      // [(n_target + B) * nch_t * k_t] top-k lists of filtered target rows
+  Cand* kept_d;      // [n_draft * k_d] kept sets (probability, column) of filtered draft rows
+  Cand* kept_t;      // [(n_target + B) * k_t] kept sets of filtered target rows
+  KeptHead* head_d;  // [n_draft] their headers
+  KeptHead* head_t;  // [n_target + B]
   size_t bytes;
 };
 
@@ -80,6 +92,12 @@ __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_d
       take(sizeof(Cand) * size_t(n_draft) * n_chunks(V_d) * size_t(k_d > 0 ? k_d : 0)));
   w.cand_t = reinterpret_cast<Cand*>(
       take(sizeof(Cand) * size_t(n_target + B) * n_chunks(V_t) * size_t(k_t > 0 ? k_t : 0)));
+  w.kept_d = reinterpret_cast<Cand*>(take(sizeof(Cand) * size_t(n_draft) * size_t(k_d > 0 ? k_d : 0)));
+  w.kept_t = reinterpret_cast<Cand*>(
+      take(sizeof(Cand) * size_t(n_target + B) * size_t(k_t > 0 ? k_t : 0)));
+  w.head_d = reinterpret_cast<KeptHead*>(take(k_d > 0 ? sizeof(KeptHead) * size_t(n_draft) : 0));
+  w.head_t = reinterpret_cast<KeptHead*>(
+      take(k_t > 0 ? sizeof(KeptHead) * (size_t(n_target) + B) : 0));
   w.bytes = off;
   return w;
 }

@@ -93,6 +93,22 @@ struct DecideArgs {
   int warm_ctas;  // CTAs b < warm_ctas run a warming pass before the wait (see decide.cu)
   float top_p_d, top_p_t;    // top-p of filtered families (d.top_k / t.top_k > 0)
   const int32_t* status_q;   // status of the kernel that produced q_hat_in, or NULL
+  const Cand* kept_d;        // kept sets of filtered families (written by the kept kernel)
+  const Cand* kept_t;
+  const KeptHead* head_d;
+  const KeptHead* head_t;
+};
+
+// The kept-set stage of filtered families: one warp per row merges the row's
+// unit lists into its top-k and applies temperature and top-p.
+struct KeptArgs {
+  RowSet d, t;             // families with top_k > 0 are done, the others skipped
+  int64_t rows_d, rows_t;  // rows of each family (draft rows with d.need[row] == 0 skipped)
+  float top_p_d, top_p_t;
+  Cand* kept_d;
+  Cand* kept_t;
+  KeptHead* head_d;
+  KeptHead* head_t;
 };
 
 struct PrepArgs {
@@ -112,9 +128,11 @@ cudaError_t launch_rowpass(const RowPassArgs& args, int dt_d, int dt_t, cudaStre
 cudaError_t launch_decide(const DecideArgs& args, cudaStream_t stream, bool pdl);
 cudaError_t launch_prep(const PrepArgs& args, cudaStream_t stream);
 
-// Filtered families (filter.cu): q_hat of every target position from the
-// top-k lists of the mapped draft rows, and the decision over filtered target
-// rows (args.t.top_k > 0) with q_hat_in given.
+// Filtered families (filter.cu): the kept sets of the filtered rows from their
+// top-k lists, then q_hat of every target position from the kept sets of the
+// mapped draft rows, and the decision over filtered target rows
+// (args.t.top_k > 0) with q_hat_in given.
+cudaError_t launch_kept(const KeptArgs& args, cudaStream_t stream, int sm_count, bool pdl);
 cudaError_t launch_filter_q(const DecideArgs& args, cudaStream_t stream, bool pdl);
 cudaError_t launch_decide_filtered(const DecideArgs& args, cudaStream_t stream, bool pdl);
 
@@ -123,6 +141,7 @@ cudaError_t launch_decide_filtered(const DecideArgs& args, cudaStream_t stream, 
 cudaError_t preload_align();
 cudaError_t preload_rowpass();
 cudaError_t preload_decide();
+cudaError_t preload_filter();
 
 // Records a failed CUDA call for tt_last_cuda_error() and returns TT_ERR_CUDA.
 tt_status record_cuda_error(cudaError_t e);
