@@ -47,6 +47,7 @@ struct Desc {
 // so a warp never waits on a stage more than one phase ahead of it: an
 // mbarrier parity wait cannot tell phase n from phase n + 2.
 constexpr int kCandCap = 128;   // top-k candidates of one unit a warp keeps in shared memory
+constexpr int kDirectCap = 32;  // vectors at or above tau1 taken directly (more: tau2)
 constexpr int kLevel2Cap = 64;  // vector maxima ranked by counting (more: radix search)
 
 template <int DTD, int DTT, bool SEL>
@@ -55,8 +56,7 @@ struct Ring {
   static constexpr int kCpsD = DTD == TT_F32 ? 1 : 2;  // chunks per stage, draft rows
   static constexpr int kCpsT = DTT == TT_F32 ? 1 : 2;  // chunks per stage, target rows
   static constexpr int kStages = kRingBytes / kStageBytes;
-  static constexpr size_t kScratch =
-      SEL ? size_t(kConsumerWarps) * (kCandCap + 1) * sizeof(Cand) : 0;
+  static constexpr size_t kScratch = SEL ? size_t(kConsumerWarps) * kCandCap * sizeof(Cand) : 0;
   static constexpr size_t kSmem =
       size_t(kRingBytes) + kStages * (2 * sizeof(uint64_t) + sizeof(Desc)) + kScratch;
   static_assert(kStages % kConsumerWarps == 0, "each stage belongs to one consumer warp");
@@ -259,8 +259,10 @@ __device__ __forceinline__ float vec_max(const uint4& w) {
   }
 }
 
-// Bitonic sort of one value per lane across the warp, largest at lane 0.
-__device__ __forceinline__ float warp_sort_desc(float x, int lane) {
+// Bitonic sort of one value per lane across the warp: largest at lane 0
+// (DESC) or smallest at lane 0.
+template <bool DESC>
+__device__ __forceinline__ float warp_sort(float x, int lane) {
 #pragma unroll
   for (int k = 2; k <= 32; k <<= 1) {
 #pragma unroll
@@ -268,9 +270,19 @@ __device__ __forceinline__ float warp_sort_desc(float x, int lane) {
       const float o = __shfl_xor_sync(0xffffffffu, x, j);
       // lanes [i, i + k) form a run sorted descending when (i & k) == 0 (k = 32:
       // the whole warp); the lower lane of a pair keeps the larger value there
-      const bool keep_max = ((lane & j) == 0) == (k == 32 || (lane & k) == 0);
-      x = keep_max ? fmaxf(x, o) : fminf(x, o);
+      const bool up = ((lane & j) == 0) == (k == 32 || (lane & k) == 0);
+      x = (DESC ? up : !up) ? fmaxf(x, o) : fminf(x, o);
     }
+  }
+  return x;
+}
+
+// Sorts a bitonic sequence held one value per lane, largest at lane 0.
+__device__ __forceinline__ float warp_merge_desc(float x, int lane) {
+#pragma unroll
+  for (int j = 16; j > 0; j >>= 1) {
+    const float o = __shfl_xor_sync(0xffffffffu, x, j);
+    x = (lane & j) == 0 ? fmaxf(x, o) : fminf(x, o);
   }
   return x;
 }
@@ -279,17 +291,20 @@ __device__ __forceinline__ float warp_sort_desc(float x, int lane) {
 // shared memory (its whole 16-byte vectors) plus a ragged tail of fewer than
 // 16 bytes read directly, ordered by cand_before, padded with (-inf, -1);
 // columns are absolute. Each lane owns 16 vectors and keeps their maxima in
-// registers. Two thresholds bound the unit's K-th largest element from below:
-//   tau1, the K-th largest of the 32 lane maxima (a bitonic sort; K <= 32);
-//   tau2, the K-th largest vector maximum (K vectors reach it, so at least K
-//   elements do), found among the vectors that reach tau1: by counting when
-//   they are few, else by a radix search over the maxima in registers.
-// Only elements at or above tau2 can be in the list: about K of them, in
-// about K vectors, whatever the spread of the large logits over the lanes.
-// They are gathered in `scratch` and ranked by counting; more than kCandCap
-// (runs of equal logits) take K rounds of a warp-wide extraction over the
-// same vectors instead. The work per unit is thus nearly the same for every
-// unit, which keeps the stage ring from waiting on one slow warp.
+// registers. A threshold at or below the unit's K-th largest element bounds
+// the candidates:
+//   tau1, the K-th largest of the 64 values formed by each lane's two largest
+//   vector maxima (two bitonic sorts and a merge; K <= 32); K vectors reach
+//   it, so K elements do. Usually about K vectors reach tau1 and their
+//   elements at or above it are the candidates.
+//   When more than 32 vectors reach tau1 (large logits crowded into few
+//   lanes), tau2, the K-th largest vector maximum, is found among them: by
+//   counting when they are at most 64, else by a radix search over the maxima
+//   in registers, and about K vectors reach it whatever the crowding.
+// The candidates are gathered in `scratch` and ranked by counting; more than
+// kCandCap (runs of equal logits) take K rounds of a warp-wide extraction over
+// the same vectors instead. The work per unit is thus nearly the same for
+// every unit, which keeps the stage ring from waiting on one slow warp.
 template <int DT>
 __device__ void select_unit(const char* stage, const Desc& d, const RowSet& S, int lane, int K,
                             Cand* scratch, Cand* out) {
@@ -300,106 +315,125 @@ __device__ void select_unit(const char* stage, const Desc& d, const RowSet& S, i
   const uint4* sv = reinterpret_cast<const uint4*>(stage);
   const int col0 = d.chunk * kChunk;
   const int nvec = d.n_smem / VEC;  // whole vectors delivered (the copy moves 16-byte units)
-  // the tail element, NaN where the lane has none (NaN never compares >= and
-  // fmaxf skips it)
+  // this lane's vectors v < nvl lie within the copy
+  const int nvl = max(0, min(NV, (nvec - lane + 31) >> 5));
+  const bool has_tail = lane < d.n - d.n_smem;
+  // the tail element, NaN where the lane has none (NaN never compares >=)
   float zt = kNaN;
-  if (lane < d.n - d.n_smem) {
+  if (has_tail) {
     const char* row = S.data + d.row * S.stride_bytes;
     zt = load_logit<DT>(row, int64_t(col0) + d.n_smem + lane);
   }
-  float vm[NV];  // vector maxima; NaN for a vector past the copy
-  float m = -INFINITY;
+  const uint32_t valid = ((1u << nvl) - 1) | (has_tail ? kTailBit : 0u);
+  float vm[NV];  // vector maxima; -inf for a vector past the copy
+  float m1 = has_tail ? zt : -INFINITY, m2 = -INFINITY;  // the lane's two largest
 #pragma unroll
   for (int v = 0; v < NV; ++v) {
-    const int vi = v * 32 + lane;
-    const float x = vec_max<DT>(sv[vi]);
-    vm[v] = vi < nvec ? x : kNaN;
-    m = fmaxf(m, vm[v]);
+    const float x = vec_max<DT>(sv[v * 32 + lane]);
+    vm[v] = v < nvl ? x : -INFINITY;
+    m2 = fmaxf(m2, fminf(m1, vm[v]));
+    m1 = fmaxf(m1, vm[v]);
   }
-  m = fmaxf(m, zt);
   auto at_or_above = [&](float t) {
     uint32_t f = zt >= t ? kTailBit : 0u;
 #pragma unroll
     for (int v = 0; v < NV; ++v) f |= vm[v] >= t ? (1u << v) : 0u;
-    return f;
+    return f & valid;
   };
-  const float tau1 = __shfl_sync(0xffffffffu, warp_sort_desc(m, lane), K - 1);
-  uint32_t flags = at_or_above(tau1);
-
-  // tau2: the K-th largest maximum; every vector that reaches it reaches tau1
+  // the 32 largest of the 64: half-cleaner of (m1 descending, m2 ascending)
+  const float top = warp_merge_desc(fmaxf(warp_sort<true>(m1, lane), warp_sort<false>(m2, lane)),
+                                    lane);
+  float tau = __shfl_sync(0xffffffffu, top, K - 1);
+  uint32_t flags = at_or_above(tau);
   const int nf = __popc(flags);
-  int incl = nf;
+  const int F1 = int(__reduce_add_sync(0xffffffffu, unsigned(nf)));
+  if (F1 > kDirectCap) {
+    // tau2: the K-th largest maximum; every vector that reaches it reaches tau1
+    if (F1 <= kLevel2Cap) {
+      int incl = nf;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int x = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += x;
+      }
+      float* vals = reinterpret_cast<float*>(scratch);
+      int p = incl - nf;
+#pragma unroll
+      for (int v = 0; v < NV; ++v)
+        if (flags & (1u << v)) vals[p++] = vm[v];
+      if (flags & kTailBit) vals[p] = zt;
+      __syncwarp();
+      // the K-th largest w is the largest with #{values >= w} >= K; lane l
+      // tests values l and l + 32 (NaN: absent)
+      const float w0 = lane < F1 ? vals[lane] : kNaN;
+      const float w1 = lane + 32 < F1 ? vals[lane + 32] : kNaN;
+      int c0 = 0, c1 = 0;
+#pragma unroll 4
+      for (int j = 0; j < F1; ++j) {
+        const float x = vals[j];
+        c0 += x >= w0;
+        c1 += x >= w1;
+      }
+      float best = -INFINITY;
+      if (c0 >= K) best = w0;
+      if (c1 >= K) best = fmaxf(best, w1);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, o));
+      tau = best;
+      __syncwarp();  // the values are read before the scratch takes candidates
+    } else {
+      // radix search on order-preserving keys (x >= 0: bits | 2^31, else
+      // ~bits): the largest key t with #{maxima whose key >= t} >= K, one bit
+      // at a time. A probe's float is compared, so probes below the key of
+      // -inf (NaN floats) never pass: a K-th largest of -inf ends at t = 0.
+      uint32_t t = 0;
+      for (int b = 31; b >= 0; --b) {
+        const uint32_t probe = t | (1u << b);
+        const float pf = __uint_as_float((probe & 0x80000000u) ? (probe & 0x7fffffffu) : ~probe);
+        int c = zt >= pf;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) c += vm[v] >= pf;
+        if (int(__reduce_add_sync(0xffffffffu, unsigned(c))) >= K) t = probe;
+      }
+      tau = t < 0x007fffffu ? -INFINITY
+                            : __uint_as_float((t & 0x80000000u) ? (t & 0x7fffffffu) : ~t);
+    }
+    flags = at_or_above(tau);
+  }
+  const float tau2 = tau;
+
+  // candidates: the elements at or above tau2, counted, then written at their
+  // lane's offset in the warp
+  int nc = (flags & kTailBit) ? 1 : 0;
+  for (uint32_t f = flags & (kTailBit - 1); f; f &= f - 1) {
+    const uint4 w = sv[(__ffs(f) - 1) * 32 + lane];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) nc += lane_elem<DT>(w, q) >= tau2;
+  }
+  int cincl = nc;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const int x = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += x;
+    const int x = __shfl_up_sync(0xffffffffu, cincl, o);
+    if (lane >= o) cincl += x;
   }
-  const int F1 = __shfl_sync(0xffffffffu, incl, 31);
-  float tau2;
-  if (F1 <= kLevel2Cap) {
-    float* vals = reinterpret_cast<float*>(scratch);
-    int p = incl - nf;
-#pragma unroll
-    for (int v = 0; v < NV; ++v)
-      if (flags & (1u << v)) vals[p++] = vm[v];
-    if (flags & kTailBit) vals[p] = zt;
-    __syncwarp();
-    // the K-th largest w is the largest with #{values >= w} >= K (fewer than
-    // K values: none, -inf)
-    float best = -INFINITY;
-    for (int i = lane; i < F1; i += 32) {
-      const float w = vals[i];
-      int c = 0;
-#pragma unroll 4
-      for (int j = 0; j < F1; ++j) c += vals[j] >= w;
-      if (c >= K) best = fmaxf(best, w);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, o));
-    tau2 = best;
-    __syncwarp();  // the values are read before the scratch takes candidates
-  } else {
-    // radix search on order-preserving keys (x >= 0: bits | 2^31, else ~bits):
-    // the largest key t with #{maxima whose key >= t} >= K, one bit at a
-    // time. A probe's float is compared, so probes below the key of -inf
-    // (NaN floats) never pass: a K-th largest of -inf ends at t = 0.
-    uint32_t t = 0;
-    for (int b = 31; b >= 0; --b) {
-      const uint32_t probe = t | (1u << b);
-      const float pf = __uint_as_float((probe & 0x80000000u) ? (probe & 0x7fffffffu) : ~probe);
-      int c = zt >= pf;
-#pragma unroll
-      for (int v = 0; v < NV; ++v) c += vm[v] >= pf;
-      if (int(__reduce_add_sync(0xffffffffu, unsigned(c))) >= K) t = probe;
-    }
-    tau2 = t < 0x007fffffu ? -INFINITY
-                           : __uint_as_float((t & 0x80000000u) ? (t & 0x7fffffffu) : ~t);
-  }
-  flags = at_or_above(tau2);
-
-  int* count = reinterpret_cast<int*>(scratch + kCandCap);
-  if (lane == 0) *count = 0;
-  __syncwarp();
-  auto push = [&](float x, int c) {
-    const int p = atomicAdd(count, 1);
-    if (p < kCandCap) scratch[p] = Cand{x, c};
-  };
-  if (flags & kTailBit) push(zt, d.n_smem + lane);
-  for (uint32_t f = flags & (kTailBit - 1); f; f &= f - 1) {
-    const int v = __ffs(f) - 1;
-    const uint4 w = sv[v * 32 + lane];
-#pragma unroll
-    for (int q = 0; q < VEC; ++q) {
-      const float x = lane_elem<DT>(w, q);
-      if (x >= tau2) push(x, (v * 32 + lane) * VEC + q);
-    }
-  }
-  __syncwarp();
-  const int C = *reinterpret_cast<volatile int*>(count);
+  const int C = __shfl_sync(0xffffffffu, cincl, 31);
   if (C <= kCandCap) {
+    int p = cincl - nc;
+    if (flags & kTailBit) scratch[p++] = Cand{zt, d.n_smem + lane};
+    for (uint32_t f = flags & (kTailBit - 1); f; f &= f - 1) {
+      const int v = __ffs(f) - 1;
+      const uint4 w = sv[v * 32 + lane];
+#pragma unroll
+      for (int q = 0; q < VEC; ++q) {
+        const float x = lane_elem<DT>(w, q);
+        if (x >= tau2) scratch[p++] = Cand{x, (v * 32 + lane) * VEC + q};
+      }
+    }
+    __syncwarp();
     for (int i = lane; i < C; i += 32) {
       const Cand ci = scratch[i];
       int r = 0;
+#pragma unroll 4
       for (int j = 0; j < C; ++j) {
         const Cand cj = scratch[j];
         r += cand_before(cj.v, cj.c, ci.v, ci.c);
@@ -464,7 +498,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
   Desc* desc = reinterpret_cast<Desc*>(empty + R::kStages);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // a consumer warp's candidate scratch (filtered rows only)
-  Cand* scratch = reinterpret_cast<Cand*>(desc + R::kStages) + (SEL ? warp * (kCandCap + 1) : 0);
+  Cand* scratch = reinterpret_cast<Cand*>(desc + R::kStages) + (SEL ? warp * kCandCap : 0);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < R::kStages; ++s) {
