@@ -245,9 +245,99 @@ __device__ void row_topk_wide(const Cand* lists, int nch, int K, int lane, Cand*
   __syncwarp();
 }
 
+constexpr int kPre = 4;  // entries of each list loaded before the threshold is known
+
+// The top-K of one filtered row of nl <= 32 * kMergeLists unit lists, by a
+// threshold. Lane l owns lists l, l + 32, ...; tau, the K-th largest of the
+// 64 values formed by each lane's two largest first-or-second list entries,
+// bounds the row's K-th largest from below (they are 64 distinct elements of
+// the row, so K elements reach tau). Every list entry at or above tau is a candidate: the
+// leading run of each list, usually a little over K entries in all. They are
+// gathered in `scr` and ranked by counting; more than kRowCap (runs of equal
+// logits) take the K-way merge instead.
+__device__ void row_topk_thresh(const Cand* lists, int nl, int K, int lane, Cand* scr,
+                                Cand* top) {
+  Cand e[kMergeLists][kPre];
+  float m1 = -INFINITY, m2 = -INFINITY;  // the lane's two largest heads
+#pragma unroll
+  for (int i = 0; i < kMergeLists; ++i) {
+    const int c = lane + 32 * i;
+#pragma unroll
+    for (int j = 0; j < kPre; ++j)
+      e[i][j] = (c < nl && j < K) ? lists[int64_t(c) * K + j] : Cand{-INFINITY, -1};
+    // a list's first two entries are distinct elements: each lane offers the
+    // two largest first-or-second entries of its lists
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const float h = e[i][j].c >= 0 ? e[i][j].v : -INFINITY;
+      m2 = fmaxf(m2, fminf(m1, h));
+      m1 = fmaxf(m1, h);
+    }
+  }
+  // the 32 largest of the 64: half-cleaner of (m1 descending, m2 ascending)
+  const float top32 =
+      warp_merge_desc(fmaxf(warp_sort<true>(m1, lane), warp_sort<false>(m2, lane)), lane);
+  const float tau = __shfl_sync(0xffffffffu, top32, K - 1);
+  // leading run of each list at or above tau (entries past kPre read here)
+  int cnt[kMergeLists];
+  int nc = 0;
+#pragma unroll
+  for (int i = 0; i < kMergeLists; ++i) {
+    const int c = lane + 32 * i;
+    int k = 0;
+#pragma unroll
+    for (int j = 0; j < kPre; ++j) k += (k == j && e[i][j].c >= 0 && e[i][j].v >= tau) ? 1 : 0;
+    if (k == kPre && c < nl) {
+      // the run may go on: a list is ordered, so counting its entries at or
+      // above tau gives the run's length, with independent loads
+#pragma unroll 8
+      for (int j = kPre; j < K; ++j) {
+        const Cand x = lists[int64_t(c) * K + j];
+        k += (x.c >= 0 && x.v >= tau) ? 1 : 0;
+      }
+    }
+    cnt[i] = k;
+    nc += k;
+  }
+  int incl = nc;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int x = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += x;
+  }
+  const int C = __shfl_sync(0xffffffffu, incl, 31);
+  if (C > kRowCap) {
+    row_topk_merge(lists, nl, K, lane, top);
+    return;
+  }
+  int p = incl - nc;
+#pragma unroll
+  for (int i = 0; i < kMergeLists; ++i) {
+    const int c = lane + 32 * i;
+#pragma unroll
+    for (int j = 0; j < kPre; ++j)
+      if (j < cnt[i]) scr[p++] = e[i][j];
+#pragma unroll 4
+    for (int j = kPre; j < cnt[i]; ++j) scr[p++] = lists[int64_t(c) * K + j];
+  }
+  __syncwarp();
+  for (int i = lane; i < C; i += 32) {
+    const Cand ci = scr[i];
+    int r = 0;
+#pragma unroll 4
+    for (int j = 0; j < C; ++j) {
+      const Cand cj = scr[j];
+      r += cand_before(cj.v, cj.c, ci.v, ci.c);
+    }
+    if (r < K) top[r] = ci;
+  }
+  for (int r = C + lane; r < K; r += 32) top[r] = Cand{-INFINITY, -1};
+  __syncwarp();
+}
+
 __device__ __forceinline__ void row_topk(const Cand* lists, int nch, int K, int lane, Cand* scr,
                                          Cand* top) {
-  if (nch <= 32 * kMergeLists) row_topk_merge(lists, nch, K, lane, top);
+  if (nch <= 32 * kMergeLists) row_topk_thresh(lists, nch, K, lane, scr, top);
   else row_topk_wide(lists, nch, K, lane, scr, top);
 }
 
@@ -274,9 +364,8 @@ __device__ int kept_set(const Cand* top, int K, float scale, float top_p, int la
   // top-p: keep while the mass before the token is below top_p
   const bool keep = valid && (!(top_p < 1.f) || f2_lt(before, f2_mul_f(all, top_p)));
   const unsigned km = __ballot_sync(0xffffffffu, keep);
-  const int n = __popc(km);  // a prefix of the lanes
-  const F2 kept_incl = warp_scan_f2(F2{keep ? e : 0.f, 0.f}, lane);
-  const float S = __shfl_sync(0xffffffffu, __fadd_rn(kept_incl.hi, kept_incl.lo), 31);
+  const int n = __popc(km);  // a prefix of the lanes, so the kept sum is the prefix at n - 1
+  const float S = __shfl_sync(0xffffffffu, __fadd_rn(incl.hi, incl.lo), n > 0 ? n - 1 : 0);
   col = keep ? me.c : -1;
   prob = keep ? e * __frcp_rn(S) : 0.f;
   lse = (M + lg2_approx(S)) * 0.6931471805599453f;

@@ -260,6 +260,36 @@ __device__ __forceinline__ void report_error(int32_t* err, int32_t epoch, int32_
   atomicExch(&err[0], epoch);
 }
 
+// ------------------------------------------------------------ warp sorting
+
+// Bitonic sort of one value per lane across the warp: largest at lane 0
+// (DESC) or smallest at lane 0.
+template <bool DESC>
+__device__ __forceinline__ float warp_sort(float x, int lane) {
+#pragma unroll
+  for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      const float o = __shfl_xor_sync(0xffffffffu, x, j);
+      // lanes [i, i + k) form a run sorted descending when (i & k) == 0 (k = 32:
+      // the whole warp); the lower lane of a pair keeps the larger value there
+      const bool up = ((lane & j) == 0) == (k == 32 || (lane & k) == 0);
+      x = (DESC ? up : !up) ? fmaxf(x, o) : fminf(x, o);
+    }
+  }
+  return x;
+}
+
+// Sorts a bitonic sequence held one value per lane, largest at lane 0.
+__device__ __forceinline__ float warp_merge_desc(float x, int lane) {
+#pragma unroll
+  for (int j = 16; j > 0; j >>= 1) {
+    const float o = __shfl_xor_sync(0xffffffffu, x, j);
+    x = (lane & j) == 0 ? fmaxf(x, o) : fminf(x, o);
+  }
+  return x;
+}
+
 // ------------------------------------------------------------ CSR helpers
 
 // Offsets of request b are usable: 0 <= off[b] <= off[b+1] <= n.
