@@ -8,7 +8,7 @@
  *                  draft tokens D = (d_1..d_k) and its proxy target tokens
  *                  T = (t_1..t_m) = encode_t(decode_d(D)) (§4.2, App. A.1),
  *                  with the Levenshtein distance over the tokens' UTF-8 bytes as
- *                  the local cost (App. F) and a Sakoe-Chiba band (§4.1);
+ *                  the local cost (App. H) and a Sakoe-Chiba band (§4.1);
  *   (b) transfer -- MapProbabilities (Alg. 2, App. A.2): target position j
  *                  takes the draft probability of the last draft token aligned
  *                  to it (terminal rule / copy rule), one-hot (Limitations);
@@ -103,7 +103,7 @@ typedef struct {
 
 typedef struct {
   int32_t window;      /* Sakoe-Chiba half-width w >= 0 (the paper settles on 8,
-                          App. G); negative = no band. The band used for a request
+                          App. K); negative = no band. The band used for a request
                           is max(w, |k - m|) so that (k, m) stays reachable. */
   float temp_draft;    /* T_d > 0: draft rows are softmax(z / T_d) */
   float temp_target;   /* T_t > 0: target rows are softmax(z / T_t) */
@@ -116,7 +116,7 @@ typedef struct {
   void* const* events; /* host array of 4 cudaEvent_t or NULL: tt_step records
                           them before align, before the row pass, before the
                           decision kernel and after it (profiling only) */
-  /* Sampling filters of the paper's generation hyperparameters, per family,
+  /* Sampling filters of the paper's generation hyperparameters (App. F), per family,
      after the temperature: keep the top_k largest logits of a row (0 = off,
      at most TT_MAX_TOP_K; among equal logits the smaller column first), then
      keep tokens in decreasing probability while the mass before a token is
@@ -166,12 +166,13 @@ typedef struct {
  * 256-byte aligned pointer. */
 size_t tt_workspace_bytes(const tt_batch* batch, int32_t V_d, int32_t V_t);
 
-/* The same with the sampling filters of `prm` (a filtered family keeps
- * top_k candidates of 8 bytes per 2048-column chunk of each row). */
+/* The same with the sampling filters of `prm` (a filtered family keeps, per
+ * row, top_k candidates of 8 bytes per unit of 8 KB of logits -- 2048 fp32
+ * or 4096 bf16 columns -- and its kept set of top_k entries of 8 bytes). */
 size_t tt_workspace_bytes_for(const tt_batch* batch, int32_t V_d, int32_t V_t,
                               const tt_params* prm);
 
-/* (a) DTW alignment (§4.1, Alg. 1; App. F token distance).
+/* (a) DTW alignment (§4.1, Alg. 1; App. H token distance).
  * Per request: local cost d(i,j) = Levenshtein distance between the byte
  * strings of d_i (in vd) and t_j (in vt), for cells inside the band;
  * C_{0,0} = 0, border and out-of-band cells infinite,
@@ -250,7 +251,7 @@ tt_status tt_step_noalloc(const tt_batch* batch, const tt_vocab* vd, const tt_vo
 
 /* Static text for a tt_status. */
 /* ------------------------------------------------------------------------
- * Re-encoding and its checks (§4.2; App. A.1, Lemma 1; §4.1 and App. G).
+ * Re-encoding and its checks (§4.2; App. A.1, Lemma 1; §4.1 and App. K).
  * ---------------------------------------------------------------------- */
 
 /* Size of the re-encoding index of a vocabulary with n_tokens tokens and
@@ -299,7 +300,7 @@ tt_status tt_encode(int32_t B, int32_t n_draft, const int32_t* draft_off, const 
 tt_status tt_consistency(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
                          int32_t* status, void* stream);
 
-/* Delta-pos (§4.1, App. G), the position deviation of DTW-matched tokens,
+/* Delta-pos (§4.1, App. K), the position deviation of DTW-matched tokens,
  * counted into hist[min(delta, n_bins - 1)] (int64, device, ADDED to: zero it
  * before the first call; many steps can be accumulated). mode 0: delta = |i - j|
  * for every pair on each request's path (tt_align's path / path_len); mode 1:

@@ -12,7 +12,7 @@
  *  - Band: |i - j| <= w_eff with w_eff = max(w, |k - m|), so (k, m) is always
  *    reachable; w < 0 means no band (§4.1 band, Alg. 1).
  *  - Backtrack ties: prefer (i-1, j-1), then (i-1, j), then (i, j-1).
- *  - Token distance is Levenshtein over the tokens' UTF-8 bytes (App. F, and
+ *  - Token distance is Levenshtein over the tokens' UTF-8 bytes (App. H, and
  *    the byte-level resolution of the fragmented-tokenization study).
  *  - Transfer: target position j takes the draft token with the largest i
  *    aligned to it (terminal rule for many-to-one, copy rule for one-to-many,
@@ -41,7 +41,7 @@
 #define MAX_TOKEN_BYTES 256
 #define BOUNDARY_EPS 1e-6
 
-/* ------------------------------------------------------------------ App. F */
+/* ------------------------------------------------------------------ App. H */
 
 int32_t tto_lev(const uint8_t* s, int32_t ns, const uint8_t* t, int32_t nt) {
   /* D(i,0) = i, D(0,j) = j; D(i,j) = min(D(i-1,j)+1, D(i,j-1)+1,

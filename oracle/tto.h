@@ -22,7 +22,7 @@
 extern "C" {
 #endif
 
-/* App. F: Levenshtein distance between byte strings, unit costs. */
+/* App. H: Levenshtein distance between byte strings, unit costs. */
 int32_t tto_lev(const uint8_t* s, int32_t ns, const uint8_t* t, int32_t nt);
 
 /* Alg. 1 on a given k x m local cost matrix d (row-major, d[i*m+j] =
@@ -42,7 +42,7 @@ double tto_uniform(uint64_t seed, uint64_t pos, uint64_t stream, uint64_t reques
 void tto_softmax(const void* row, int32_t dtype, int64_t V, double T, double* p_out);
 double tto_logsumexp(const void* row, int32_t dtype, int64_t V, double T);
 
-/* Batched DTW alignment (§4.1, Alg. 1, App. F). Outputs are per request:
+/* Batched DTW alignment (§4.1, Alg. 1, App. H). Outputs are per request:
  * path pairs at pair offset draft_off[b] + target_off[b], path_len[b],
  * cost[b] = C*, map[j] = max{i : (i,j) on the path} for the request's target
  * positions, status[b]. */
@@ -134,7 +134,7 @@ void tto_consistency(int32_t B, const int32_t* draft_off, const int32_t* draft_i
                      const uint8_t* vt_bytes, const int64_t* vt_off, int32_t Vt,
                      int32_t max_k, int32_t max_m, int32_t* status);
 
-/* Delta-pos (§4.1, App. G): the position deviation |i - j| of matched tokens,
+/* Delta-pos (§4.1, App. K): the position deviation |i - j| of matched tokens,
  * counted into hist[min(|i - j|, n_bins - 1)] (hist is added to, not cleared).
  * mode 0: every (i, j) on each request's DTW path; mode 1: every target
  * position j with its mapped draft index map[j]. Requests with path_len[b] == 0

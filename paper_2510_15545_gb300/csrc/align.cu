@@ -1,5 +1,5 @@
 // align.cu -- Dynamic Token Warping between draft and proxy target tokens
-// (§4.1, Alg. 1) with the byte-level Levenshtein token distance (App. F).
+// (§4.1, Alg. 1) with the byte-level Levenshtein token distance (App. H).
 //
 // One warp per request (sequence pair), several pairs per CTA. Per pair:
 //  1. stage the tokens' byte strings in shared memory (packed 8-byte words);

@@ -1,6 +1,6 @@
 // encode.cu -- re-encoding of the draft string into target tokens (§4.2,
 // App. A.1), the Lemma-1 byte check (App. A.1) and the delta-pos histogram of
-// the DTW paths (§4.1, App. G).
+// the DTW paths (§4.1, App. K).
 //
 // Re-encoding is greedy longest match over the target vocabulary, through an
 // index of every prefix of every token: an open-addressing table whose slot

@@ -108,15 +108,15 @@ constexpr int kMergeLists = 4;  // lists a lane owns in the K-way merge (rows of
 // next entry in registers; every round a warp-wide arg-best takes the winner
 // and its owner advances that list, loading the entry after next. Exact, no
 // candidate buffer. Rows of more than 32 * kMergeLists units use row_topk_wide.
-__device__ void row_topk_merge(const Cand* lists, int nch, int K, int lane, Cand* top) {
+__device__ void row_topk_merge(const Cand* lists, int nch, int K, int Ls, int lane, Cand* top) {
   Cand cur[kMergeLists], nxt[kMergeLists];
   int pos[kMergeLists];
 #pragma unroll
   for (int i = 0; i < kMergeLists; ++i) {
     const int c = lane + 32 * i;
     const bool ok = c < nch;
-    cur[i] = ok ? lists[int64_t(c) * K] : Cand{-INFINITY, -1};
-    nxt[i] = ok && K > 1 ? lists[int64_t(c) * K + 1] : Cand{-INFINITY, -1};
+    cur[i] = ok ? lists[int64_t(c) * Ls] : Cand{-INFINITY, -1};
+    nxt[i] = ok && K > 1 ? lists[int64_t(c) * Ls + 1] : Cand{-INFINITY, -1};
     pos[i] = 1;  // index of nxt in its list
   }
   for (int r = 0; r < K; ++r) {
@@ -144,7 +144,7 @@ __device__ void row_topk_merge(const Cand* lists, int nch, int K, int lane, Cand
           cur[i] = nxt[i];
           ++pos[i];
           const int c = lane + 32 * i;
-          nxt[i] = pos[i] < K ? lists[int64_t(c) * K + pos[i]] : Cand{-INFINITY, -1};
+          nxt[i] = pos[i] < K ? lists[int64_t(c) * Ls + pos[i]] : Cand{-INFINITY, -1};
         }
     }
   }
@@ -154,7 +154,8 @@ __device__ void row_topk_merge(const Cand* lists, int nch, int K, int lane, Cand
 // The top-K of one filtered row (its nch unit lists of K entries merged),
 // ordered by cand_before, padded with (-inf, -1). One warp; `scr` holds
 // kRowCap candidates, `top` K entries (shared memory). For rows of many units.
-__device__ void row_topk_wide(const Cand* lists, int nch, int K, int lane, Cand* scr, Cand* top) {
+__device__ void row_topk_wide(const Cand* lists, int nch, int K, int Ls, int lane, Cand* scr,
+                              Cand* top) {
   // tau: the K-th best list head (fewer than K heads: every entry counts)
   float tau = -INFINITY;
   {
@@ -165,7 +166,7 @@ __device__ void row_topk_wide(const Cand* lists, int nch, int K, int lane, Cand*
       int bc = 0x7fffffff;
       bool f = false;
       for (int c = lane; c < nch; c += 32) {
-        const Cand h = lists[int64_t(c) * K];
+        const Cand h = lists[int64_t(c) * Ls];
         if (h.c >= 0 && cand_before(pv, pc, h.v, h.c) && (!f || cand_before(h.v, h.c, bv, bc))) {
           bv = h.v;
           bc = h.c;
@@ -186,7 +187,7 @@ __device__ void row_topk_wide(const Cand* lists, int nch, int K, int lane, Cand*
   int cnt = 0;
   for (int c = lane; c < nch; c += 32)
     for (int i = 0; i < K; ++i) {
-      const Cand x = lists[int64_t(c) * K + i];
+      const Cand x = lists[int64_t(c) * Ls + i];
       if (x.c < 0 || x.v < tau) break;
       ++cnt;
     }
@@ -201,7 +202,7 @@ __device__ void row_topk_wide(const Cand* lists, int nch, int K, int lane, Cand*
     int pos = incl - cnt;
     for (int c = lane; c < nch; c += 32)
       for (int i = 0; i < K; ++i) {
-        const Cand x = lists[int64_t(c) * K + i];
+        const Cand x = lists[int64_t(c) * Ls + i];
         if (x.c < 0 || x.v < tau) break;
         scr[pos++] = x;
       }
@@ -223,7 +224,7 @@ __device__ void row_topk_wide(const Cand* lists, int nch, int K, int lane, Cand*
       bool f = false;
       for (int c = lane; c < nch; c += 32)
         for (int i = 0; i < K; ++i) {
-          const Cand x = lists[int64_t(c) * K + i];
+          const Cand x = lists[int64_t(c) * Ls + i];
           if (x.c < 0) break;
           if (cand_before(pv, pc, x.v, x.c) && (!f || cand_before(x.v, x.c, bv, bc))) {
             bv = x.v;
@@ -246,6 +247,7 @@ __device__ void row_topk_wide(const Cand* lists, int nch, int K, int lane, Cand*
 }
 
 constexpr int kPre = 4;  // entries of each list loaded before the threshold is known
+static_assert(kPre == 4, "the first entries are loaded as two 16-byte pairs");
 
 // The top-K of one filtered row of nl <= 32 * kMergeLists unit lists, by a
 // threshold. Lane l owns lists l, l + 32, ...; tau, the K-th largest of the
@@ -255,16 +257,28 @@ constexpr int kPre = 4;  // entries of each list loaded before the threshold is 
 // leading run of each list, usually a little over K entries in all. They are
 // gathered in `scr` and ranked by counting; more than kRowCap (runs of equal
 // logits) take the K-way merge instead.
-__device__ void row_topk_thresh(const Cand* lists, int nl, int K, int lane, Cand* scr,
+__device__ void row_topk_thresh(const Cand* lists, int nl, int K, int Ls, int lane, Cand* scr,
                                 Cand* top) {
   Cand e[kMergeLists][kPre];
   float m1 = -INFINITY, m2 = -INFINITY;  // the lane's two largest heads
+  const Cand pad = {-INFINITY, -1};
 #pragma unroll
   for (int i = 0; i < kMergeLists; ++i) {
     const int c = lane + 32 * i;
-#pragma unroll
-    for (int j = 0; j < kPre; ++j)
-      e[i][j] = (c < nl && j < K) ? lists[int64_t(c) * K + j] : Cand{-INFINITY, -1};
+    // entries 0-3 as two 16-byte loads (a list starts on a 16-byte boundary
+    // and holds an even number of slots; slots past K are not read)
+    e[i][0] = e[i][1] = e[i][2] = e[i][3] = pad;
+    if (c < nl) {
+      const uint4* L = reinterpret_cast<const uint4*>(lists + int64_t(c) * Ls);
+      const uint4 a = L[0];
+      e[i][0] = Cand{__uint_as_float(a.x), int32_t(a.y)};
+      if (K > 1) e[i][1] = Cand{__uint_as_float(a.z), int32_t(a.w)};
+      if (K > 2) {
+        const uint4 b = L[1];
+        e[i][2] = Cand{__uint_as_float(b.x), int32_t(b.y)};
+        if (K > 3) e[i][3] = Cand{__uint_as_float(b.z), int32_t(b.w)};
+      }
+    }
     // a list's first two entries are distinct elements: each lane offers the
     // two largest first-or-second entries of its lists
 #pragma unroll
@@ -292,7 +306,7 @@ __device__ void row_topk_thresh(const Cand* lists, int nl, int K, int lane, Cand
       // above tau gives the run's length, with independent loads
 #pragma unroll 8
       for (int j = kPre; j < K; ++j) {
-        const Cand x = lists[int64_t(c) * K + j];
+        const Cand x = lists[int64_t(c) * Ls + j];
         k += (x.c >= 0 && x.v >= tau) ? 1 : 0;
       }
     }
@@ -307,7 +321,7 @@ __device__ void row_topk_thresh(const Cand* lists, int nl, int K, int lane, Cand
   }
   const int C = __shfl_sync(0xffffffffu, incl, 31);
   if (C > kRowCap) {
-    row_topk_merge(lists, nl, K, lane, top);
+    row_topk_merge(lists, nl, K, Ls, lane, top);
     return;
   }
   int p = incl - nc;
@@ -318,7 +332,7 @@ __device__ void row_topk_thresh(const Cand* lists, int nl, int K, int lane, Cand
     for (int j = 0; j < kPre; ++j)
       if (j < cnt[i]) scr[p++] = e[i][j];
 #pragma unroll 4
-    for (int j = kPre; j < cnt[i]; ++j) scr[p++] = lists[int64_t(c) * K + j];
+    for (int j = kPre; j < cnt[i]; ++j) scr[p++] = lists[int64_t(c) * Ls + j];
   }
   __syncwarp();
   for (int i = lane; i < C; i += 32) {
@@ -335,10 +349,50 @@ __device__ void row_topk_thresh(const Cand* lists, int nl, int K, int lane, Cand
   __syncwarp();
 }
 
-__device__ __forceinline__ void row_topk(const Cand* lists, int nch, int K, int lane, Cand* scr,
-                                         Cand* top) {
-  if (nch <= 32 * kMergeLists) row_topk_thresh(lists, nch, K, lane, scr, top);
-  else row_topk_wide(lists, nch, K, lane, scr, top);
+// The top-K of a row of at most 64 list entries (nl * K <= 64): every entry
+// is a candidate, loaded one or two per lane. Entry s (place s % K of list
+// s / K) comes after the s % K entries ahead of it in its own list (a list's
+// real entries lead it) and after those entries of the other lists that
+// cand_before puts first.
+__device__ void row_topk_small(const Cand* lists, int nl, int K, int Ls, int lane, Cand* scr,
+                               Cand* top) {
+  const int n = nl * K;
+  Cand x[2];
+  int own[2], place[2];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int s = lane + 32 * h;
+    own[h] = s / K;
+    place[h] = s - own[h] * K;
+    x[h] = s < n ? lists[int64_t(own[h]) * Ls + place[h]] : Cand{-INFINITY, -1};
+    scr[s] = x[h];
+  }
+  __syncwarp();
+  const int nvalid = __popc(__ballot_sync(0xffffffffu, x[0].c >= 0)) +
+                     __popc(__ballot_sync(0xffffffffu, x[1].c >= 0));
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    if (x[h].c < 0) continue;
+    int r = place[h];
+    for (int l = 0; l < nl; ++l) {
+      if (l == own[h]) continue;
+#pragma unroll 4
+      for (int j = 0; j < K; ++j) {
+        const Cand y = scr[l * K + j];
+        r += (y.c >= 0 && cand_before(y.v, y.c, x[h].v, x[h].c)) ? 1 : 0;
+      }
+    }
+    if (r < K) top[r] = x[h];
+  }
+  for (int r = nvalid + lane; r < K; r += 32) top[r] = Cand{-INFINITY, -1};
+  __syncwarp();
+}
+
+__device__ __forceinline__ void row_topk(const Cand* lists, int nch, int K, int Ls, int lane,
+                                         Cand* scr, Cand* top) {
+  if (nch * K <= 64) row_topk_small(lists, nch, K, Ls, lane, scr, top);
+  else if (nch <= 32 * kMergeLists) row_topk_thresh(lists, nch, K, Ls, lane, scr, top);
+  else row_topk_wide(lists, nch, K, Ls, lane, scr, top);
 }
 
 // The kept set of a filtered row from its top-K (in shared memory): lane i < n
@@ -404,7 +458,8 @@ __global__ void __launch_bounds__(kFThreads) kept_kernel(KeptArgs a) {
     const RowSet& S = tgt ? a.t : a.d;
     if (!tgt && S.need && S.need[row] == 0) continue;
     const int K = S.top_k;
-    row_topk(S.cand + row * S.nlist * K, S.nlist, K, lane, s_scr[warp], s_top[warp]);
+    const int Ls = cand_stride(K);
+    row_topk(S.cand + row * S.nlist * Ls, S.nlist, K, Ls, lane, s_scr[warp], s_top[warp]);
     int col;
     float prob, lse;
     const int n = kept_set(s_top[warp], K, S.scale, tgt ? a.top_p_t : a.top_p_d, lane, col,

@@ -658,7 +658,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
     const int esz = (d.set ? DTT : DTD) == TT_F32 ? 4 : 2;
     if (SEL && (d.set ? a.t : a.d).top_k > 0) {  // filtered rows: the unit's top-k list
       const RowSet& S = d.set ? a.t : a.d;
-      Cand* out = S.cand + (d.row * S.nlist + d.chunk / cps) * S.top_k;
+      Cand* out = S.cand + (d.row * S.nlist + d.chunk / cps) * cand_stride(S.top_k);
       if (d.set) {
         select_unit<DTT>(stage, d, a.t, lane, S.top_k, scratch, out);
       } else {

@@ -34,6 +34,10 @@ struct Cand {
   int32_t c;
 };
 
+// Entries between the starts of two consecutive top-k lists: k rounded up to
+// an even count, so that every list starts on a 16-byte boundary.
+__host__ __device__ inline int cand_stride(int k) { return k + (k & 1); }
+
 // Header of a filtered row's kept set (the set itself is k Cand entries
 // holding (probability, column), larger logit first, unused entries (0, -1)):
 // natural log of the kept normaliser, and the kept count (0: not finite).
@@ -58,8 +62,8 @@ struct Workspace {
   int32_t* err;      // two words: epoch of a call whose row pass failed, and why
   unsigned long long* work;  // row-pass work counters (kWorkShards, kWorkStride apart), zeroed
                              // by the kernel before the row pass
-  Cand* cand_d;      // [n_draft * nch_d * k_d] top-k lists of filtered draft rows
-  Cand* cand_t;      // [(n_target + B) * nch_t * k_t] top-k lists of filtered target rows
+  Cand* cand_d;      // [n_draft * nch_d * cand_stride(k_d)] top-k lists of filtered draft rows
+  Cand* cand_t;      // [(n_target + B) * nch_t * cand_stride(k_t)] top-k lists of filtered target rows
   Cand* kept_d;      // [n_draft * k_d] kept sets (probability, column) of filtered draft rows
   Cand* kept_t;      // [(n_target + B) * k_t] kept sets of filtered target rows
   KeptHead* head_d;  // [n_draft] their headers
@@ -89,9 +93,9 @@ __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_d
   w.err = reinterpret_cast<int32_t*>(take(2 * sizeof(int32_t)));
   w.work = reinterpret_cast<unsigned long long*>(take(kWorkShards * kWorkStride * sizeof(unsigned long long)));
   w.cand_d = reinterpret_cast<Cand*>(
-      take(sizeof(Cand) * size_t(n_draft) * n_chunks(V_d) * size_t(k_d > 0 ? k_d : 0)));
+      take(sizeof(Cand) * size_t(n_draft) * n_chunks(V_d) * size_t(k_d > 0 ? cand_stride(k_d) : 0)));
   w.cand_t = reinterpret_cast<Cand*>(
-      take(sizeof(Cand) * size_t(n_target + B) * n_chunks(V_t) * size_t(k_t > 0 ? k_t : 0)));
+      take(sizeof(Cand) * size_t(n_target + B) * n_chunks(V_t) * size_t(k_t > 0 ? cand_stride(k_t) : 0)));
   w.kept_d = reinterpret_cast<Cand*>(take(sizeof(Cand) * size_t(n_draft) * size_t(k_d > 0 ? k_d : 0)));
   w.kept_t = reinterpret_cast<Cand*>(
       take(sizeof(Cand) * size_t(n_target + B) * size_t(k_t > 0 ? k_t : 0)));

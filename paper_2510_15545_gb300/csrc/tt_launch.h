@@ -47,7 +47,7 @@ struct RowSet {
   Partial* part;
   const uint8_t* need;  // rows to visit (NULL = all)
   int top_k;            // > 0: filtered rows, the row pass writes top-k lists to cand
-  Cand* cand;           // [n_rows * nlist * top_k]: one list per row unit
+  Cand* cand;           // [n_rows * nlist * cand_stride(top_k)]: one list per row unit
   int nlist;            // units (8 KB stages: 2048 fp32 or 4096 bf16 columns) per row
 };
 

@@ -1,4 +1,4 @@
-"""Pins of the oracle's token distance and DTW (App. F, §4.1, Alg. 1) against
+"""Pins of the oracle's token distance and DTW (App. H, §4.1, Alg. 1) against
 facts that do not come from the oracle itself: textbook values, the edit
 distance's own definition searched by brute force, the worked example printed
 in the paper, and exhaustive enumeration of warping paths."""
@@ -34,7 +34,7 @@ def test_lev_textbook_values(s, t, d):
 
 def _edit_distance_bfs(s: bytes, t: bytes, alphabet: bytes) -> int:
     """Minimum number of single-byte insertions, deletions and substitutions
-    turning s into t, by breadth-first search over strings (App. F's definition
+    turning s into t, by breadth-first search over strings (App. H's definition
     of the distance, independent of its dynamic program)."""
     limit = len(s) + len(t)
     seen = {s: 0}

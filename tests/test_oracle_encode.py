@@ -4,7 +4,7 @@ Re-encoding (section 4.2, App. A.1): T = encode_t(decode_d(D)) with greedy
 longest match over the target vocabulary's byte strings. Pins: the paper's
 'Scaling' example (section 2), brute-force maximality and Lemma 1 on random
 vocabularies, agreement with the workload generator's own greedy encoder on the
-synthetic vocabularies, and the status rules. Delta-pos (section 4.1, App. G):
+synthetic vocabularies, and the status rules. Delta-pos (section 4.1, App. K):
 hand-counted histograms of the Fig. 2 path.
 """
 import json
