@@ -311,6 +311,50 @@ tt_status tt_dpos_hist(const tt_batch* batch, const int32_t* path, const int32_t
                        const int32_t* map, int32_t mode, int32_t n_bins, int64_t* hist,
                        void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Vocabulary-sharded verification, emulated on one GPU.
+ *
+ * A tensor-parallel target model leaves each rank with a column slice of every
+ * target logits row. The verification step (c) then needs one exchange: every
+ * rank reduces its slice of each row to a summary (its max and sum of
+ * exponentials with the scored token left out, and the scored token's logit
+ * if the rank owns it); the summaries of all ranks are gathered; the merged
+ * normalisers give p(t_j) and the accept test exactly as in tt_verify; the
+ * residual row's mass per shard picks the shard that holds the drawn point,
+ * and only that shard's slice is read again to find the column.
+ * tt_verify_sharded runs that protocol with the S shards as S logits arrays on
+ * one device: each shard's slice is reduced by its own row pass, and the
+ * gathered summaries are a device buffer in the layout an all-gather would
+ * produce ([S][n_target + B] records of 16 bytes). Results equal tt_verify's
+ * on the concatenated rows up to rounding (same uniforms, same column order).
+ * One-hot transfer only, no sampling filters (TT_ERR_UNSUPPORTED otherwise).
+ */
+#define TT_MAX_SHARDS 8
+
+typedef struct {
+  int32_t S;                /* shards, 1 .. TT_MAX_SHARDS */
+  const tt_logits* shards;  /* HOST array of S descriptors; shard s holds columns
+                               col0[s] .. col0[s] + shards[s].n_cols - 1 of every
+                               target row (n_target + B rows, as in tt_verify) */
+  const int32_t* col0;      /* HOST array of S first columns: col0[0] = 0 and the
+                               shards tile the row in order without gaps */
+} tt_shards;
+
+/* Scratch bytes of tt_verify_sharded (256-byte aligned size). */
+size_t tt_sharded_workspace_bytes(const tt_batch* batch, const tt_shards* target);
+
+/* Verification over sharded target rows. q_hat [n_target] as for tt_verify;
+ * accepted / next_token / status [B], p_hat [n_target] and lse [n_target + B]
+ * (both optional) as for tt_verify; next_token is a column of the whole row.
+ * summaries (optional, [S * (n_target + B) * 4] floats) receives the gathered
+ * per-shard records (max and sum of 2^(z * log2(e) / T - max) over the shard's
+ * columns without the scored one, that sum's low word, and the scored
+ * token's scaled logit or NaN), for inspection. */
+tt_status tt_verify_sharded(const tt_batch* batch, const float* q_hat, const tt_shards* target,
+                            const tt_params* prm, void* workspace, size_t workspace_bytes,
+                            int32_t* accepted, int32_t* next_token, float* p_hat, float* lse,
+                            float* summaries, int32_t* status, void* stream);
+
 const char* tt_status_string(tt_status s);
 
 /* cudaError_t of the last failed launch in this process (0 if none). */

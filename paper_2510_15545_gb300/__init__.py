@@ -8,11 +8,11 @@ missing build raises."""
 from .binding import (Batch, Params, StepCall, TTError, VocabTable, device_inputs, load,
                       step_outputs, tt_align, tt_consistency, tt_dpos_hist, tt_encode,
                       tt_encode_workspace_bytes, tt_status_string, tt_step, tt_step_noalloc,
-                      tt_transfer, tt_verify, tt_version, tt_workspace_bytes, vocab_index,
+                      tt_transfer, tt_verify, tt_verify_sharded, tt_version, tt_workspace_bytes, vocab_index,
                       workspace)
 
 __all__ = ["Batch", "Params", "StepCall", "TTError", "VocabTable", "device_inputs", "load",
            "step_outputs", "tt_align", "tt_consistency", "tt_dpos_hist", "tt_encode",
            "tt_encode_workspace_bytes", "tt_status_string", "tt_step", "tt_step_noalloc",
-           "tt_transfer", "tt_verify", "tt_version", "tt_workspace_bytes", "vocab_index",
+           "tt_transfer", "tt_verify", "tt_verify_sharded", "tt_version", "tt_workspace_bytes", "vocab_index",
            "workspace"]

@@ -41,6 +41,10 @@ class _Logits(ctypes.Structure):
                 ("n_rows", c_i64)]
 
 
+class _Shards(ctypes.Structure):
+    _fields_ = [("S", c_i32), ("shards", ctypes.POINTER(_Logits)), ("col0", ctypes.POINTER(c_i32))]
+
+
 class _Params(ctypes.Structure):
     _fields_ = [("window", c_i32), ("temp_draft", c_f32), ("temp_target", c_f32),
                 ("full_q", c_i32), ("seed", c_u64), ("request_base", c_u64), ("events", c_p),
@@ -64,7 +68,9 @@ _lib = None
 EXPORTS = ("tt_workspace_bytes", "tt_workspace_bytes_for", "tt_align", "tt_transfer", "tt_verify", "tt_step",
            "tt_step_noalloc", "tt_status_string", "tt_last_cuda_error", "tt_version",
            "tt_vocab_index_bytes", "tt_vocab_index_build", "tt_encode_workspace_bytes",
-           "tt_encode", "tt_consistency", "tt_dpos_hist")
+           "tt_encode", "tt_consistency", "tt_dpos_hist", "tt_sharded_workspace_bytes",
+           "tt_verify_sharded")
+TT_MAX_SHARDS = 8
 TT_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
@@ -104,6 +110,11 @@ def load(build_if_missing: bool = False):
     L.tt_step_noalloc.argtypes = [P(_Batch), P(_Vocab), P(_Vocab), P(_Logits), c_p, P(_Logits),
                                   P(_Params), P(_StepOut), c_p]
     L.tt_step_noalloc.restype = c_i32
+    L.tt_sharded_workspace_bytes.argtypes = [P(_Batch), P(_Shards)]
+    L.tt_sharded_workspace_bytes.restype = ctypes.c_size_t
+    L.tt_verify_sharded.argtypes = [P(_Batch), c_p, P(_Shards), P(_Params), c_p, ctypes.c_size_t,
+                                    c_p, c_p, c_p, c_p, c_p, c_p, c_p]
+    L.tt_verify_sharded.restype = c_i32
     L.tt_status_string.argtypes = [c_i32]
     L.tt_status_string.restype = ctypes.c_char_p
     L.tt_last_cuda_error.argtypes = []
@@ -330,6 +341,54 @@ def tt_verify(batch: Batch, q_hat: torch.Tensor, target_logits: torch.Tensor, pa
                             _ptr(o["accepted"]), _ptr(o["next_token"]), _ptr(o["p_hat"]),
                             _ptr(o["lse"]), _ptr(o["status"]), _stream(stream))
     _check("tt_verify", code)
+    return o
+
+
+def _shards(shards):
+    """ctypes view of a list of per-shard logits tensors (columns in order)."""
+    S = len(shards)
+    arr = (_Logits * max(S, 1))()
+    col0 = (c_i32 * max(S, 1))()
+    c = 0
+    for k, t in enumerate(shards):
+        arr[k] = _logits(t)
+        col0[k] = c
+        c += t.shape[1]
+    return _Shards(S, arr, col0), (arr, col0)
+
+
+def tt_verify_sharded(batch: Batch, q_hat: torch.Tensor, shards, params: Params, *,
+                      ws=None, out=None, stream=None, summaries: bool = False) -> dict:
+    """Verification over target rows split by columns into len(shards) logits
+    tensors (shard k holds the next shards[k].shape[1] columns), emulating a
+    vocabulary-sharded target on one GPU; results as tt_verify's, next_token a
+    column of the whole row. summaries=True also returns the gathered per-shard
+    records [S, n_target + B, 4] (max, sum hi, sum lo, scored logit or NaN)."""
+    dev = batch.target_off.device
+    o = dict(out or {})
+    o.setdefault("accepted", _empty(batch.B, torch.int32, dev))
+    o.setdefault("next_token", _empty(batch.B, torch.int32, dev))
+    o.setdefault("status", _empty(batch.B, torch.int32, dev))
+    o.setdefault("p_hat", _empty(batch.n_target, torch.float32, dev))
+    o.setdefault("lse", _empty(batch.n_target + batch.B, torch.float32, dev))
+    rows = batch.n_target + batch.B
+    if summaries:
+        o.setdefault("summaries", torch.empty((len(shards), rows, 4), dtype=torch.float32,
+                                              device=dev))
+    sh, keep_sh = _shards(shards)
+    L = load()
+    if ws is None:
+        n = int(L.tt_sharded_workspace_bytes(ctypes.byref(batch._c()), ctypes.byref(sh)))
+        if n == 0:
+            raise TTError("tt_sharded_workspace_bytes", TT_ERR_INVALID_ARG, "invalid argument")
+        ws = torch.empty(n, dtype=torch.uint8, device=dev)
+    keep = []
+    code = L.tt_verify_sharded(ctypes.byref(batch._c()), _ptr(q_hat), ctypes.byref(sh),
+                               ctypes.byref(params._c(keep)), _ptr(ws), ws.numel(),
+                               _ptr(o["accepted"]), _ptr(o["next_token"]), _ptr(o["p_hat"]),
+                               _ptr(o["lse"]), _ptr(o.get("summaries")), _ptr(o["status"]),
+                               _stream(stream))
+    _check("tt_verify_sharded", code)
     return o
 
 

@@ -34,6 +34,7 @@ cudaError_t ensure_loaded() {
   if ((e = preload_rowpass()) != cudaSuccess) return e;
   if ((e = preload_decide()) != cudaSuccess) return e;
   if ((e = preload_filter()) != cudaSuccess) return e;
+  if ((e = preload_shard()) != cudaSuccess) return e;
   if (dev >= 0 && dev < 64) done[dev] = true;
   return cudaSuccess;
 }
@@ -94,6 +95,27 @@ bool filters_supported(const tt_params* p) {
 
 int k_draft(const tt_params* p) { return p->top_k_draft; }
 int k_target(const tt_params* p) { return p->top_k_target; }
+
+// Shards usable by tt_verify_sharded: 1..TT_MAX_SHARDS logits arrays of
+// rows_needed rows that tile the row in order from column 0; V = the row width.
+bool shards_ok(const tt_shards* sh, int64_t rows_needed, int32_t* V) {
+  if (!sh || sh->S < 1 || sh->S > TT_MAX_SHARDS || !sh->shards || !sh->col0) return false;
+  int64_t c = 0;
+  for (int s = 0; s < sh->S; ++s) {
+    if (!logits_ok(&sh->shards[s], rows_needed)) return false;
+    if (sh->col0[s] != c) return false;
+    c += sh->shards[s].n_cols;
+  }
+  if (c > INT32_MAX) return false;
+  *V = int32_t(c);
+  return true;
+}
+
+ShardWorkspace shard_workspace(void* base, const tt_batch* batch, const tt_shards* sh) {
+  int32_t nch[TT_MAX_SHARDS] = {0};
+  for (int s = 0; s < sh->S; ++s) nch[s] = n_chunks(sh->shards[s].n_cols);
+  return shard_layout(base, int64_t(batch->n_target) + batch->B, sh->S, nch);
+}
 
 bool vocab_ok(const tt_vocab* v) {
   return v && v->bytes && v->offsets && v->n_tokens >= 1 && v->n_bytes >= 0;
@@ -556,6 +578,105 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
     return cuda_fail(e);
   }
   record(prm, 3, s);
+  return TT_OK;
+}
+
+size_t tt_sharded_workspace_bytes(const tt_batch* batch, const tt_shards* target) {
+  if (!batch_ok(batch)) return 0;
+  int32_t V = 0;
+  if (!shards_ok(target, int64_t(batch->n_target) + batch->B, &V)) return 0;
+  return shard_workspace(nullptr, batch, target).bytes;
+}
+
+tt_status tt_verify_sharded(const tt_batch* batch, const float* q_hat, const tt_shards* target,
+                            const tt_params* prm, void* workspace, size_t workspace_bytes,
+                            int32_t* accepted, int32_t* next_token, float* p_hat, float* lse,
+                            float* summaries, int32_t* status, void* stream) {
+  if (!batch_ok(batch) || !params_ok(prm)) return TT_ERR_INVALID_ARG;
+  if (batch->B == 0) return TT_OK;
+  if (!accepted || !next_token || !status) return TT_ERR_INVALID_ARG;
+  if (batch->n_target > 0 && !q_hat) return TT_ERR_INVALID_ARG;
+  const int32_t* tcols = batch->target_cols ? batch->target_cols : batch->target_ids;
+  if (batch->n_target > 0 && !tcols) return TT_ERR_INVALID_ARG;
+  const int64_t rows = int64_t(batch->n_target) + batch->B;
+  int32_t V = 0;
+  if (!shards_ok(target, rows, &V)) return TT_ERR_INVALID_ARG;
+  // one-hot transfer, no filters
+  if (prm->full_q != 0 || prm->top_k_target != 0 || prm->top_p_target < 1.f)
+    return TT_ERR_UNSUPPORTED;
+  const ShardWorkspace ws0 = shard_workspace(nullptr, batch, target);
+  if (!workspace || workspace_bytes < ws0.bytes ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
+    return TT_ERR_INVALID_ARG;
+  const ShardWorkspace ws = shard_workspace(workspace, batch, target);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = ensure_loaded();
+  if (e != cudaSuccess) return cuda_fail(e);
+
+  ShardArgs a;
+  std::memset(&a, 0, sizeof a);
+  a.B = batch->B;
+  a.n_target = batch->n_target;
+  a.S = target->S;
+  a.V = V;
+  a.max_m = batch->max_m;
+  a.rows = rows;
+  a.target_off = batch->target_off;
+  a.target_cols = tcols;
+  a.excl = ws.excl;
+  a.rec = ws.rec;
+  a.work = ws.work;
+  a.scale = log2e_over(prm->temp_target);
+  a.q_hat = q_hat;
+  a.seed = prm->seed;
+  a.request_base = prm->request_base;
+  a.err = ws.err;
+  a.epoch = next_epoch();
+  a.accepted = accepted;
+  a.next_token = next_token;
+  a.status = status;
+  a.p_hat = p_hat;
+  a.lse = lse;
+  for (int k = 0; k < target->S; ++k) {
+    const tt_logits& L = target->shards[k];
+    ShardDesc& d = a.sh[k];
+    d.data = static_cast<const char*>(L.data);
+    d.stride_bytes = L.row_stride * (L.dtype == TT_F32 ? 4 : 2);
+    d.V = L.n_cols;
+    d.col0 = target->col0[k];
+    d.nch = n_chunks(L.n_cols);
+    d.dtype = L.dtype;
+    d.part = ws.part[k];
+  }
+  if ((e = launch_shard_excl(a, s)) != cudaSuccess) return cuda_fail(e);
+  // each shard's slice reduced by its own row pass (what one rank does)
+  for (int k = 0; k < target->S; ++k) {
+    RowPassArgs r;
+    std::memset(&r, 0, sizeof r);
+    r.t = rowset(&target->shards[k], ws.part[k], nullptr, prm->temp_target);
+    r.rows_t = rows;
+    r.d = no_rows();
+    r.rows_d = 0;
+    r.excl = ws.excl + int64_t(k) * rows;
+    r.B = batch->B;
+    r.n_target = batch->n_target;
+    r.target_off = batch->target_off;
+    r.target_cols = tcols;
+    r.err = ws.err;
+    r.epoch = a.epoch;
+    r.work = reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(ws.work) +
+                                                   size_t(k) * kWorkShards * kWorkStride *
+                                                       sizeof(unsigned long long));
+    if ((e = launch_rowpass(r, TT_F32, target->shards[k].dtype, s, sm_count_current(), false)) !=
+        cudaSuccess)
+      return cuda_fail(e);
+  }
+  if ((e = launch_shard_summary(a, s, sm_count_current())) != cudaSuccess) return cuda_fail(e);
+  if (summaries &&
+      (e = cudaMemcpyAsync(summaries, ws.rec, sizeof(ShardRec) * size_t(target->S) * rows,
+                           cudaMemcpyDeviceToDevice, s)) != cudaSuccess)
+    return cuda_fail(e);
+  if ((e = launch_decide_sharded(a, s)) != cudaSuccess) return cuda_fail(e);
   return TT_OK;
 }
 

@@ -51,6 +51,7 @@ def test_struct_layouts_match_the_header():
     assert ctypes.sizeof(binding._Vocab) == 32 and binding._Vocab.n_bytes.offset == 24
     assert binding._Batch.draft_off.offset == 24 and ctypes.sizeof(binding._Batch) == 72
     assert ctypes.sizeof(binding._StepOut) == 80
+    assert ctypes.sizeof(binding._Shards) == 24 and binding._Shards.col0.offset == 16
 
 
 def test_status_strings_and_version(lib):
@@ -110,6 +111,44 @@ def test_host_validation_rejects_bad_arguments(lib):
     e = tt.Batch.from_host([0], [], [0], [], device="cpu")
     assert lib.tt_align(P(e._c()), P(vd._c()), P(vd._c()), P(prm._c(keep)), None, None, None,
                         None, None, None) == binding.TT_OK
+
+
+def _shards(widths, col0=None):
+    arr = (binding._Logits * len(widths))()
+    c0 = (ctypes.c_int32 * len(widths))()
+    c = 0
+    for k, w in enumerate(widths):
+        arr[k] = binding._Logits(256 * (k + 1), binding.TT_F32, w, (w + 3) // 4 * 4, 10)
+        c0[k] = c if col0 is None else col0[k]
+        c += w
+    return binding._Shards(len(widths), arr, c0), (arr, c0)
+
+
+def test_sharded_verify_host_rules(lib):
+    b = _batch_host()
+    keep = []
+    P = ctypes.byref
+    prm = binding.Params()._c(keep)
+    one = lib.tt_sharded_workspace_bytes(P(b._c()), P(_shards([100])[0]))
+    three = lib.tt_sharded_workspace_bytes(P(b._c()), P(_shards([40, 4096, 3000])[0]))
+    assert 0 < one < three
+    # shards must tile the row from column 0, in order, and number 1..8
+    for sh, _ in (_shards([40, 60], col0=[0, 41]), _shards([40, 60], col0=[1, 41]),
+                  _shards([8] * (binding.TT_MAX_SHARDS + 1))):
+        assert lib.tt_sharded_workspace_bytes(P(b._c()), P(sh)) == 0
+        assert lib.tt_verify_sharded(P(b._c()), ctypes.c_void_p(16), P(sh), P(prm),
+                                     ctypes.c_void_p(256), 1 << 30, ctypes.c_void_p(16),
+                                     ctypes.c_void_p(16), None, None, None, ctypes.c_void_p(16),
+                                     None) == binding.TT_ERR_INVALID_ARG
+    sh, _ = _shards([40, 60])
+    call = lambda p, n=1 << 30: lib.tt_verify_sharded(
+        P(b._c()), ctypes.c_void_p(16), P(sh), P(p), ctypes.c_void_p(256), n, ctypes.c_void_p(16),
+        ctypes.c_void_p(16), None, None, None, ctypes.c_void_p(16), None)
+    # one-hot transfer without filters only
+    assert call(binding.Params(full_q=True)._c(keep)) == binding.TT_ERR_UNSUPPORTED
+    assert call(binding.Params(top_k_target=5)._c(keep)) == binding.TT_ERR_UNSUPPORTED
+    # workspace too small
+    assert call(prm, 8) == binding.TT_ERR_INVALID_ARG
 
 
 def test_alignment_tile_too_large_is_unsupported(lib):
