@@ -57,6 +57,10 @@ def parse_args(argv=None):
                     help="top-k filter of draft and target rows (0 = off)")
     ap.add_argument("--top-p", type=float, default=1.0,
                     help="top-p filter after the top-k (1 = off)")
+    ap.add_argument("--shards", type=int, default=0,
+                    help="also time the vocabulary-sharded verification with the target "
+                         "rows split into this many column slices (1-8), against the "
+                         "unsplit verification (outside the timed region)")
     ap.add_argument("--no-reencode", action="store_true",
                     help="skip timing the re-encoding, Lemma-1 check and delta-pos histogram")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -404,6 +408,9 @@ def run_mine(args):
         e2e = run_e2e(tt, wl, inp, prm, dev, stream, K, ws)
 
     reenc = None if args.no_reencode else run_reencode(tt, wl, inp, prm, dev, stream, rank, ws)
+    sharded = None
+    if args.shards > 0 and not filtered and not prm.full_q:
+        sharded = run_sharded(tt, wl, inp, prm, full["q_hat"], dev, stream, args.shards)
 
     cpu = cpu_all = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -441,13 +448,15 @@ def run_mine(args):
                      "peak_kind": "%s copy bandwidth (hbm_gbs)" % peak_kind,
                      "traffic": traffic, "algorithmic_bytes": ab["total"],
                      "vs_nominal_8tbs": achieved / 8000.0},
-        "gpu_launches": (4 if filtered else 3) * K,
+        "gpu_launches": (5 if filtered else 3) * K,
         "clocks": clk,
     }
     if e2e is not None:
         line["e2e"] = e2e
     if reenc is not None:
         line["reencode"] = reenc
+    if sharded is not None:
+        line["sharded"] = sharded
     if cpu is not None:
         line["cpu_baseline"] = cpu
     if cpu_all is not None:
@@ -471,6 +480,43 @@ def _time_calls(fn, stream, n, warm=3):
     e1.record(stream)
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) / n  # ms per call
+
+
+def run_sharded(tt, wl, inp, prm, q_hat, dev, stream, S):
+    """The verification of the batch's target rows split by columns into S
+    near-equal slices held in separate arrays (tt_verify_sharded: per-shard row
+    passes, the gathered records, the merged decision), against tt_verify on the
+    unsplit rows with the same q_hat; each timed alone with CUDA events over
+    repeated calls, outside the step's timed region. Also reports how many
+    requests the two agree on and the bytes an all-gather of the records moves."""
+    import torch
+    tl = inp["target_logits"]
+    V = tl.shape[1]
+    per16 = 16 // tl.element_size()
+    cuts = [round(V * k / S) for k in range(S + 1)]
+    shards = []
+    for a, b in zip(cuts, cuts[1:]):
+        buf = torch.empty((tl.shape[0], (b - a + per16 - 1) // per16 * per16), dtype=tl.dtype,
+                          device=dev)
+        buf[:, :b - a] = tl[:, a:b]
+        shards.append(buf[:, :b - a])
+    batch = inp["batch"]
+    ws_v = tt.binding.workspace(batch, 0, V, dev, prm)
+    ws_s = tt.binding.sharded_workspace(batch, shards, dev)
+    out_v, out_s = {}, {}
+    unsplit = lambda: out_v.update(tt.tt_verify(batch, q_hat, tl, prm, ws=ws_v, out=out_v,
+                                                 stream=stream))
+    split = lambda: out_s.update(tt.tt_verify_sharded(batch, q_hat, shards, prm, ws=ws_s,
+                                                       out=out_s, stream=stream))
+    n = 50
+    t_unsplit = _time_calls(unsplit, stream, n)
+    t_split = _time_calls(split, stream, n)
+    rows = batch.n_target + batch.B
+    agree_a = int((out_v["accepted"] == out_s["accepted"]).sum())
+    agree_t = int((out_v["next_token"] == out_s["next_token"]).sum())
+    return {"shards": S, "verify_ms_unsplit": t_unsplit, "verify_ms_sharded": t_split,
+            "exchange_bytes": 16 * S * rows, "requests": batch.B,
+            "agree_accepted": agree_a, "agree_next_token": agree_t}
 
 
 def run_reencode(tt, wl, inp, prm, dev, stream, rank, ws):

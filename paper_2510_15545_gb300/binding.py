@@ -357,6 +357,15 @@ def _shards(shards):
     return _Shards(S, arr, col0), (arr, col0)
 
 
+def sharded_workspace(batch: Batch, shards, device="cuda") -> torch.Tensor:
+    """Scratch for tt_verify_sharded with these shards."""
+    sh, keep = _shards(shards)
+    n = int(load().tt_sharded_workspace_bytes(ctypes.byref(batch._c()), ctypes.byref(sh)))
+    if n == 0:
+        raise TTError("tt_sharded_workspace_bytes", TT_ERR_INVALID_ARG, "invalid argument")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
 def tt_verify_sharded(batch: Batch, q_hat: torch.Tensor, shards, params: Params, *,
                       ws=None, out=None, stream=None, summaries: bool = False) -> dict:
     """Verification over target rows split by columns into len(shards) logits
@@ -378,10 +387,7 @@ def tt_verify_sharded(batch: Batch, q_hat: torch.Tensor, shards, params: Params,
     sh, keep_sh = _shards(shards)
     L = load()
     if ws is None:
-        n = int(L.tt_sharded_workspace_bytes(ctypes.byref(batch._c()), ctypes.byref(sh)))
-        if n == 0:
-            raise TTError("tt_sharded_workspace_bytes", TT_ERR_INVALID_ARG, "invalid argument")
-        ws = torch.empty(n, dtype=torch.uint8, device=dev)
+        ws = sharded_workspace(batch, shards, dev)
     keep = []
     code = L.tt_verify_sharded(ctypes.byref(batch._c()), _ptr(q_hat), ctypes.byref(sh),
                                ctypes.byref(params._c(keep)), _ptr(ws), ws.numel(),

@@ -8,6 +8,7 @@
 
 #include "tt_device.cuh"
 #include "tt_launch.h"
+#include "tt_shard.h"
 
 namespace {
 

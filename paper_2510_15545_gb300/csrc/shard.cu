@@ -19,6 +19,7 @@
 
 #include "tt_device.cuh"
 #include "tt_launch.h"
+#include "tt_shard.h"
 
 namespace tt {
 
