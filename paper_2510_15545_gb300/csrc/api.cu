@@ -650,7 +650,11 @@ tt_status tt_verify_sharded(const tt_batch* batch, const float* q_hat, const tt_
     d.part = ws.part[k];
   }
   if ((e = launch_shard_excl(a, s)) != cudaSuccess) return cuda_fail(e);
-  // each shard's slice reduced by its own row pass (what one rank does)
+  // each shard's slice reduced by its own row pass (what one rank does). Passes
+  // after the first start while the one before drains (programmatic dependent
+  // launch): what they read before their grid-dependency wait -- the scored
+  // columns and their zeroed work counters -- was written by the excl kernel,
+  // which finished before the first pass, launched without the attribute, began.
   for (int k = 0; k < target->S; ++k) {
     RowPassArgs r;
     std::memset(&r, 0, sizeof r);
@@ -668,7 +672,7 @@ tt_status tt_verify_sharded(const tt_batch* batch, const float* q_hat, const tt_
     r.work = reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(ws.work) +
                                                    size_t(k) * kWorkShards * kWorkStride *
                                                        sizeof(unsigned long long));
-    if ((e = launch_rowpass(r, TT_F32, target->shards[k].dtype, s, sm_count_current(), false)) !=
+    if ((e = launch_rowpass(r, TT_F32, target->shards[k].dtype, s, sm_count_current(), k > 0)) !=
         cudaSuccess)
       return cuda_fail(e);
   }

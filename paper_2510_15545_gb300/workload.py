@@ -169,6 +169,7 @@ class WorkloadSpec:
     noise: float = 0.0
     corr_frac: float = 0.0
     corr_rho: float = 0.0
+    corr_shift: float = 0.0  # correlated rows: target-only columns lowered by this (nats)
     verify_V: Optional[int] = None  # width of the logits rows if smaller than the vocab
     exact_m: bool = False  # target length drawn uniformly, exact segmentation
     share: float = 0.85
@@ -180,20 +181,22 @@ class WorkloadSpec:
 
 SPECS: Dict[str, WorkloadSpec] = {
     "b1_g4_v32k": WorkloadSpec("b1_g4_v32k", B=1, k=4, m_lo=3, m_hi=6, V_d=32000, V_t=32768,
-                               dtype=torch.float32, logits="normal3"),
+                               dtype=torch.float32, logits="normal3", corr_frac=1.0,
+                               corr_rho=0.9, corr_shift=3.0),
     "b64_g8_v152k": WorkloadSpec("b64_g8_v152k", B=64, k=8, m_lo=5, m_hi=12, V_d=32000,
                                  V_t=151936, dtype=torch.float32, logits="zipf", zipf_s=1.1,
-                                 noise=0.5),
+                                 noise=0.5, corr_frac=1.0, corr_rho=0.9, corr_shift=3.0),
     "b256_g16_v152k_bf16": WorkloadSpec("b256_g16_v152k_bf16", B=256, k=16, m_lo=10, m_hi=24,
                                         V_d=128256, V_t=151936, dtype=torch.bfloat16,
-                                        logits="zipf", zipf_s=1.2, noise=1.0, corr_frac=0.3,
-                                        corr_rho=0.8),
+                                        logits="zipf", zipf_s=1.2, noise=1.0, corr_frac=1.0,
+                                        corr_rho=0.9, corr_shift=3.0),
     "dtw_4096x64": WorkloadSpec("dtw_4096x64", B=4096, k=64, m_lo=48, m_hi=96, V_d=32000,
                                 V_t=151936, dtype=torch.float32, logits="zipf", zipf_s=1.1,
                                 noise=0.5, verify_V=4096, exact_m=True),
     "b1024_g8_v201k_bf16": WorkloadSpec("b1024_g8_v201k_bf16", B=1024, k=8, m_lo=5, m_hi=14,
                                         V_d=151936, V_t=201088, dtype=torch.bfloat16,
-                                        logits="zipf", zipf_s=1.0, noise=1.0),
+                                        logits="zipf", zipf_s=1.0, noise=1.0, corr_frac=1.0,
+                                        corr_rho=0.9, corr_shift=3.0),
 }
 # Order of the five workloads (smallest first).
 SPEC_ORDER = ["b1_g4_v32k", "b64_g8_v152k", "b256_g16_v152k_bf16", "dtw_4096x64",
@@ -416,8 +419,11 @@ def _correlate(spec, target_logits, draft_logits, draft_off, target_off, draft_i
     """Makes the target rows of a fraction ``corr_frac`` of the requests
     correlated (coefficient ``corr_rho``) with the draft row holding the same
     bytes, through the injection that sends a target string to the draft id
-    spelling it: z_t = rho * z_d + sqrt(1 - rho^2) * sd(z_d) * N(0, 1). The
-    bonus row follows the last draft row."""
+    spelling it: z_t = rho * z_d + sqrt(1 - rho^2) * sd(z_d) * N(0, 1) on the
+    columns the two vocabularies share; the target-only columns of those rows
+    are lowered by ``corr_shift``, standing for a target that puts little mass
+    on strings the draft cannot spell. The bonus row follows the last draft
+    row. Rows are processed in blocks of bounded size."""
     inj = np.full(vt.n_tokens, -1, dtype=np.int64)
     for tid, s in enumerate(vt.strings):
         did = vd.index.get(s)
@@ -431,17 +437,29 @@ def _correlate(spec, target_logits, draft_logits, draft_off, target_off, draft_i
     gen = torch.Generator(device=device)
     gen.manual_seed(int(rng.integers(0, 2**31)))
     chosen = rng.random(B) < spec.corr_frac
+    rows_t, rows_d = [], []
     for b in np.nonzero(chosen)[0]:
         d0, d1 = int(draft_off[b]), int(draft_off[b + 1])
         t0, t1 = int(target_off[b]), int(target_off[b + 1])
         src = _source_rows(vd, vt, draft_ids[d0:d1], target_ids[t0:t1])
         src = np.concatenate([src, [d1 - d0 - 1]])
-        for j, i in enumerate(src):
-            zd = draft_logits[d0 + int(i), from_d]
-            sd = float(zd.std())
-            noise = torch.randn(zd.shape, generator=gen, device=device) * sd
-            row = target_logits[t0 + b + j]
-            row[have_t] = rho * zd + math.sqrt(1 - rho * rho) * noise
+        rows_t.extend(t0 + int(b) + np.arange(len(src)))
+        rows_d.extend(d0 + src.astype(np.int64))
+    if not rows_t:
+        return
+    rows_t = torch.as_tensor(np.asarray(rows_t, dtype=np.int64), device=device)
+    rows_d = torch.as_tensor(np.asarray(rows_d, dtype=np.int64), device=device)
+    step = max(1, (1 << 26) // max(target_logits.shape[1], 1))
+    for r0 in range(0, len(rows_t), step):
+        rt, rd = rows_t[r0:r0 + step], rows_d[r0:r0 + step]
+        zd = draft_logits[rd][:, from_d]
+        sd = zd.std(dim=1, keepdim=True)
+        noise = torch.randn(zd.shape, generator=gen, device=device) * sd
+        blk = target_logits[rt]
+        if spec.corr_shift:
+            blk -= spec.corr_shift
+        blk[:, have_t] = rho * zd + math.sqrt(1 - rho * rho) * noise
+        target_logits[rt] = blk
 
 
 def homogeneous_workload(B: int, k: int, V: int, *, seed: int = 0, device: str = "cpu",
