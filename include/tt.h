@@ -180,8 +180,10 @@ size_t tt_workspace_bytes_for(const tt_batch* batch, int32_t V_d, int32_t V_t,
  * (k, m) taking the smallest predecessor, ties broken diagonal, then (i-1, j),
  * then (i, j-1). Writes path/path_len/cost/map/status; map[j] is the largest
  * draft index on the path in column j. Uses batch ids (not cols). Needs no
- * workspace. TT_ERR_UNSUPPORTED when the on-chip tile for max_k x max_m (and
- * the band) does not fit in shared memory. */
+ * workspace. The on-chip tile of a pair takes one byte per band cell (at most
+ * about 145 KB of shared memory at max_k = TT_MAX_K, max_m = TT_MAX_M with no
+ * band), so every allowed size fits; TT_ERR_UNSUPPORTED would report one that
+ * did not. */
 tt_status tt_align(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
                    const tt_params* prm, int32_t* path, int32_t* path_len, int32_t* cost,
                    int32_t* map, int32_t* status, void* stream);

@@ -54,6 +54,46 @@ __device__ __forceinline__ int lev_packed8(uint64_t P, int lp, uint64_t T, int l
   return score;
 }
 
+// Two independent lev_packed8 evaluations advanced in lockstep (each column
+// step applied only while that pair's text lasts): the same results, with two
+// dependency chains interleaved. Pairs with an empty string take the closed form.
+__device__ __forceinline__ void lev_packed8_x2(uint64_t P0, int lp0, uint64_t T0, int lt0,
+                                               uint64_t P1, int lp1, uint64_t T1, int lt1,
+                                               int& d0, int& d1) {
+  const uint32_t mask0 = lp0 > 0 ? (1u << lp0) - 1u : 0u, hb0 = lp0 > 0 ? 1u << (lp0 - 1) : 0u;
+  const uint32_t mask1 = lp1 > 0 ? (1u << lp1) - 1u : 0u, hb1 = lp1 > 0 ? 1u << (lp1 - 1) : 0u;
+  uint32_t Pv0 = mask0, Mv0 = 0, Pv1 = mask1, Mv1 = 0;
+  int s0 = lp0, s1 = lp1;
+  const int n = max(lp0 > 0 ? lt0 : 0, lp1 > 0 ? lt1 : 0);
+  for (int x = 0; x < n; ++x) {
+    const uint32_t Eq0 = eq_mask8(P0, uint32_t(T0 >> (8 * x)) & 0xFFu) & mask0;
+    const uint32_t Eq1 = eq_mask8(P1, uint32_t(T1 >> (8 * x)) & 0xFFu) & mask1;
+    const uint32_t Xv0 = Eq0 | Mv0, Xv1 = Eq1 | Mv1;
+    const uint32_t Xh0 = (((Eq0 & Pv0) + Pv0) ^ Pv0) | Eq0;
+    const uint32_t Xh1 = (((Eq1 & Pv1) + Pv1) ^ Pv1) | Eq1;
+    uint32_t Ph0 = Mv0 | ~(Xh0 | Pv0), Ph1 = Mv1 | ~(Xh1 | Pv1);
+    uint32_t Mh0 = Pv0 & Xh0, Mh1 = Pv1 & Xh1;
+    const int e0 = int((Ph0 & hb0) != 0) - int((Mh0 & hb0) != 0);
+    const int e1 = int((Ph1 & hb1) != 0) - int((Mh1 & hb1) != 0);
+    Ph0 = (Ph0 << 1) | 1u;
+    Ph1 = (Ph1 << 1) | 1u;
+    Mh0 <<= 1;
+    Mh1 <<= 1;
+    if (x < lt0) {
+      s0 += e0;
+      Pv0 = Mh0 | ~(Xv0 | Ph0);
+      Mv0 = Ph0 & Xv0;
+    }
+    if (x < lt1) {
+      s1 += e1;
+      Pv1 = Mh1 | ~(Xv1 | Ph1);
+      Mv1 = Ph1 & Xv1;
+    }
+  }
+  d0 = lp0 == 0 ? lt0 : (lt0 == 0 ? lp0 : s0);
+  d1 = lp1 == 0 ? lt1 : (lt1 == 0 ? lp1 : s1);
+}
+
 // Edit distance by the textbook row recurrence, for tokens longer than 8
 // bytes (bytes read from the global tables; ns, nt <= TT_MAX_TOKEN_BYTES).
 __device__ int lev_rows(const uint8_t* s, int ns, const uint8_t* t, int nt) {
@@ -81,7 +121,7 @@ struct PairSmem {
   uint64_t* tok;  // [K + M] packed bytes (valid when len <= 8)
   int32_t* diag;  // [3 * (K + 2)] rotating anti-diagonals, indexed by i
   uint32_t* path; // [K + M] backtracked cells (i << 16 | j), reverse order
-  uint16_t* tile; // [K * TW] cost, then direction
+  uint8_t* tile;  // [K * TW] cost (255: 255 or more, recomputed), then direction
   uint16_t* len;  // [K + M] token byte lengths
 };
 
@@ -94,8 +134,8 @@ __device__ __forceinline__ PairSmem carve(char* base, int K, int M, int TW) {
   off += sizeof(int32_t) * 3 * (K + 2);
   s.path = reinterpret_cast<uint32_t*>(base + off);
   off += sizeof(uint32_t) * (K + M);
-  s.tile = reinterpret_cast<uint16_t*>(base + off);
-  off += sizeof(uint16_t) * size_t(K) * TW;
+  s.tile = reinterpret_cast<uint8_t*>(base + off);
+  off += (size_t(K) * TW + 15) & ~size_t(15);
   s.len = reinterpret_cast<uint16_t*>(base + off);
   return s;
 }
@@ -175,54 +215,134 @@ __global__ void __launch_bounds__(kAlignWarpsMax * 32)
   const int W0 = a.window < 0 ? k + m : max(a.window, abs(k - m));  // band half-width
   const int tw = min(m, 2 * W0 + 1);                                 // tile cells per row
 
-  // 1. banded local costs; row i (1-based) holds j = jlo(i) .. jhi(i)
-  for (int idx = lane; idx < k * tw; idx += 32) {
-    const int i = idx / tw + 1, c = idx - (i - 1) * tw;
-    const int jlo = max(1, i - W0), j = jlo + c;
-    if (j > min(m, i + W0)) continue;
+  // local cost d(i, j) of draft token i and target token j (1-based)
+  auto token_cost = [&](int i, int j) -> int {
     const int ld = sm.len[i - 1], lt = sm.len[k + j - 1];
-    int d;
     if (ld <= 8 && lt <= 8) {
       // pattern = the longer string, text = the shorter (fewer steps)
-      d = ld >= lt ? lev_packed8(sm.tok[i - 1], ld, sm.tok[k + j - 1], lt)
-                   : lev_packed8(sm.tok[k + j - 1], lt, sm.tok[i - 1], ld);
-    } else {
-      const int di = a.draft_ids[d0 + i - 1], ti = a.target_ids[t0 + j - 1];
-      d = lev_rows(a.vd.bytes + a.vd.offsets[di], ld, a.vt.bytes + a.vt.offsets[ti], lt);
+      return ld >= lt ? lev_packed8(sm.tok[i - 1], ld, sm.tok[k + j - 1], lt)
+                      : lev_packed8(sm.tok[k + j - 1], lt, sm.tok[i - 1], ld);
     }
-    sm.tile[size_t(i - 1) * TW + c] = uint16_t(d);
+    const int di = a.draft_ids[d0 + i - 1], ti = a.target_ids[t0 + j - 1];
+    return lev_rows(a.vd.bytes + a.vd.offsets[di], ld, a.vt.bytes + a.vt.offsets[ti], lt);
+  };
+
+  // 1. banded local costs, one byte each (a cost of 255 or more is stored as
+  // 255 and recomputed in the sweep); row i (1-based) holds j = jlo(i) .. jhi(i).
+  // Each lane takes two cells per step: when both are short tokens their two
+  // bit-parallel evaluations run interleaved.
+  for (int idx = lane; idx < k * tw; idx += 64) {
+    int ii[2], cc[2], jj[2];
+    bool ok[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int id = idx + 32 * h;
+      ii[h] = id / tw + 1;
+      cc[h] = id - (ii[h] - 1) * tw;
+      jj[h] = max(1, ii[h] - W0) + cc[h];
+      ok[h] = id < k * tw && jj[h] <= min(m, ii[h] + W0);
+    }
+    int d[2] = {0, 0};
+    const bool short0 = ok[0] && sm.len[ii[0] - 1] <= 8 && sm.len[k + jj[0] - 1] <= 8;
+    const bool short1 = ok[1] && sm.len[ii[1] - 1] <= 8 && sm.len[k + jj[1] - 1] <= 8;
+    if (short0 && short1) {
+      // pattern = the longer string, text = the shorter, for each pair
+      uint64_t P[2], T[2];
+      int lp[2], lt[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int ld = sm.len[ii[h] - 1], ltk = sm.len[k + jj[h] - 1];
+        const uint64_t pd = sm.tok[ii[h] - 1], pt = sm.tok[k + jj[h] - 1];
+        const bool dl = ld >= ltk;
+        P[h] = dl ? pd : pt;
+        lp[h] = dl ? ld : ltk;
+        T[h] = dl ? pt : pd;
+        lt[h] = dl ? ltk : ld;
+      }
+      lev_packed8_x2(P[0], lp[0], T[0], lt[0], P[1], lp[1], T[1], lt[1], d[0], d[1]);
+    } else {
+      if (ok[0]) d[0] = token_cost(ii[0], jj[0]);
+      if (ok[1]) d[1] = token_cost(ii[1], jj[1]);
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+      if (ok[h]) sm.tile[size_t(ii[h] - 1) * TW + cc[h]] = uint8_t(min(d[h], 255));
   }
 
-  // 2. anti-diagonal sweep; buffer s % 3 holds C(i, s - i) at index i
-  int32_t* D[3] = {sm.diag, sm.diag + (K + 2), sm.diag + 2 * (K + 2)};
-  for (int i = lane; i <= k + 1; i += 32) {
-    D[0][i] = i == 0 ? 0 : kInf;  // s = 0: C(0,0) = 0
-    D[1][i] = kInf;               // s = 1: border cells only
-  }
-  __syncwarp();
-  for (int s = 2; s <= k + m; ++s) {
-    int32_t* cur = D[s % 3];
-    const int32_t* p1 = D[(s + 2) % 3];
-    const int32_t* p2 = D[(s + 1) % 3];
-    const int lo = max(max(1, s - m), (s - W0 + 1) >> 1);  // ceil((s - W0) / 2)
-    const int hi = min(min(k, s - 1), (s + W0) >> 1);
-    for (int i = lo + lane; i <= hi; i += 32) {
-      const int j = s - i;
-      const int up = p1[i - 1], left = p1[i], dg = p2[i - 1];
-      int best = dg, dir = 0;
-      if (up < best) { best = up; dir = 1; }
-      if (left < best) { best = left; dir = 2; }
-      uint16_t* cell = sm.tile + size_t(i - 1) * TW + (j - max(1, i - W0));
-      cur[i] = best >= kInf ? kInf : best + int(*cell);
-      *cell = uint16_t(dir);
+  // 2. anti-diagonal sweep. A diagonal s = i + j holds the cells
+  // i = lo(s) .. hi(s); each depends on the two diagonals before it.
+  int cstar;
+  if (W0 <= 31) {
+    // at most W0 + 1 <= 32 cells per diagonal: lane l holds cell lo(s) + l of
+    // diagonal s in a register, and the previous two diagonals' values come by
+    // shuffles (a cell outside their ranges is infinite: a border, or outside
+    // the band); diagonal 0 is C(0,0) = 0, diagonal 1 holds borders only
+    int v1 = kInf, lo1 = 1, n1 = 0;                // diagonal s - 1
+    int v2 = lane == 0 ? 0 : kInf, lo2 = 0, n2 = 1;  // diagonal s - 2
+    for (int s = 2; s <= k + m; ++s) {
+      const int lo = max(max(1, s - m), (s - W0 + 1) >> 1);
+      const int hi = min(min(k, s - 1), (s + W0) >> 1);
+      const int i = lo + lane, j = s - i;
+      const int su = i - 1 - lo1, sl = i - lo1, sd = i - 1 - lo2;
+      const int up0 = __shfl_sync(0xffffffffu, v1, su & 31);
+      const int left0 = __shfl_sync(0xffffffffu, v1, sl & 31);
+      const int dg0 = __shfl_sync(0xffffffffu, v2, sd & 31);
+      int v = kInf;
+      if (i <= hi) {
+        const int up = (su >= 0 && su < n1) ? up0 : kInf;
+        const int left = (sl >= 0 && sl < n1) ? left0 : kInf;
+        int best = (sd >= 0 && sd < n2) ? dg0 : kInf, dir = 0;
+        if (up < best) { best = up; dir = 1; }
+        if (left < best) { best = left; dir = 2; }
+        uint8_t* cell = sm.tile + size_t(i - 1) * TW + (j - max(1, i - W0));
+        int cost = *cell;
+        if (cost == 255) cost = token_cost(i, j);
+        v = best >= kInf ? kInf : best + cost;
+        *cell = uint8_t(dir);
+      }
+      v2 = v1;
+      lo2 = lo1;
+      n2 = n1;
+      v1 = v;
+      lo1 = lo;
+      n1 = hi - lo + 1;
     }
-    if (lane == 0) {  // guards: neighbours just outside the diagonal read as infinite
-      if (lo - 1 >= 0) cur[lo - 1] = kInf;
-      if (hi + 1 <= k + 1) cur[hi + 1] = kInf;
+    cstar = __shfl_sync(0xffffffffu, v1, (k - lo1) & 31);  // C(k, m): the last diagonal's cell k
+    __syncwarp();
+  } else {
+    // buffer s % 3 holds C(i, s - i) at index i
+    int32_t* D[3] = {sm.diag, sm.diag + (K + 2), sm.diag + 2 * (K + 2)};
+    for (int i = lane; i <= k + 1; i += 32) {
+      D[0][i] = i == 0 ? 0 : kInf;  // s = 0: C(0,0) = 0
+      D[1][i] = kInf;               // s = 1: border cells only
     }
     __syncwarp();
+    for (int s = 2; s <= k + m; ++s) {
+      int32_t* cur = D[s % 3];
+      const int32_t* p1 = D[(s + 2) % 3];
+      const int32_t* p2 = D[(s + 1) % 3];
+      const int lo = max(max(1, s - m), (s - W0 + 1) >> 1);  // ceil((s - W0) / 2)
+      const int hi = min(min(k, s - 1), (s + W0) >> 1);
+      for (int i = lo + lane; i <= hi; i += 32) {
+        const int j = s - i;
+        const int up = p1[i - 1], left = p1[i], dg = p2[i - 1];
+        int best = dg, dir = 0;
+        if (up < best) { best = up; dir = 1; }
+        if (left < best) { best = left; dir = 2; }
+        uint8_t* cell = sm.tile + size_t(i - 1) * TW + (j - max(1, i - W0));
+        int cost = *cell;
+        if (cost == 255) cost = token_cost(i, j);
+        cur[i] = best >= kInf ? kInf : best + cost;
+        *cell = uint8_t(dir);
+      }
+      if (lane == 0) {  // guards: neighbours just outside the diagonal read as infinite
+        if (lo - 1 >= 0) cur[lo - 1] = kInf;
+        if (hi + 1 <= k + 1) cur[hi + 1] = kInf;
+      }
+      __syncwarp();
+    }
+    cstar = D[(k + m) % 3][k];
   }
-  const int cstar = D[(k + m) % 3][k];
 
   // 3. backtrack on lane 0, from (k, m) to (1, 1)
   int L = 0;
@@ -268,7 +388,7 @@ __global__ void __launch_bounds__(kAlignWarpsMax * 32)
 
 size_t align_smem_per_warp(int max_k, int max_m, int tile_w) {
   size_t n = sizeof(uint64_t) * (max_k + max_m) + sizeof(int32_t) * 3 * (max_k + 2) +
-             sizeof(uint32_t) * (max_k + max_m) + sizeof(uint16_t) * size_t(max_k) * tile_w +
+             sizeof(uint32_t) * (max_k + max_m) + ((size_t(max_k) * tile_w + 15) & ~size_t(15)) +
              sizeof(uint16_t) * (max_k + max_m);
   return (n + 15) & ~size_t(15);
 }

@@ -110,11 +110,14 @@ def _random_pairs(rng, B, kmax, mmax, vocab_sz, max_len, empty_ok=False):
 
 
 @pytest.mark.parametrize("max_len,kmax,mmax,nvoc", [(8, 9, 13, 300), (24, 6, 6, 300),
-                                                    (3, 70, 40, 150), (8, 1, 1, 300)])
+                                                    (3, 70, 40, 150), (8, 1, 1, 300),
+                                                    (3, 256, 512, 150), (256, 4, 4, 60)])
 def test_align_random_pairs_and_token_lengths(max_len, kmax, mmax, nvoc):
     """Random byte strings (zero and 0xff bytes, empty strings, tokens longer
     than 8 bytes take the plain dynamic program), random k and m with
-    |k - m| often above the window."""
+    |k - m| often above the window; the largest tile (256 x 512 tokens with no
+    band); tokens up to 256 bytes, whose distances can reach 255 and more (the
+    one-byte cost tile's escape, recomputed in the sweep)."""
     rng = np.random.default_rng(max_len * 100 + kmax)
     voc, d_off, d_ids, t_off, t_ids = _random_pairs(rng, 40, kmax, mmax, nvoc, max_len,
                                                     empty_ok=True)

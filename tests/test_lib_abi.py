@@ -151,17 +151,6 @@ def test_sharded_verify_host_rules(lib):
     assert call(prm, 8) == binding.TT_ERR_INVALID_ARG
 
 
-def test_alignment_tile_too_large_is_unsupported(lib):
-    # no band with 256 x 512 tokens needs a 256 KB tile per pair: refused, not launched
-    b = tt.Batch.from_host([0, 2], [1, 2], [0, 3], [1, 2, 3], device="cpu", max_k=256, max_m=512)
-    vd = tt.VocabTable.from_host([97, 98, 99], [0, 1, 2, 3], device="cpu")
-    keep = []
-    code = lib.tt_align(ctypes.byref(b._c()), ctypes.byref(vd._c()), ctypes.byref(vd._c()),
-                        ctypes.byref(binding.Params(window=-1)._c(keep)), None, None, None, None,
-                        ctypes.c_void_p(16), None)
-    assert code == binding.TT_ERR_UNSUPPORTED
-
-
 def test_workspace_bytes_grow_with_the_batch(lib):
     small = tt.Batch.from_host([0, 2], [1, 2], [0, 3], [1, 2, 3], device="cpu")
     big = tt.Batch.from_host([0, 20], list(range(20)), [0, 30], list(range(30)), device="cpu")
