@@ -14,6 +14,7 @@
 
 #include "tt_device.cuh"
 #include "tt_launch.h"
+#include "tt_f2.cuh"
 
 namespace tt {
 
@@ -25,10 +26,6 @@ constexpr int kDecSmemMax = 64 * 1024;  // largest dynamic shared memory of a de
 // Dynamic shared memory up to which a decision CTA fits beside three row-pass
 // CTAs on one SM (3 x 66 KB of the 228 KB, less per-CTA reservations).
 constexpr int kDecSmemBeside = 24 * 1024;
-
-__device__ __forceinline__ void grid_dependency_wait() {
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-}
 
 __device__ __forceinline__ float load_dt(const char* row, int dt, int64_t col) {
   return dt == TT_F32 ? load_logit<TT_F32>(row, col) : load_logit<TT_BF16>(row, col);
@@ -48,37 +45,7 @@ __device__ __forceinline__ float load_checked(const DecideArgs& a, const RowSet&
 // ------------------------------------------------------------------------
 // Arithmetic of the decision kernel. Row normalisers are fp32 with compensated
 // (TwoSum) reductions and exactly split exponents; the prefix scans that pick
-// the next token run in fp64.
-
-struct F2 {  // unevaluated sum hi + lo
-  float hi, lo;
-};
-
-__device__ __forceinline__ F2 two_sum(float a, float b) {
-  const float s = __fadd_rn(a, b);
-  const float bb = __fsub_rn(s, a);
-  return {s, __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb))};
-}
-
-__device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
-  const F2 s = two_sum(a.hi, b.hi);
-  const float lo = __fadd_rn(s.lo, __fadd_rn(a.lo, b.lo));
-  const float hi = __fadd_rn(s.hi, lo);
-  return {hi, __fsub_rn(lo, __fsub_rn(hi, s.hi))};
-}
-
-// 2^(z * scale - M) with the exponent split exactly into n + f, |f| <= 1/2:
-// z * scale = xh + xl and xh - M = dh + dl are error-free transformations, so
-// only 2^f (from the SFU, relative error about 2^-22) is approximate.
-__device__ __forceinline__ float exp2_scaled(float z, float scale, float M) {
-  const float xh = __fmul_rn(z, scale);
-  const float xl = fmaf(z, scale, -xh);
-  const F2 d = two_sum(xh, -M);
-  const float n = rintf(d.hi);
-  const float f = __fadd_rn(__fsub_rn(d.hi, n), __fadd_rn(d.lo, xl));
-  if (!(n > -126.f)) return 0.f;
-  return ex2_approx(f) * __int_as_float((int(n) + 127) << 23);
-}
+// the next token run in compensated pairs (tt_f2.cuh).
 
 struct RowResult {
   float M, S;  // reference maximum and sum of 2^(s - M) over the whole row
@@ -94,28 +61,10 @@ __device__ __forceinline__ RowResult with_token(float mx, float S, float zt, flo
 
 __device__ __forceinline__ F2 f2_neg(F2 a) { return {-a.hi, -a.lo}; }
 
-// a * b as a normalised pair (the product's rounding error from a fused
-// multiply-add).
-__device__ __forceinline__ F2 f2_mul_f(F2 a, float b) {
-  const float p = __fmul_rn(a.hi, b);
-  const float e = fmaf(a.hi, b, -p);
-  const float lo = fmaf(a.lo, b, e);
-  const float hi = __fadd_rn(p, lo);
-  return {hi, __fsub_rn(lo, __fsub_rn(hi, p))};
-}
-
-// Order of normalised pairs (hi = fl(hi + lo)): lexicographic, which is the
-// order of their values. Intervals whose ends are the same pairs tile exactly.
-__device__ __forceinline__ bool f2_lt(F2 a, F2 b) {
-  return a.hi < b.hi || (a.hi == b.hi && a.lo < b.lo);
-}
 __device__ __forceinline__ bool f2_le(F2 a, F2 b) {
   return a.hi < b.hi || (a.hi == b.hi && a.lo <= b.lo);
 }
 
-__device__ __forceinline__ F2 shfl_up_f2(F2 v, int o, int width) {
-  return {__shfl_up_sync(0xffffffffu, v.hi, o, width), __shfl_up_sync(0xffffffffu, v.lo, o, width)};
-}
 __device__ __forceinline__ F2 shfl_f2(F2 v, int src, int width) {
   return {__shfl_sync(0xffffffffu, v.hi, src, width), __shfl_sync(0xffffffffu, v.lo, src, width)};
 }
