@@ -316,7 +316,9 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
     r.work = ws.work;
     d.err = ws.err;
     d.epoch = r.epoch;
-    if ((e = launch_rowpass(r, draft->dtype, TT_F32, s, sm_count_current(), true)) != cudaSuccess)
+    // (the absent family's type is a placeholder: the draft's, one kernel variant)
+    if ((e = launch_rowpass(r, draft->dtype, draft->dtype, s, sm_count_current(), true)) !=
+        cudaSuccess)
       return cuda_fail(e);
   }
   if (kd > 0) {
@@ -393,7 +395,7 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   r.work = full_q ? ws.work : nullptr;  // zeroed by the prep kernel
   // the first kernel of the chain starts only after the caller's work is
   // complete: it reads the logits before its grid-dependency wait
-  if ((e = launch_rowpass(r, full_q ? draft->dtype : TT_F32, target->dtype, s,
+  if ((e = launch_rowpass(r, full_q ? draft->dtype : target->dtype, target->dtype, s,
                           sm_count_current(), full_q)) != cudaSuccess)
     return cuda_fail(e);
 
@@ -508,7 +510,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   // programmatic dependent launch: target rows stream while the alignment runs
   // (unless stage events sit between the kernels)
   const bool pdl = prm->events == nullptr;
-  if ((e = launch_rowpass(r, from_logits ? draft->dtype : TT_F32, target->dtype, s,
+  if ((e = launch_rowpass(r, from_logits ? draft->dtype : target->dtype, target->dtype, s,
                           sm_count_current(), pdl)) != cudaSuccess)
     return cuda_fail(e);
   record(prm, 2, s);
@@ -672,8 +674,8 @@ tt_status tt_verify_sharded(const tt_batch* batch, const float* q_hat, const tt_
     r.work = reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(ws.work) +
                                                    size_t(k) * kWorkShards * kWorkStride *
                                                        sizeof(unsigned long long));
-    if ((e = launch_rowpass(r, TT_F32, target->shards[k].dtype, s, sm_count_current(), k > 0)) !=
-        cudaSuccess)
+    if ((e = launch_rowpass(r, target->shards[k].dtype, target->shards[k].dtype, s,
+                            sm_count_current(), k > 0)) != cudaSuccess)
       return cuda_fail(e);
   }
   if ((e = launch_shard_summary(a, s, sm_count_current())) != cudaSuccess) return cuda_fail(e);

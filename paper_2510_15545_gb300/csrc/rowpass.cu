@@ -16,6 +16,7 @@
 // an error word that the decision kernel turns into a per-request status.
 #include <algorithm>
 #include <cstdint>
+#include <cstdlib>
 
 #include "tt_device.cuh"
 #include "tt_launch.h"
@@ -94,13 +95,14 @@ __device__ __forceinline__ uint64_t global_ns() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
-// Waits for the phase of the given parity to complete; false after kWaitLimitNs.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// Waits for the phase of the given parity to complete; false after limit_ns.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
+                                          const uint64_t& limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   for (uint32_t i = 1; i < (1u << 30); ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 63) == 0 && global_ns() - t0 > kWaitLimitNs) return false;
+    if ((i & 63) == 0 && global_ns() - t0 > limit_ns) return false;
   }
   return false;
 }
@@ -534,7 +536,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
         d.n_smem = int(bytes) / esz;
         const int s = it % R::kStages;
         const uint32_t par = ((it / R::kStages) & 1) ^ 1;
-        if (!mbar_wait(&empty[s], par)) {
+        if (!mbar_wait(&empty[s], par, a.wait_ns)) {
           report_error(a.err, a.epoch, TT_REQ_TIMEOUT);
           return false;
         }
@@ -627,7 +629,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       for (int w = 0; ok && w < kConsumerWarps; ++w) {
         const int s = it % R::kStages;
         const uint32_t par = ((it / R::kStages) & 1) ^ 1;
-        if (!mbar_wait(&empty[s], par)) {
+        if (!mbar_wait(&empty[s], par, a.wait_ns)) {
           report_error(a.err, a.epoch, TT_REQ_TIMEOUT);
           ok = false;
           break;
@@ -647,7 +649,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
   for (int it = warp;; it += kConsumerWarps) {
     const int s = it % R::kStages;
     const uint32_t par = (it / R::kStages) & 1;
-    if (!mbar_wait(&full[s], par)) {
+    if (!mbar_wait(&full[s], par, a.wait_ns)) {
       if (lane == 0) report_error(a.err, a.epoch, TT_REQ_TIMEOUT);
       break;
     }
@@ -664,7 +666,8 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       } else {
         select_unit<DTD>(stage, d, a.d, lane, S.top_k, scratch, out);
       }
-      if (lane == 0) mbar_arrive(&empty[s]);  // the stage's bytes are consumed
+      if (lane == 0 && !(blockIdx.x == 0 && it == a.stall_stage))
+        mbar_arrive(&empty[s]);  // the stage's bytes are consumed
       continue;
     }
     float m[2], sum[2];
@@ -686,7 +689,10 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       }
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(&empty[s]);  // the stage's bytes are consumed
+    // (test hook: in CTA 0 the consumer of its stall_stage-th stage never frees
+    // it, so the producer's bounded wait for it runs out, then the others')
+    if (lane == 0 && !(blockIdx.x == 0 && it == a.stall_stage))
+      mbar_arrive(&empty[s]);  // the stage's bytes are consumed
     const RowSet& S = d.set ? a.t : a.d;
 #pragma unroll
     for (int c = 0; c < 2; ++c) {
@@ -765,8 +771,20 @@ cudaError_t preload_rowpass() {
   return preload_pair<TT_BF16, TT_BF16>();
 }
 
-cudaError_t launch_rowpass(const RowPassArgs& a, int dt_d, int dt_t, cudaStream_t stream,
+// Test hooks, read from the environment at each launch (off unless set):
+// TT_TEST_STALL_STAGE=n makes CTA 0 hold the stage of its n-th consumer step, and
+// TT_TEST_WAIT_MS=t sets the limit of every pipeline wait, so that a test can
+// watch the bounded waits run out and the call report TT_REQ_TIMEOUT.
+cudaError_t launch_rowpass(const RowPassArgs& args, int dt_d, int dt_t, cudaStream_t stream,
                            int sm_count, bool pdl) {
+  RowPassArgs a = args;
+  a.stall_stage = -1;
+  a.wait_ns = kWaitLimitNs;
+  if (const char* v = std::getenv("TT_TEST_STALL_STAGE")) a.stall_stage = std::atoi(v);
+  if (const char* v = std::getenv("TT_TEST_WAIT_MS")) {
+    const long long ms = std::atoll(v);
+    if (ms > 0) a.wait_ns = uint64_t(ms) * 1000000ull;
+  }
   if (dt_d == TT_F32 && dt_t == TT_F32) return launch_pair<TT_F32, TT_F32>(a, stream, sm_count, pdl);
   if (dt_d == TT_F32 && dt_t == TT_BF16) return launch_pair<TT_F32, TT_BF16>(a, stream, sm_count, pdl);
   if (dt_d == TT_BF16 && dt_t == TT_F32) return launch_pair<TT_BF16, TT_F32>(a, stream, sm_count, pdl);

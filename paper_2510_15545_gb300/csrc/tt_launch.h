@@ -67,6 +67,10 @@ struct RowPassArgs {
   // this one depends on and read only after the grid-dependency wait; NULL:
   // every item belongs to a fixed share.
   unsigned long long* work;
+  int32_t stall_stage;       // test hook (-1 = off): in CTA 0 the stage consumed at
+                             // consumer step stall_stage is never freed, so the
+                             // bounded waits run out
+  uint64_t wait_ns;          // limit of every pipeline wait (set by launch_rowpass: 2 s)
 };
 
 struct DecideArgs {
