@@ -184,6 +184,18 @@ __device__ __forceinline__ float raw_max_plain(const uint4* sv, int lane) {
   }
 }
 
+// A unit's family as a consumer sees it: the kernel's arguments and which of
+// the two families (d.set) the unit belongs to, so that both families share
+// one copy of the code; the row's base is formed only where a ragged tail is
+// read directly.
+struct RowView {
+  const RowPassArgs& a;
+  float scale;
+  __device__ __forceinline__ const char* row(const Desc& d) const {
+    return d.set ? a.t.data + d.row * a.t.stride_bytes : a.d.data + d.row * a.d.stride_bytes;
+  }
+};
+
 // One consumer warp reduces one chunk held in shared memory (plus a ragged
 // tail of fewer than 16 bytes read directly) to (max, sum of 2^(s - max)).
 // The stage is read twice (max, then sum) rather than held in registers.
@@ -218,8 +230,22 @@ __device__ __forceinline__ void reduce_stage(const uint4* sv, const Desc& d, flo
   }
 }
 
+// The chunks that are not whole or hold the scored column -- at most two per
+// row -- take this out-of-line copy, which keeps the consumer loop's code (and
+// its share of the instruction cache) to the whole-chunk path.
 template <int DT>
-__device__ __forceinline__ void reduce_chunk(const char* stage, const Desc& d, const RowSet& S,
+__device__ __noinline__ float2 reduce_stage_edge(const uint4* sv, int n_smem, int excl, float scale,
+                                                 int lane, float mx) {
+  Desc d;
+  d.n_smem = n_smem;  // the only fields the per-element checks read
+  d.excl = excl;
+  float sum = 0.f;
+  reduce_stage<DT, false>(sv, d, scale, lane, mx, sum);
+  return make_float2(mx, sum);
+}
+
+template <int DT>
+__device__ __forceinline__ void reduce_chunk(const char* stage, const Desc& d, const RowView& S,
                                              int lane, float& m_out, float& s_out) {
   const uint4* sv = reinterpret_cast<const uint4*>(stage);
   const float scale = S.scale;
@@ -229,15 +255,16 @@ __device__ __forceinline__ void reduce_chunk(const char* stage, const Desc& d, c
   if (lane < tail) {
     const int e = d.n_smem + lane;
     if (e != d.excl) {
-      const char* row = S.data + d.row * S.stride_bytes;
-      ztail = load_logit<DT>(row, int64_t(d.chunk) * kChunk + e) * scale;
+      ztail = load_logit<DT>(S.row(d), int64_t(d.chunk) * kChunk + e) * scale;
     }
   }
   float mx = ztail, sum = 0.f;
   if (d.n_smem == kChunk && d.excl < 0) {
     reduce_stage<DT, true>(sv, d, scale, lane, mx, sum);
   } else {
-    reduce_stage<DT, false>(sv, d, scale, lane, mx, sum);
+    const float2 r = reduce_stage_edge<DT>(sv, d.n_smem, d.excl, scale, lane, mx);
+    mx = r.x;
+    sum = r.y;
   }
   if (ztail != -INFINITY) sum += ex2_approx(ztail - mx);
   m_out = mx;
@@ -280,7 +307,7 @@ __device__ __forceinline__ float vec_max(const uint4& w) {
 // the same vectors instead. The work per unit is thus nearly the same for
 // every unit, which keeps the stage ring from waiting on one slow warp.
 template <int DT>
-__device__ void select_unit(const char* stage, const Desc& d, const RowSet& S, int lane, int K,
+__device__ void select_unit(const char* stage, const Desc& d, const RowView& S, int lane, int K,
                             Cand* scratch, Cand* out) {
   constexpr int VEC = DT == TT_F32 ? 4 : 8;  // logits per 16-byte vector
   constexpr int NV = kChunk * 4 / (16 * 32);   // vectors per lane in one stage
@@ -295,8 +322,7 @@ __device__ void select_unit(const char* stage, const Desc& d, const RowSet& S, i
   // the tail element, NaN where the lane has none (NaN never compares >=)
   float zt = kNaN;
   if (has_tail) {
-    const char* row = S.data + d.row * S.stride_bytes;
-    zt = load_logit<DT>(row, int64_t(col0) + d.n_smem + lane);
+    zt = load_logit<DT>(S.row(d), int64_t(col0) + d.n_smem + lane);
   }
   const uint32_t valid = ((1u << nvl) - 1) | (has_tail ? kTailBit : 0u);
   float vm[NV];  // vector maxima; -inf for a vector past the copy
@@ -661,10 +687,13 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
     if (SEL && (d.set ? a.t : a.d).top_k > 0) {  // filtered rows: the unit's top-k list
       const RowSet& S = d.set ? a.t : a.d;
       Cand* out = S.cand + (d.row * S.nlist + d.chunk / cps) * cand_stride(S.top_k);
-      if (d.set) {
-        select_unit<DTT>(stage, d, a.t, lane, S.top_k, scratch, out);
+      const RowView V = {a, S.scale};
+      if constexpr (DTD == DTT) {
+        select_unit<DTT>(stage, d, V, lane, S.top_k, scratch, out);
+      } else if (d.set) {
+        select_unit<DTT>(stage, d, V, lane, S.top_k, scratch, out);
       } else {
-        select_unit<DTD>(stage, d, a.d, lane, S.top_k, scratch, out);
+        select_unit<DTD>(stage, d, V, lane, S.top_k, scratch, out);
       }
       if (lane == 0 && !(blockIdx.x == 0 && it == a.stall_stage))
         mbar_arrive(&empty[s]);  // the stage's bytes are consumed
@@ -682,10 +711,12 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       e.n = min(kChunk, d.n - lo);
       e.n_smem = max(0, min(kChunk, d.n_smem - lo));
       e.excl = (d.excl >= lo && d.excl < lo + kChunk) ? d.excl - lo : -1;
+      // (one copy per family here: shared, the bf16 kernel needs more
+      // registers than the decision kernel beside it leaves)
       if (d.set) {
-        reduce_chunk<DTT>(stage + size_t(lo) * esz, e, a.t, lane, m[c], sum[c]);
+        reduce_chunk<DTT>(stage + size_t(lo) * esz, e, RowView{a, a.t.scale}, lane, m[c], sum[c]);
       } else {
-        reduce_chunk<DTD>(stage + size_t(lo) * esz, e, a.d, lane, m[c], sum[c]);
+        reduce_chunk<DTD>(stage + size_t(lo) * esz, e, RowView{a, a.d.scale}, lane, m[c], sum[c]);
       }
     }
     __syncwarp();
