@@ -699,24 +699,32 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
         mbar_arrive(&empty[s]);  // the stage's bytes are consumed
       continue;
     }
-    float m[2], sum[2];
-#pragma unroll
-    for (int c = 0; c < 2; ++c) {  // the unit's chunks, each reduced on its own
-      m[c] = -INFINITY;
-      sum[c] = 0.f;
+    // the unit's chunks (two for bf16 rows), each reduced on its own by one
+    // copy of the code; the results are named, not indexed, to stay in registers
+    float m0 = -INFINITY, s0 = 0.f, m1 = -INFINITY, s1 = 0.f;
+#pragma unroll 1
+    for (int c = 0; c < cps; ++c) {
       const int lo = c * kChunk;
-      if (c >= cps || lo >= d.n) continue;
+      if (lo >= d.n) break;
       Desc e = d;
       e.chunk = d.chunk + c;
       e.n = min(kChunk, d.n - lo);
       e.n_smem = max(0, min(kChunk, d.n_smem - lo));
       e.excl = (d.excl >= lo && d.excl < lo + kChunk) ? d.excl - lo : -1;
+      float mc = -INFINITY, sc = 0.f;
       // (one copy per family here: shared, the bf16 kernel needs more
       // registers than the decision kernel beside it leaves)
       if (d.set) {
-        reduce_chunk<DTT>(stage + size_t(lo) * esz, e, RowView{a, a.t.scale}, lane, m[c], sum[c]);
+        reduce_chunk<DTT>(stage + size_t(lo) * esz, e, RowView{a, a.t.scale}, lane, mc, sc);
       } else {
-        reduce_chunk<DTD>(stage + size_t(lo) * esz, e, RowView{a, a.d.scale}, lane, m[c], sum[c]);
+        reduce_chunk<DTD>(stage + size_t(lo) * esz, e, RowView{a, a.d.scale}, lane, mc, sc);
+      }
+      if (c == 0) {
+        m0 = mc;
+        s0 = sc;
+      } else {
+        m1 = mc;
+        s1 = sc;
       }
     }
     __syncwarp();
@@ -725,11 +733,12 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
     if (lane == 0 && !(blockIdx.x == 0 && it == a.stall_stage))
       mbar_arrive(&empty[s]);  // the stage's bytes are consumed
     const RowSet& S = d.set ? a.t : a.d;
-#pragma unroll
-    for (int c = 0; c < 2; ++c) {
-      if (c >= cps || c * kChunk >= d.n) continue;
-      warp_merge_ms(m[c], sum[c]);
-      if (lane == 0) S.part[d.row * S.nch + d.chunk + c] = Partial{m[c], sum[c]};
+    if (d.n <= 0) continue;  // nothing copied (a failed check: the row may not exist)
+    warp_merge_ms(m0, s0);
+    if (lane == 0) S.part[d.row * S.nch + d.chunk] = Partial{m0, s0};
+    if (cps > 1 && kChunk < d.n) {
+      warp_merge_ms(m1, s1);
+      if (lane == 0) S.part[d.row * S.nch + d.chunk + 1] = Partial{m1, s1};
     }
   }
 }
