@@ -712,9 +712,12 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       e.n_smem = max(0, min(kChunk, d.n_smem - lo));
       e.excl = (d.excl >= lo && d.excl < lo + kChunk) ? d.excl - lo : -1;
       float mc = -INFINITY, sc = 0.f;
-      // (one copy per family here: shared, the bf16 kernel needs more
-      // registers than the decision kernel beside it leaves)
-      if (d.set) {
+      // fp32 rows: one copy for both families; bf16 rows: one per family (shared,
+      // the kernel needs more registers than the decision kernel beside it leaves)
+      if constexpr (DTD == TT_F32 && DTT == TT_F32) {
+        reduce_chunk<TT_F32>(stage + size_t(lo) * esz, e,
+                             RowView{a, d.set ? a.t.scale : a.d.scale}, lane, mc, sc);
+      } else if (d.set) {
         reduce_chunk<DTT>(stage + size_t(lo) * esz, e, RowView{a, a.t.scale}, lane, mc, sc);
       } else {
         reduce_chunk<DTD>(stage + size_t(lo) * esz, e, RowView{a, a.d.scale}, lane, mc, sc);
