@@ -356,8 +356,9 @@ def run_mine(args):
 
     call = tt.StepCall(batch, vd, vt, dl, tl, prm, out=tt.step_outputs(batch, dev, full=False),
                        stream=stream)
-    # stage events on a strided subset of the timed steps
-    stride = max(1, math.ceil(K / 2000))
+    # stage events on a strided subset of the timed steps: at most one step in
+    # ten (events between the kernels break their dependent-launch overlap)
+    stride = max(10, math.ceil(K / 2000))
     sampled = list(range(0, K, stride))
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in sampled]
     for e4 in ev:

@@ -11,6 +11,7 @@
 //     tile (diagonal, then (i-1,j), then (i,j-1) on ties);
 //  4. backtrack from (k, m) on one lane, then write path, C*, the map
 //     i*(j) = max{i : (i,j) on the path} and the needed-draft-row flags.
+#include <algorithm>
 #include <cstdint>
 
 #include "tt_device.cuh"
@@ -140,19 +141,10 @@ __device__ __forceinline__ PairSmem carve(char* base, int K, int M, int TW) {
   return s;
 }
 
-__global__ void __launch_bounds__(kAlignWarpsMax * 32)
-    align_kernel(AlignArgs a) {
-  extern __shared__ __align__(16) char smem_raw[];
-  // the row pass may start streaming target rows now; it waits for this grid
-  // before it reads the needed-draft-row flags
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  if (a.work && blockIdx.x == 0 && threadIdx.x < kWorkShards)
-    a.work[threadIdx.x * kWorkStride] = 0ull;  // read after this grid ends
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int b = blockIdx.x * a.warps_per_block + warp;
-  if (b >= a.B) return;
+// One warp aligns pair b in its own shared-memory region.
+__device__ __forceinline__ void align_pair(const AlignArgs& a, int b, char* region, int lane) {
   const int K = a.max_k, M = a.max_m, TW = a.tile_w;
-  PairSmem sm = carve(smem_raw + size_t(warp) * a.smem_per_warp, K, M, TW);
+  PairSmem sm = carve(region, K, M, TW);
 
   if (!csr_ok(a.draft_off, b, a.n_draft) || !csr_ok(a.target_off, b, a.n_target)) {
     if (lane == 0) {
@@ -384,6 +376,25 @@ __global__ void __launch_bounds__(kAlignWarpsMax * 32)
   }
 }
 
+// At most one CTA per SM, its warps looping over the pairs: the row pass's
+// CTAs fit beside it and stream target rows while the pairs are aligned.
+__global__ void __launch_bounds__(kAlignWarpsMax * 32)
+    align_kernel(AlignArgs a) {
+  extern __shared__ __align__(16) char smem_raw[];
+  // the row pass may start streaming target rows now; it waits for this grid
+  // before it reads the needed-draft-row flags
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (a.work && blockIdx.x == 0 && threadIdx.x < kWorkShards)
+    a.work[threadIdx.x * kWorkStride] = 0ull;  // read after this grid ends
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  char* region = smem_raw + size_t(warp) * a.smem_per_warp;
+  for (int b = blockIdx.x * a.warps_per_block + warp; b < a.B;
+       b += int(gridDim.x) * a.warps_per_block) {
+    align_pair(a, b, region, lane);
+    __syncwarp();  // the region is reused by the warp's next pair
+  }
+}
+
 }  // namespace
 
 size_t align_smem_per_warp(int max_k, int max_m, int tile_w) {
@@ -404,7 +415,14 @@ cudaError_t preload_align() {
 }
 
 cudaError_t launch_align(const AlignArgs& args, cudaStream_t stream) {
-  const int blocks = (args.B + args.warps_per_block - 1) / args.warps_per_block;
+  static int n_sm[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
+  if (n_sm[dev] == 0 &&
+      cudaDeviceGetAttribute(&n_sm[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    n_sm[dev] = 148;
+  const int blocks = std::min((args.B + args.warps_per_block - 1) / args.warps_per_block,
+                              n_sm[dev]);
   const size_t smem = args.smem_per_warp * size_t(args.warps_per_block);
   align_kernel<<<blocks, args.warps_per_block * 32, smem, stream>>>(args);
   return cudaGetLastError();

@@ -3,6 +3,7 @@
 // launch sequences of align / transfer / verify / step.
 #include <atomic>
 #include <cmath>
+#include <algorithm>
 #include <cstdint>
 #include <cstring>
 
@@ -196,9 +197,13 @@ tt_status fill_align_args(const tt_batch* bt, const tt_vocab* vd, const tt_vocab
   a.tile_w = align_tile_width(bt->max_k, bt->max_m, prm->window);
   a.smem_per_warp = align_smem_per_warp(bt->max_k, bt->max_m, a.tile_w);
   if (a.smem_per_warp > size_t(kAlignSmemMax)) return TT_ERR_UNSUPPORTED;
+  // pairs spread over the SMs (one warp each while the batch is small), at
+  // most kAlignWarpsMax warps and 96 KB per CTA; launch_align caps the grid at
+  // one CTA per SM, whose warps then loop over the pairs
   int wpb = int(size_t(96 * 1024) / a.smem_per_warp);
-  wpb = wpb < 1 ? 1 : (wpb > kAlignWarpsMax ? kAlignWarpsMax : wpb);
-  a.warps_per_block = wpb;
+  const int spread = (bt->B + sm_count_current() - 1) / sm_count_current();
+  wpb = std::min(wpb, std::min(kAlignWarpsMax, spread));
+  a.warps_per_block = wpb < 1 ? 1 : wpb;
   return TT_OK;
 }
 

@@ -11,7 +11,7 @@ namespace tt {
 
 struct Partial;
 
-constexpr int kAlignWarpsMax = 4;             // sequence pairs per align CTA
+constexpr int kAlignWarpsMax = 8;             // warps (pairs at a time) per align CTA
 constexpr int kAlignSmemMax = 200 * 1024;     // dynamic shared memory cap of one align CTA
 constexpr int kMaxChunksPerRow = 1024;        // rows up to 1024 * 2048 = 2,097,152 columns
 
