@@ -197,10 +197,12 @@ def rowpass_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload: str):
+def profiled_traffic(workload: str, top_k: int = 0):
     """DRAM bytes per row-pass launch from the committed ncu summary, if it was
-    taken on the current row-pass source."""
-    path = os.path.join(ROOT, "profiles", "rowpass_%s.md" % workload)
+    taken on the current row-pass source (and, with filters, at the same top_k:
+    the lists the pass writes are top_k entries per unit)."""
+    name = "rowpass_filtered_%s.md" if top_k > 0 else "rowpass_%s.md"
+    path = os.path.join(ROOT, "profiles", name % workload)
     try:
         txt = open(path).read()
     except OSError:
@@ -211,6 +213,8 @@ def profiled_traffic(workload: str):
             k, v = line.strip()[2:].split(":", 1)
             vals[k.strip()] = v.strip().strip("`")
     if vals.get("source_sha256") != rowpass_source_hash():
+        return None
+    if top_k > 0 and vals.get("top_k") != str(top_k):
         return None
     try:
         return float(vals["traffic_bytes_per_launch"])
@@ -402,12 +406,13 @@ def run_mine(args):
     peak, peak_kind = measured_hbm_peak()
     achieved = ab["total"] / (row_ms / 1e3) / 1e9
     step_gbs = ab["total"] / (sec / K) / 1e9
-    traffic = profiled_traffic(name) if not filtered else None  # captured without filters
+    traffic = profiled_traffic(name, args.top_k)
 
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(tt, wl, inp, prm, dev, stream, K, ws)
 
+    align_alone_ms = run_align_alone(tt, wl, inp, prm, dev, stream)
     reenc = None if args.no_reencode else run_reencode(tt, wl, inp, prm, dev, stream, rank, ws)
     sharded = None
     if args.shards > 0 and not filtered and not prm.full_q:
@@ -441,7 +446,11 @@ def run_mine(args):
                    "accept_rate": float(acc.sum() / max(1, m.sum())),
                    "mean_accepted": float(acc.mean())},
         "hbm_gbs_step": step_gbs,
-        "dtw_pairs_per_s": wl.B / (align_ms / 1e3),
+        "dtw_pairs_per_s": wl.B / (align_alone_ms / 1e3),
+        "dtw": {"ms_alone": align_alone_ms, "ms_in_step": align_ms,
+                "pairs_per_s_in_step": wl.B / (align_ms / 1e3),
+                "note": "dtw_pairs_per_s: tt_align alone (one warp per pair), 200 calls; in "
+                        "the step the alignment takes one CTA per SM beside the row pass"},
         "stage_ms": {"align": align_ms, "rowpass": row_ms, "decide": dec_ms,
                      "sampled_steps": len(sampled)},
         "roofline": {"bound": "hbm", "kernel": "rowpass_kernel", "achieved": achieved,
@@ -481,6 +490,22 @@ def _time_calls(fn, stream, n, warm=3):
     e1.record(stream)
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) / n  # ms per call
+
+
+def run_align_alone(tt, wl, inp, prm, dev, stream):
+    """tt_align on its own (DTW and the map i*(j), nothing after it), timed with
+    CUDA events over repeated calls outside the step's timed region. Alone it
+    takes one warp per pair and as many CTAs as fit; inside tt_step the same
+    kernel runs on one CTA per SM so that the row pass streams beside it."""
+    import torch
+    out = {"path": torch.empty(2 * (wl.n_draft + wl.n_target), dtype=torch.int32, device=dev),
+           "path_len": torch.empty(wl.B, dtype=torch.int32, device=dev),
+           "cost": torch.empty(wl.B, dtype=torch.int32, device=dev),
+           "map": torch.empty(max(1, wl.n_target), dtype=torch.int32, device=dev),
+           "status": torch.empty(wl.B, dtype=torch.int32, device=dev)}
+    ms = _time_calls(lambda: tt.tt_align(inp["batch"], inp["vd"], inp["vt"], prm, out=out,
+                                         stream=stream), stream, 200)
+    return ms
 
 
 def run_sharded(tt, wl, inp, prm, q_hat, dev, stream, S):

@@ -421,8 +421,12 @@ cudaError_t launch_align(const AlignArgs& args, cudaStream_t stream) {
   if (n_sm[dev] == 0 &&
       cudaDeviceGetAttribute(&n_sm[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     n_sm[dev] = 148;
-  const int blocks = std::min((args.B + args.warps_per_block - 1) / args.warps_per_block,
-                              n_sm[dev]);
+  // A grid followed by the row pass (it zeroes the row pass's work counters)
+  // takes at most one CTA per SM, whose warps loop over the pairs, so that the
+  // row pass's CTAs fit beside it and stream target rows while it runs; an
+  // alignment on its own takes one warp per pair and as many CTAs as fit.
+  const int per_pair = (args.B + args.warps_per_block - 1) / args.warps_per_block;
+  const int blocks = args.work ? std::min(per_pair, n_sm[dev]) : per_pair;
   const size_t smem = args.smem_per_warp * size_t(args.warps_per_block);
   align_kernel<<<blocks, args.warps_per_block * 32, smem, stream>>>(args);
   return cudaGetLastError();

@@ -198,8 +198,9 @@ tt_status fill_align_args(const tt_batch* bt, const tt_vocab* vd, const tt_vocab
   a.smem_per_warp = align_smem_per_warp(bt->max_k, bt->max_m, a.tile_w);
   if (a.smem_per_warp > size_t(kAlignSmemMax)) return TT_ERR_UNSUPPORTED;
   // pairs spread over the SMs (one warp each while the batch is small), at
-  // most kAlignWarpsMax warps and 96 KB per CTA; launch_align caps the grid at
-  // one CTA per SM, whose warps then loop over the pairs
+  // most kAlignWarpsMax warps and 96 KB per CTA; before the row pass,
+  // launch_align caps the grid at one CTA per SM, whose warps then loop over
+  // the pairs
   int wpb = int(size_t(96 * 1024) / a.smem_per_warp);
   const int spread = (bt->B + sm_count_current() - 1) / sm_count_current();
   wpb = std::min(wpb, std::min(kAlignWarpsMax, spread));

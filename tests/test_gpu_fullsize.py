@@ -129,3 +129,29 @@ def test_full_size_sharded_verify_sampled():
         oo = dict(o)
         oo["q_hat"] = q[t0:t1]
         compare(sw, gg, oo, req_index=[b], check_align=False)
+
+
+def test_full_size_alignment_alone_and_in_step():
+    """All 4096 pairs of the DTW workload (64 draft tokens, 48..96 target
+    tokens each) against the oracle, in both launch shapes of the alignment
+    kernel: tt_align alone (one warp per pair, more CTAs than SMs) and inside
+    tt_step (one CTA per SM, its warps looping over about 27 pairs each)."""
+    wl = W.make_workload("dtw_4096x64", seed=0, device="cuda")
+    inp = tt.device_inputs(wl, "cuda")
+    prm = inp["params"]
+    o = oracle.align(wl.draft_off, wl.draft_ids, wl.target_off, wl.target_ids, wl.vd.blob,
+                     wl.vd.off, wl.vt.blob, wl.vt.off, prm.window)
+    alone = to_np(tt.tt_align(inp["batch"], inp["vd"], inp["vt"], prm))
+    step = to_np(tt.tt_step(inp["batch"], inp["vd"], inp["vt"], inp["draft_logits"],
+                            inp["target_logits"], prm))
+    torch.cuda.synchronize()
+    assert np.all(o["status"] == 0)
+    for g in (alone, step):
+        assert np.array_equal(g["status"], o["status"])
+        assert np.array_equal(g["path_len"], o["path_len"])
+        assert np.array_equal(g["cost"], o["cost"])
+        assert np.array_equal(g["map"], o["map"])
+        for b in range(wl.B):
+            p0 = int(wl.draft_off[b] + wl.target_off[b])
+            L = int(o["path_len"][b])
+            assert np.array_equal(g["path"][2 * p0:2 * (p0 + L)], o["path"][p0:p0 + L].ravel())
