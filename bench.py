@@ -497,15 +497,8 @@ def run_align_alone(tt, wl, inp, prm, dev, stream):
     CUDA events over repeated calls outside the step's timed region. Alone it
     takes one warp per pair and as many CTAs as fit; inside tt_step the same
     kernel runs on one CTA per SM so that the row pass streams beside it."""
-    import torch
-    out = {"path": torch.empty(2 * (wl.n_draft + wl.n_target), dtype=torch.int32, device=dev),
-           "path_len": torch.empty(wl.B, dtype=torch.int32, device=dev),
-           "cost": torch.empty(wl.B, dtype=torch.int32, device=dev),
-           "map": torch.empty(max(1, wl.n_target), dtype=torch.int32, device=dev),
-           "status": torch.empty(wl.B, dtype=torch.int32, device=dev)}
-    ms = _time_calls(lambda: tt.tt_align(inp["batch"], inp["vd"], inp["vt"], prm, out=out,
-                                         stream=stream), stream, 200)
-    return ms
+    call = tt.AlignCall(inp["batch"], inp["vd"], inp["vt"], prm, stream=stream)
+    return _time_calls(call, stream, 200)
 
 
 def run_sharded(tt, wl, inp, prm, q_hat, dev, stream, S):

@@ -285,21 +285,40 @@ def workspace(batch: Batch, V_d: int, V_t: int, device="cuda",
                        device=device)
 
 
+class AlignCall:
+    """A prepared tt_align call: the ctypes argument blocks and the output
+    pointers are built once, so a repeated alignment costs one foreign call."""
+
+    def __init__(self, batch: Batch, vd: VocabTable, vt: VocabTable, params: Params, *,
+                 out=None, stream=None):
+        dev = batch.draft_off.device
+        o = dict(out or {})
+        o.setdefault("path", _empty(2 * (batch.n_draft + batch.n_target), torch.int32, dev))
+        o.setdefault("path_len", _empty(batch.B, torch.int32, dev))
+        o.setdefault("cost", _empty(batch.B, torch.int32, dev))
+        o.setdefault("map", _empty(batch.n_target, torch.int32, dev))
+        o.setdefault("status", _empty(batch.B, torch.int32, dev))
+        self.out = o
+        self._keep = [batch, vd, vt, o]
+        self._b = batch._c()
+        self._vd = vd._c()
+        self._vt = vt._c()
+        self._prm = params._c(self._keep)
+        self._ptrs = [_ptr(o[k]) for k in ("path", "path_len", "cost", "map", "status")]
+        self._stream = _stream(stream)
+        self._lib = load()
+
+    def __call__(self) -> dict:
+        code = self._lib.tt_align(ctypes.byref(self._b), ctypes.byref(self._vd),
+                                  ctypes.byref(self._vt), ctypes.byref(self._prm), *self._ptrs,
+                                  self._stream)
+        _check("tt_align", code)
+        return self.out
+
+
 def tt_align(batch: Batch, vd: VocabTable, vt: VocabTable, params: Params, *, out=None,
              stream=None) -> dict:
-    dev = batch.draft_off.device
-    o = dict(out or {})
-    o.setdefault("path", _empty(2 * (batch.n_draft + batch.n_target), torch.int32, dev))
-    o.setdefault("path_len", _empty(batch.B, torch.int32, dev))
-    o.setdefault("cost", _empty(batch.B, torch.int32, dev))
-    o.setdefault("map", _empty(batch.n_target, torch.int32, dev))
-    o.setdefault("status", _empty(batch.B, torch.int32, dev))
-    keep = []
-    code = load().tt_align(ctypes.byref(batch._c()), ctypes.byref(vd._c()), ctypes.byref(vt._c()),
-                           ctypes.byref(params._c(keep)), _ptr(o["path"]), _ptr(o["path_len"]),
-                           _ptr(o["cost"]), _ptr(o["map"]), _ptr(o["status"]), _stream(stream))
-    _check("tt_align", code)
-    return o
+    return AlignCall(batch, vd, vt, params, out=out, stream=stream)()
 
 
 def tt_transfer(batch: Batch, map: torch.Tensor, params: Params, *, draft_logits=None,
