@@ -1,14 +1,18 @@
 // align.cu -- Dynamic Token Warping between draft and proxy target tokens
 // (§4.1, Alg. 1) with the byte-level Levenshtein token distance (App. H).
 //
-// One warp per request (sequence pair), several pairs per CTA. Per pair:
+// One warp per request (sequence pair), several pairs per CTA, each warp
+// looping over pairs when the grid is smaller than the batch. Per pair:
 //  1. stage the tokens' byte strings in shared memory (packed 8-byte words);
-//  2. fill the banded local-cost tile d(i,j) with all 32 lanes (bit-parallel
-//     edit distance for tokens of <= 8 bytes, a plain DP otherwise);
+//  2. fill the banded local-cost tile d(i,j), one byte per cell, with all 32
+//     lanes (two interleaved bit-parallel edit distances per lane for tokens
+//     of <= 8 bytes, a plain DP otherwise);
 //  3. sweep the anti-diagonals i + j = s: every cell of a diagonal depends
-//     only on the two previous diagonals, kept in three rotating shared
-//     buffers; each cell's choice of predecessor overwrites its cost in the
-//     tile (diagonal, then (i-1,j), then (i,j-1) on ties);
+//     only on the two previous diagonals, kept in registers (one cell per
+//     lane, neighbours by shuffles) while the band's half-width is at most
+//     31, else in three rotating shared buffers; each cell's choice of
+//     predecessor overwrites its cost in the tile (diagonal, then (i-1,j),
+//     then (i,j-1) on ties);
 //  4. backtrack from (k, m) on one lane, then write path, C*, the map
 //     i*(j) = max{i : (i,j) on the path} and the needed-draft-row flags.
 #include <algorithm>
@@ -376,8 +380,9 @@ __device__ __forceinline__ void align_pair(const AlignArgs& a, int b, char* regi
   }
 }
 
-// At most one CTA per SM, its warps looping over the pairs: the row pass's
-// CTAs fit beside it and stream target rows while the pairs are aligned.
+// Before the row pass, at most one CTA per SM whose warps loop over the pairs
+// (the row pass's CTAs fit beside it and stream target rows while the pairs
+// are aligned); alone, one warp per pair (launch_align).
 __global__ void __launch_bounds__(kAlignWarpsMax * 32)
     align_kernel(AlignArgs a) {
   extern __shared__ __align__(16) char smem_raw[];

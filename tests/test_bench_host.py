@@ -1,0 +1,91 @@
+"""Host logic of bench.py on CPU: the default arguments the run contract needs,
+the algorithmic bytes of a step (the roofline's numerator), the rule that a
+committed ncu summary feeds `traffic` only when it was taken on the current
+row-pass source (and, with filters, at the same top-k), and the reference
+arm's JSON line (the oracle on the host cores)."""
+import json
+import os
+import subprocess
+import sys
+from types import SimpleNamespace
+
+import numpy as np
+import pytest
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+def test_defaults_are_one_gpu_and_enough_warmup():
+    a = bench.parse_args([])
+    assert a.gpus == 1 and a.impl == "mine" and a.warmup >= 3
+    assert a.workload == bench.DEFAULT_WORKLOAD
+    assert a.top_k == 0 and a.top_p == 1.0 and a.shards == 0
+
+
+def test_algorithmic_bytes_count_each_distinct_mapped_draft_row_once():
+    # request 0: targets map to draft rows 0, 0, 2 (two distinct rows, 3 target
+    # rows + its bonus row); request 1: one target mapped to row 1 (one distinct
+    # row, 1 target row + bonus)
+    wl = SimpleNamespace(
+        B=2, n_target=4, target_off=np.array([0, 3, 4]),
+        draft_logits=torch.empty(5, 100, dtype=torch.float32),
+        target_logits=torch.empty(6, 300, dtype=torch.bfloat16))
+    mp = np.array([0, 0, 2, 1])
+    ab = bench.algorithmic_bytes(wl, mp)
+    assert ab["draft_rows"] == 3
+    assert ab["target_rows"] == 6
+    assert ab["draft_bytes"] == 3 * 100 * 4
+    assert ab["target_bytes"] == 6 * 300 * 2
+    assert ab["total"] == 1200 + 3600
+
+
+def _summary(path, sha, traffic, top_k=None):
+    lines = ["# a summary", "", "- source_sha256: `%s`" % sha]
+    if top_k is not None:
+        lines.append("- top_k: %d" % top_k)
+    lines.append("- traffic_bytes_per_launch: %d" % traffic)
+    path.write_text("\n".join(lines) + "\n")
+
+
+def test_traffic_only_from_a_summary_of_the_current_source(tmp_path, monkeypatch):
+    (tmp_path / "profiles").mkdir()
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    monkeypatch.setattr(bench, "rowpass_source_hash", lambda: "0123456789abcdef")
+    assert bench.profiled_traffic("wl") is None  # no summary
+    _summary(tmp_path / "profiles" / "rowpass_wl.md", "0123456789abcdef", 123456)
+    assert bench.profiled_traffic("wl") == 123456.0
+    _summary(tmp_path / "profiles" / "rowpass_wl.md", "fedcba9876543210", 123456)
+    assert bench.profiled_traffic("wl") is None  # taken on another source
+    # filtered runs read their own summary, only at the top-k it was taken at
+    assert bench.profiled_traffic("wl", 20) is None
+    _summary(tmp_path / "profiles" / "rowpass_filtered_wl.md", "0123456789abcdef", 777, 20)
+    assert bench.profiled_traffic("wl", 20) == 777.0
+    assert bench.profiled_traffic("wl", 10) is None
+
+
+def test_source_hash_covers_the_row_pass_sources():
+    for rel in bench.ROWPASS_SOURCES:
+        assert os.path.isfile(os.path.join(ROOT, rel)), rel
+    h = bench.rowpass_source_hash()
+    assert len(h) == 16 and int(h, 16) >= 0
+
+
+def test_reference_arm_prints_one_contract_line():
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--workload",
+                        "b1_g4_v32k", "--steps", "2", "--warmup", "3"], cwd=ROOT, env=env,
+                       capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == bench.UNIT
+    assert d["value"] > 0 and d["steps"] == 2 and d["warmup"] >= 3 and d["n_gpus"] == 1
+    assert d["higher_is_better"] is True and d["config"]["workload"] == "b1_g4_v32k"
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}
