@@ -414,6 +414,10 @@ def run_mine(args):
 
     align_alone_ms = run_align_alone(tt, wl, inp, prm, dev, stream)
     reenc = None if args.no_reencode else run_reencode(tt, wl, inp, prm, dev, stream, rank, ws)
+    verify = None
+    if not filtered and not prm.full_q:
+        verify = run_verify_alone(tt, wl, inp, prm, full["q_hat"], dev, stream)
+    cells = band_cells(wl, prm.window)
     sharded = None
     if args.shards > 0 and not filtered and not prm.full_q:
         sharded = run_sharded(tt, wl, inp, prm, full["q_hat"], dev, stream, args.shards)
@@ -449,6 +453,7 @@ def run_mine(args):
         "dtw_pairs_per_s": wl.B / (align_alone_ms / 1e3),
         "dtw": {"ms_alone": align_alone_ms, "ms_in_step": align_ms,
                 "pairs_per_s_in_step": wl.B / (align_ms / 1e3),
+                "band_cells": cells, "band_cells_per_s": cells / (align_alone_ms / 1e3),
                 "note": "dtw_pairs_per_s: tt_align alone (one warp per pair), 200 calls; in "
                         "the step the alignment takes one CTA per SM beside the row pass"},
         "stage_ms": {"align": align_ms, "rowpass": row_ms, "decide": dec_ms,
@@ -465,6 +470,8 @@ def run_mine(args):
         line["e2e"] = e2e
     if reenc is not None:
         line["reencode"] = reenc
+    if verify is not None:
+        line["verify"] = verify
     if sharded is not None:
         line["sharded"] = sharded
     if cpu is not None:
@@ -499,6 +506,38 @@ def run_align_alone(tt, wl, inp, prm, dev, stream):
     kernel runs on one CTA per SM so that the row pass streams beside it."""
     call = tt.AlignCall(inp["batch"], inp["vd"], inp["vt"], prm, stream=stream)
     return _time_calls(call, stream, 200)
+
+
+def band_cells(wl, window: int) -> int:
+    """DTW cells inside the band over the whole batch: pairs (i, j), 1 <= i <= k,
+    1 <= j <= m, with |i - j| <= max(w, |k - m|) (every cell when w < 0)."""
+    import numpy as np
+    k = np.diff(np.asarray(wl.draft_off, dtype=np.int64))
+    m = np.diff(np.asarray(wl.target_off, dtype=np.int64))
+    total = 0
+    for kb, mb in zip(k.tolist(), m.tolist()):
+        if window < 0:
+            total += kb * mb
+            continue
+        W = max(window, abs(kb - mb))
+        i = np.arange(1, kb + 1)
+        total += int(np.maximum(0, np.minimum(mb, i + W) - np.maximum(1, i - W) + 1).sum())
+    return total
+
+
+def run_verify_alone(tt, wl, inp, prm, q_hat, dev, stream):
+    """tt_verify on its own (target row pass and decision, with the step's
+    q_hat), timed with CUDA events over repeated calls outside the step's timed
+    region: the metric's positions over the verification alone."""
+    batch, tl = inp["batch"], inp["target_logits"]
+    ws_v = tt.binding.workspace(batch, 0, tl.shape[1], dev, prm)
+    out = {}
+    ms = _time_calls(lambda: out.update(tt.tt_verify(batch, q_hat, tl, prm, ws=ws_v, out=out,
+                                                     stream=stream)), stream, 50)
+    tbytes = (wl.n_target + wl.B) * tl.shape[1] * tl.element_size()
+    return {"ms_per_call": ms, "positions_per_s": wl.n_draft / (ms / 1e3),
+            "target_bytes": tbytes, "target_gbs": tbytes / (ms / 1e3) / 1e9,
+            "note": "tt_verify alone on the step's q_hat, 50 calls"}
 
 
 def run_sharded(tt, wl, inp, prm, q_hat, dev, stream, S):

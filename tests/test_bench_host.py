@@ -1,8 +1,9 @@
 """Host logic of bench.py on CPU: the default arguments the run contract needs,
 the algorithmic bytes of a step (the roofline's numerator), the rule that a
 committed ncu summary feeds `traffic` only when it was taken on the current
-row-pass source (and, with filters, at the same top-k), and the reference
-arm's JSON line (the oracle on the host cores)."""
+row-pass source (and, with filters, at the same top-k), the reference
+arm's JSON line (the oracle on the host cores) and the count of DTW band
+cells behind the band-cells-per-second figure."""
 import json
 import os
 import subprocess
@@ -89,3 +90,20 @@ def test_reference_arm_prints_one_contract_line():
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}
+
+
+@pytest.mark.parametrize("window", [-1, 0, 1, 2, 8])
+def test_band_cells_match_a_count_of_the_band(window):
+    rng = np.random.default_rng(window + 5)
+    k = rng.integers(1, 30, size=40)
+    m = rng.integers(1, 30, size=40)
+    wl = SimpleNamespace(draft_off=np.concatenate([[0], np.cumsum(k)]),
+                         target_off=np.concatenate([[0], np.cumsum(m)]))
+    want = 0
+    for kb, mb in zip(k, m):
+        W = max(window, abs(int(kb) - int(mb)))
+        want += sum(1 for i in range(1, kb + 1) for j in range(1, mb + 1)
+                    if window < 0 or abs(i - j) <= W)
+    assert bench.band_cells(wl, window) == want
+    # the band always holds the diagonal corner to corner, at most every cell
+    assert int((np.minimum(k, m)).sum()) <= bench.band_cells(wl, window) <= int((k * m).sum())
