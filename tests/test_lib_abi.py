@@ -107,10 +107,20 @@ def test_host_validation_rejects_bad_arguments(lib):
     pq = binding.Params(full_q=True)._c(keep)
     assert lib.tt_step(P(b._c()), P(vd._c()), P(vd._c()), P(lg2), None, P(lg), P(pq),
                        ctypes.c_void_p(256), 1 << 30, P(out), None) == binding.TT_ERR_INVALID_ARG
-    # an empty batch is a no-op
+    # an empty batch is a no-op for every entry point (nothing is launched,
+    # no output or workspace is needed)
     e = tt.Batch.from_host([0], [], [0], [], device="cpu")
     assert lib.tt_align(P(e._c()), P(vd._c()), P(vd._c()), P(prm._c(keep)), None, None, None,
                         None, None, None) == binding.TT_OK
+    assert lib.tt_transfer(P(e._c()), None, P(lg), None, P(prm._c(keep)), None, 0, None, None,
+                           None) == binding.TT_OK
+    assert lib.tt_verify(P(e._c()), None, P(lg), None, None, P(prm._c(keep)), None, 0, None,
+                         None, None, None, None, None) == binding.TT_OK
+    assert lib.tt_step(P(e._c()), P(vd._c()), P(vd._c()), P(lg), None, P(lg), P(prm._c(keep)),
+                       None, 0, P(out), None) == binding.TT_OK
+    sh, _k = _shards([64, 64])
+    assert lib.tt_verify_sharded(P(e._c()), None, P(sh), P(prm._c(keep)), None, 0, None, None,
+                                 None, None, None, None, None) == binding.TT_OK
 
 
 def _shards(widths, col0=None):
