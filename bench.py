@@ -243,7 +243,17 @@ def default_steps(name: str) -> int:
             "dtw_4096x64": 1000, "b1024_g8_v201k_bf16": 1000}.get(name, 1000)
 
 
-def oracle_sample_rate(wl, budget_s: float, rank: int = 0):
+def step_kwargs(args) -> dict:
+    """The run's step parameters beyond the workload's own, for the oracle legs:
+    the temperature override and the sampling filters of both families."""
+    kw = {"top_k_draft": args.top_k, "top_k_target": args.top_k,
+          "top_p_draft": args.top_p, "top_p_target": args.top_p}
+    if args.temp is not None:
+        kw["temp_draft"] = kw["temp_target"] = args.temp
+    return kw
+
+
+def oracle_sample_rate(wl, budget_s: float, step_kw=None):
     """Times the oracle (as it stands) over requests of the workload, cycling
     through them until the CPU budget is spent; returns positions/s and a note."""
     import oracle
@@ -257,7 +267,7 @@ def oracle_sample_rate(wl, budget_s: float, rank: int = 0):
             subs[b] = wl.subset([b])
         sw = subs[b]
         t = time.perf_counter()
-        oracle.step(sw, request_base=b)
+        oracle.step(sw, request_base=b, **(step_kw or {}))
         elapsed += time.perf_counter() - t
         positions += int(sw.draft_off[-1])
         done_req += 1
@@ -276,8 +286,8 @@ def host_cores() -> int:
 def _oracle_job(job):
     """One worker process: the oracle, as it stands, over its list of requests
     (cycling) until `budget` seconds are spent (or once through when budget is
-    0); returns (positions, seconds, requests)."""
-    subs, budget = job
+    0), with the step parameters `kw`; returns (positions, seconds, requests)."""
+    subs, budget, kw = job
     import oracle
     oracle.build()
     positions, elapsed, done = 0, 0.0, 0
@@ -285,7 +295,7 @@ def _oracle_job(job):
     while (budget > 0 and elapsed < budget) or (budget <= 0 and i < len(subs)):
         b, sw = subs[i % len(subs)]
         t = time.perf_counter()
-        oracle.step(sw, request_base=b)
+        oracle.step(sw, request_base=b, **kw)
         elapsed += time.perf_counter() - t
         positions += int(sw.draft_off[-1])
         done += 1
@@ -299,7 +309,7 @@ def oracle_pool(n: int):
     return multiprocessing.get_context("spawn").Pool(n)
 
 
-def oracle_all_cores_rate(wl, budget_s: float, per_worker: int = 2):
+def oracle_all_cores_rate(wl, budget_s: float, per_worker: int = 2, step_kw=None):
     """The oracle on every host core: worker w cycles over its own `per_worker`
     requests of the batch for budget_s seconds; the rate is the sum of the
     workers' rates (each timed inside its process, without the pool's I/O)."""
@@ -307,7 +317,7 @@ def oracle_all_cores_rate(wl, budget_s: float, per_worker: int = 2):
     jobs = []
     for w in range(n):
         idx = [(w * per_worker + i) % wl.B for i in range(per_worker)]
-        jobs.append(([(b, wl.subset([b])) for b in idx], budget_s))
+        jobs.append(([(b, wl.subset([b])) for b in idx], budget_s, step_kw or {}))
     with oracle_pool(n) as pool:
         res = pool.map(_oracle_job, jobs, chunksize=1)
     rate = sum(p / e for p, e, _ in res if e > 0)
@@ -424,9 +434,10 @@ def run_mine(args):
 
     cpu = cpu_all = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        rate, sample, nreq, el = oracle_sample_rate(wl, args.cpu_seconds)
+        rate, sample, nreq, el = oracle_sample_rate(wl, args.cpu_seconds, step_kwargs(args))
         cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
-        rate, sample, n = oracle_all_cores_rate(wl, min(args.cpu_seconds, 8.0))
+        rate, sample, n = oracle_all_cores_rate(wl, min(args.cpu_seconds, 8.0),
+                                                step_kw=step_kwargs(args))
         cpu_all = {"value": rate, "unit": UNIT, "cores": n, "kind": "oracle", "sample": sample}
 
     clk = clocks.summary(h0, h1)
@@ -708,17 +719,24 @@ def run_reference(args):
     name = args.workload
     K = args.steps if args.steps is not None else 5
     Wm = max(3, args.warmup)
-    wl = W.make_workload(name, B=args.batch, seed=0, device="cpu")
+    import torch
+    # the same draws as the GPU arm's (its generator runs on the device); the
+    # oracle reads each request's rows copied to the host
+    gen_dev = "cuda" if torch.cuda.is_available() else "cpu"
+    wl = W.make_workload(name, B=args.batch, seed=0, device=gen_dev)
     per_worker = {"b1_g4_v32k": 1, "b64_g8_v152k": 2, "b256_g16_v152k_bf16": 1,
                   "dtw_4096x64": 8, "b1024_g8_v201k_bf16": 1}.get(name, 1)
     n = host_cores()
+    kw = step_kwargs(args)
+    spec = wl.spec
+    temps = [kw.get("temp_draft", spec.temp_draft), kw.get("temp_target", spec.temp_target)]
     # step s: worker w takes requests ((s * n + w) * per_worker + i) mod B; a
     # step's time is the slowest worker's oracle time (measured in the worker)
     def step_jobs(s):
         jobs = []
         for w in range(n):
             idx = [((s * n + w) * per_worker + i) % wl.B for i in range(per_worker)]
-            jobs.append(([(b, wl.subset([b])) for b in idx], 0.0))
+            jobs.append(([(b, wl.subset([b])) for b in idx], 0.0, kw))
         return jobs
     sec, pos = 0.0, 0
     with oracle_pool(n) as pool:
@@ -731,12 +749,22 @@ def run_reference(args):
     value = pos / sec
     per_step = n * per_worker
     sample = ("%d requests of the %s batch per step, %d per oracle process, one process per "
-              "host core (%d), fp64; a step lasts as long as its slowest process"
-              % (per_step, name, per_worker, n))
+              "host core (%d), fp64; a step lasts as long as its slowest process; inputs "
+              "drawn on %s" % (per_step, name, per_worker, n, gen_dev))
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
             "n_gpus": ws, "steps": K, "warmup": Wm, "ms_per_step": sec * 1e3 / K,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": name, "requests_per_step": per_step},
+            "data": "synthetic",
+            "config": {"workload": name, "batch_per_gpu": wl.B, "gamma": spec.k,
+                       "V_d": spec.V_d, "V_t": spec.V_t,
+                       "logits_cols": [int(wl.draft_logits.shape[1]),
+                                       int(wl.target_logits.shape[1])],
+                       "target_tokens_per_gpu": wl.n_target, "window": spec.window,
+                       "temperature": temps,
+                       "filters": ({"top_k": args.top_k, "top_p": args.top_p}
+                                   if args.top_k > 0 else None),
+                       "parallelism": "oracle processes on the host cores",
+                       "requests_per_step": per_step},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": n, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,

@@ -86,6 +86,12 @@ def test_reference_arm_prints_one_contract_line():
     assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == bench.UNIT
     assert d["value"] > 0 and d["steps"] == 2 and d["warmup"] >= 3 and d["n_gpus"] == 1
     assert d["higher_is_better"] is True and d["config"]["workload"] == "b1_g4_v32k"
+    # the workload keys of the GPU arm's config (its measured keys aside)
+    for key in ("batch_per_gpu", "gamma", "V_d", "V_t", "logits_cols", "target_tokens_per_gpu",
+                "window", "temperature", "filters", "parallelism"):
+        assert key in d["config"], key
+    assert d["config"]["batch_per_gpu"] == 1 and d["config"]["gamma"] == 4
+    assert d["config"]["filters"] is None
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0,
@@ -107,3 +113,28 @@ def test_band_cells_match_a_count_of_the_band(window):
     assert bench.band_cells(wl, window) == want
     # the band always holds the diagonal corner to corner, at most every cell
     assert int((np.minimum(k, m)).sum()) <= bench.band_cells(wl, window) <= int((k * m).sum())
+
+
+def test_oracle_legs_run_the_step_parameters_of_the_run(monkeypatch):
+    """The CPU legs time the oracle on the run's temperature and filters."""
+    import oracle
+    from paper_2510_15545_gb300 import workload as W
+    seen = []
+    real = oracle.step
+
+    def spy(sw, **kw):
+        seen.append(kw)
+        return real(sw, **kw)
+    monkeypatch.setattr(oracle, "step", spy)
+    wl = W.make_workload("b1_g4_v32k", seed=0)
+    args = bench.parse_args(["--temp", "0.6", "--top-k", "20", "--top-p", "0.95"])
+    rate, sample, n, el = bench.oracle_sample_rate(wl, 0.05, bench.step_kwargs(args))
+    assert rate > 0 and n >= 1
+    assert seen and all(k["temp_draft"] == 0.6 and k["temp_target"] == 0.6 and
+                        k["top_k_draft"] == 20 and k["top_p_target"] == 0.95 for k in seen)
+    plain = bench.step_kwargs(bench.parse_args([]))
+    assert plain == {"top_k_draft": 0, "top_k_target": 0, "top_p_draft": 1.0,
+                     "top_p_target": 1.0}
+    # a worker job carries the same parameters
+    pos, sec, done = bench._oracle_job(([(0, wl.subset([0]))], 0.0, bench.step_kwargs(args)))
+    assert done == 1 and pos == 4 and seen[-1]["top_k_target"] == 20
