@@ -181,6 +181,56 @@ def test_bonus_row_when_all_accepted():
     assert stats.chisquare(np.bincount(out["next_token"], minlength=V), want).pvalue > 1e-4
 
 
+def _np_uniform(seed, pos, stream, req):
+    """u from numpy's own Philox4x64-10 at counter (pos, stream, req, 0), key
+    (seed, 0): the top 24 bits of the block's first word times 2^-24."""
+    c = (pos + (stream << 64) + (req << 128) - 1) & ((1 << 256) - 1)
+    words = np.array([(c >> (64 * i)) & MASK64 for i in range(4)], dtype=np.uint64)
+    g = np.random.Philox(key=np.array([seed, 0], dtype=np.uint64), counter=words)
+    return (int(g.random_raw(1)[0]) >> 40) / 2.0**24
+
+
+def test_each_decision_uses_its_own_uniform_and_the_inverse_cdf():
+    """Every accept decision and every next token recomputed by hand from the
+    definitions: u_j from numpy's Philox at (j, stream 0, request_base + b),
+    accept while u_j < p_j / q_j, then the residual (p with t_a's mass lowered
+    by q_hat, or the bonus row) sampled at u' from (a, stream 1, ...) as the
+    smallest column whose running mass exceeds u' Z."""
+    rng = np.random.default_rng(21)
+    B, V, seed, base = 300, 12, 77, 1000
+    ms = rng.integers(1, 6, size=B)
+    t_off = np.concatenate([[0], np.cumsum(ms)]).astype(np.int32)
+    nt = int(t_off[-1])
+    cols = rng.integers(0, V, size=nt).astype(np.int32)
+    z = (rng.standard_normal((nt + B, V)) * 1.2).astype(np.float32)
+    qh = rng.uniform(0.02, 0.6, size=nt)
+    out = oracle.verify(t_off, cols, qh, z, seed=seed, request_base=base)
+    n_acc = n_rej = 0
+    for b in range(B):
+        if out["boundary"][b]:
+            continue
+        t0, m, row0 = int(t_off[b]), int(ms[b]), int(t_off[b]) + b
+        P = special.softmax(z[row0:row0 + m + 1].astype(np.float64), axis=1)
+        a = m
+        for j in range(m):
+            u = _np_uniform(seed, j, 0, base + b)
+            if not u < P[j, cols[t0 + j]] / qh[t0 + j]:
+                a = j
+                break
+        assert out["accepted"][b] == a, b
+        r = P[a].copy()
+        if a < m:
+            t = cols[t0 + a]
+            r[t] = max(0.0, r[t] - qh[t0 + a])
+            n_rej += 1
+        else:
+            n_acc += 1
+        u2 = _np_uniform(seed, a, 1, base + b)
+        x = int(np.argmax(np.cumsum(r) > u2 * r.sum()))
+        assert out["next_token"][b] == x, b
+    assert n_acc > 20 and n_rej > 100  # both branches are exercised
+
+
 def test_rejected_token_is_never_resampled():
     V, N = 5, 2000
     zp = _rows([0.3, 0.2, 0.2, 0.2, 0.1])
