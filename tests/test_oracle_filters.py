@@ -110,3 +110,76 @@ def test_filtered_speculative_sampling_emits_the_filtered_target(k, p):
     assert counts[~keep].sum() == 0
     assert stats.chisquare(counts[keep], pf[keep] * N).pvalue > 1e-4
     assert np.allclose(out["p_hat"][:5], pf[t[:5]])
+
+
+def _np_uniform(seed, pos, stream, req):
+    # numpy's own Philox4x64-10 at counter (pos, stream, req, 0), key (seed, 0)
+    mask = (1 << 64) - 1
+    c = (pos + (stream << 64) + (req << 128) - 1) & ((1 << 256) - 1)
+    words = np.array([(c >> (64 * i)) & mask for i in range(4)], dtype=np.uint64)
+    g = np.random.Philox(key=np.array([seed, 0], dtype=np.uint64), counter=words)
+    return (int(g.random_raw(1)[0]) >> 40) / 2.0**24
+
+
+def _kept_by_hand(z, T, k, p):
+    """Temperature, the k largest logits (ties: smaller column), softmax over
+    them, the smallest prefix whose mass reaches p, renormalised (R22-R24)."""
+    s = z.astype(np.float64) / T
+    order = np.argsort(-z, kind="stable")[:k]
+    w = np.exp(s[order] - s[order].max())
+    w /= w.sum()
+    n = 0
+    before = 0.0
+    while n < len(order) and before < p:
+        before += w[n]
+        n += 1
+    out = np.zeros(len(z))
+    out[order[:n]] = w[:n] / w[:n].sum()
+    return out
+
+
+def test_filtered_decisions_recomputed_by_hand():
+    """Every accept decision and next token of a filtered verification: p_f
+    from the kept set built by hand, accept while u_j < p_f(t_j) / q_j, the
+    residual (p_f with t_a's mass lowered by q_hat, zero outside the kept set,
+    or the bonus row's p_f) sampled in column order (R27)."""
+    rng = np.random.default_rng(33)
+    B, V, seed, T, k, p = 300, 40, 5, 0.7, 6, 0.9
+    ms = rng.integers(1, 5, size=B)
+    t_off = np.concatenate([[0], np.cumsum(ms)]).astype(np.int32)
+    nt = int(t_off[-1])
+    z = (rng.standard_normal((nt + B, V)) * 1.5).astype(np.float32)
+    # scored columns: mostly inside the row's top 3, some anywhere
+    cols = np.array([np.argsort(-z[i + b])[rng.integers(0, 3)] if rng.random() < 0.8
+                     else rng.integers(0, V) for b in range(B)
+                     for i in range(t_off[b], t_off[b + 1])], dtype=np.int32)
+    qh = rng.uniform(0.05, 0.9, size=nt)
+    out = oracle.verify(t_off, cols, qh, z, temp_target=T, seed=seed, top_k_target=k,
+                        top_p_target=p)
+    checked = rejected = 0
+    for b in range(B):
+        if out["boundary"][b]:
+            continue
+        t0, m, row0 = int(t_off[b]), int(ms[b]), int(t_off[b]) + b
+        PF = [_kept_by_hand(z[row0 + j], T, k, p) for j in range(m + 1)]
+        a = m
+        for j in range(m):
+            u = _np_uniform(seed, j, 0, b)
+            if not u < PF[j][cols[t0 + j]] / qh[t0 + j]:
+                a = j
+                break
+        assert out["accepted"][b] == a, b
+        r = PF[a].copy()
+        if a < m:
+            t = cols[t0 + a]
+            r[t] = max(0.0, r[t] - qh[t0 + a])
+            rejected += 1
+            if not r.sum() > 0:
+                r = PF[a].copy()
+        u2 = _np_uniform(seed, a, 1, b)
+        x = int(np.argmax(np.cumsum(r) > u2 * r.sum()))
+        assert r[x] > 0 and out["next_token"][b] == x, b
+        assert np.allclose(out["p_hat"][t0:t0 + m], [PF[j][cols[t0 + j]] for j in range(m)],
+                           atol=1e-12)
+        checked += 1
+    assert checked > 250 and rejected > 100
