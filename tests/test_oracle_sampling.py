@@ -231,6 +231,48 @@ def test_each_decision_uses_its_own_uniform_and_the_inverse_cdf():
     assert n_acc > 20 and n_rej > 100  # both branches are exercised
 
 
+def test_full_q_decisions_recomputed_by_hand():
+    """Full-q mode (one vocabulary, Alg. 4 as printed): each rejection's next
+    token comes from max(0, p_a - q) against the whole mapped draft row at T_d
+    (the row itself when that has no mass), each bonus token from row m."""
+    rng = np.random.default_rng(22)
+    B, V, k, seed, Td, Tt = 250, 10, 4, 31, 0.8, 1.1
+    ms = rng.integers(1, 6, size=B)
+    t_off = np.concatenate([[0], np.cumsum(ms)]).astype(np.int32)
+    d_off = np.arange(0, B * k + 1, k, dtype=np.int32)
+    nt = int(t_off[-1])
+    zt = (rng.standard_normal((nt + B, V)) * 1.3).astype(np.float32)
+    zd = (rng.standard_normal((B * k, V)) * 1.3).astype(np.float32)
+    mp = np.concatenate([np.sort(rng.integers(0, k, size=m)) for m in ms]).astype(np.int32)
+    cols = rng.integers(0, V, size=nt).astype(np.int32)
+    Q = special.softmax(zd.astype(np.float64) / Td, axis=1)
+    qh = np.array([Q[d_off[b] + mp[j], cols[j]] for b in range(B)
+                   for j in range(t_off[b], t_off[b + 1])])
+    out = oracle.verify(t_off, cols, qh, zt, temp_target=Tt, seed=seed, full_q=True,
+                        draft_off=d_off, mp=mp, draft_logits=zd, temp_draft=Td)
+    rejected = 0
+    for b in range(B):
+        if out["boundary"][b]:
+            continue
+        t0, m, row0 = int(t_off[b]), int(ms[b]), int(t_off[b]) + b
+        P = special.softmax(zt[row0:row0 + m + 1].astype(np.float64) / Tt, axis=1)
+        a = m
+        for j in range(m):
+            if not _np_uniform(seed, j, 0, b) < P[j, cols[t0 + j]] / qh[t0 + j]:
+                a = j
+                break
+        assert out["accepted"][b] == a, b
+        r = P[a].copy()
+        if a < m:
+            r = np.maximum(0.0, P[a] - Q[d_off[b] + mp[t0 + a]])
+            if not r.sum() > 0:
+                r = P[a].copy()
+            rejected += 1
+        u2 = _np_uniform(seed, a, 1, b)
+        assert out["next_token"][b] == int(np.argmax(np.cumsum(r) > u2 * r.sum())), b
+    assert rejected > 100
+
+
 def test_rejected_token_is_never_resampled():
     V, N = 5, 2000
     zp = _rows([0.3, 0.2, 0.2, 0.2, 0.1])
