@@ -73,6 +73,13 @@ def lib():
         L.tto_verify2.argtypes = [i32, P, P, P, P, i32, i64, i32, f64, P, P, P, i32, i64, i32,
                                   f64, i32, u64, u64, i32, f64, i32, f64, P, P, P, P, P, P]
         L.tto_verify2.restype = None
+        L.tto_transfer3.argtypes = [i32, P, P, P, P, P, i32, i64, i32, P, f64, i32, f64, P, P, P,
+                                    P]
+        L.tto_transfer3.restype = None
+        L.tto_verify3.argtypes = [i32, P, P, P, P, i32, i64, i32, f64, P, P, P, i32, i64, i32,
+                                  f64, i32, u64, u64, i32, f64, i32, f64, P, P, P, P, P, P, P, P,
+                                  P]
+        L.tto_verify3.restype = None
         L.tto_encode.argtypes = [i32, P, P, P, P, i32, P, P, i32, i32, i32, i32, P, P, P]
         L.tto_encode.restype = None
         L.tto_consistency.argtypes = [i32, P, P, P, P, P, P, i32, P, P, i32, i32, i32, P]
@@ -196,10 +203,12 @@ def transfer(draft_off, draft_cols, target_off, mp, draft_logits, temp_draft: fl
     else:
         buf, dt, stride, V = None, 0, 0, 0
     bnd = np.zeros(max(B, 1), np.int32)
-    lib().tto_transfer2(B, _p(draft_off), _p(draft_cols), _p(target_off), _p(mp), _p(buf), dt,
+    nd = max(int(draft_off[-1]), 0)
+    drow = np.zeros(max(nd, 1), np.int32)
+    lib().tto_transfer3(B, _p(draft_off), _p(draft_cols), _p(target_off), _p(mp), _p(buf), dt,
                         stride, V, _p(probs), float(temp_draft), int(top_k), float(top_p), _p(q),
-                        _p(status), _p(bnd))
-    return dict(q_hat=q[:nt], status=status, boundary=bnd[:B])
+                        _p(status), _p(bnd), _p(drow))
+    return dict(q_hat=q[:nt], status=status, boundary=bnd[:B], drow_bnd=drow[:nd])
 
 
 def verify(target_off, target_cols, q_hat, target_logits, *, temp_target: float = 1.0,
@@ -222,14 +231,18 @@ def verify(target_off, target_cols, q_hat, target_logits, *, temp_target: float 
     lse = np.zeros(nt + B, np.float64)
     status = np.zeros(B, np.int32)
     bnd = np.zeros(B, np.int32)
-    lib().tto_verify2(B, _p(target_off), _p(target_cols), _p(q_hat), _p(tbuf), tdt, tstride, Vt,
+    row_bnd = np.zeros(max(nt + B, 1), np.int32)
+    tok_lo = np.full(max(B, 1), -1, np.int32)
+    tok_hi = np.full(max(B, 1), -1, np.int32)
+    lib().tto_verify3(B, _p(target_off), _p(target_cols), _p(q_hat), _p(tbuf), tdt, tstride, Vt,
                       float(temp_target), _p(draft_off) if full_q else None,
                       _p(mp) if full_q else None, _p(dbuf), ddt, dstride, Vd, float(temp_draft),
                       int(bool(full_q)), int(seed), int(request_base), int(top_k_target),
                       float(top_p_target), int(top_k_draft), float(top_p_draft), _p(acc),
-                      _p(nxt), _p(p_hat), _p(lse), _p(status), _p(bnd))
+                      _p(nxt), _p(p_hat), _p(lse), _p(status), _p(bnd), _p(row_bnd), _p(tok_lo),
+                      _p(tok_hi))
     return dict(accepted=acc, next_token=nxt, p_hat=p_hat[:nt], lse=lse, status=status,
-                boundary=bnd)
+                boundary=bnd, row_bnd=row_bnd[:nt + B], tok_lo=tok_lo[:B], tok_hi=tok_hi[:B])
 
 
 def step(wl, *, window: Optional[int] = None, temp_draft: Optional[float] = None,
@@ -256,7 +269,8 @@ def step(wl, *, window: Optional[int] = None, temp_draft: Optional[float] = None
     out = dict(al)
     out.update(q_hat=tr["q_hat"], p_hat=ve["p_hat"], lse=ve["lse"], accepted=ve["accepted"],
                next_token=ve["next_token"], boundary=ve["boundary"] | tr["boundary"],
-               status=status)
+               status=status, row_bnd=ve["row_bnd"], drow_bnd=tr["drow_bnd"],
+               tok_lo=ve["tok_lo"], tok_hi=ve["tok_hi"])
     bad = status != 0
     out["accepted"] = np.where(bad, 0, out["accepted"]).astype(np.int32)
     out["next_token"] = np.where(bad, -1, out["next_token"]).astype(np.int32)

@@ -319,11 +319,15 @@ void tto_align(int32_t B, const int32_t* draft_off, const int32_t* draft_ids,
 
 /* ---------------------------------------------------------------- transfer */
 
-void tto_transfer2(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
-                   const int32_t* target_off, const int32_t* map,
-                   const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
-                   const float* draft_probs, double T_d, int32_t top_k, double top_p,
-                   double* q_hat, int32_t* status, int32_t* boundary) {
+/* The transfer with the draft rows' filters; drow_bnd (may be NULL) gets bit 4
+ * for each draft row whose top-p cut is ambiguous (the request-wide bit of
+ * `boundary` is the OR of its rows'). */
+static void transfer_impl(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                          const int32_t* target_off, const int32_t* map,
+                          const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                          const float* draft_probs, double T_d, int32_t top_k, double top_p,
+                          double* q_hat, int32_t* status, int32_t* boundary,
+                          int32_t* drow_bnd) {
   const int filtered = top_k > 0 || (top_p > 0.0 && top_p < 1.0);
   double* qf = filtered ? (double*)malloc(sizeof(double) * (size_t)(V > 0 ? V : 1)) : NULL;
   for (int32_t b = 0; b < B; ++b) {
@@ -352,7 +356,10 @@ void tto_transfer2(int32_t B, const int32_t* draft_off, const int32_t* draft_col
       } else if (filtered) {
         const void* row = row_ptr(draft_logits, dtype, row_stride, r);
         if (r != have) {
-          tto_filtered_probs(row, dtype, V, T_d, top_k, top_p, qf, boundary ? &boundary[b] : NULL);
+          int32_t rb = 0;
+          tto_filtered_probs(row, dtype, V, T_d, top_k, top_p, qf, &rb);
+          if (boundary) boundary[b] |= rb;
+          if (drow_bnd) drow_bnd[r] |= rb;
           have = r;
         }
         q_hat[t0 + j] = qf[draft_cols[r]];
@@ -366,6 +373,24 @@ void tto_transfer2(int32_t B, const int32_t* draft_off, const int32_t* draft_col
   free(qf);
 }
 
+void tto_transfer2(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                   const int32_t* target_off, const int32_t* map,
+                   const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                   const float* draft_probs, double T_d, int32_t top_k, double top_p,
+                   double* q_hat, int32_t* status, int32_t* boundary) {
+  transfer_impl(B, draft_off, draft_cols, target_off, map, draft_logits, dtype, row_stride, V,
+                draft_probs, T_d, top_k, top_p, q_hat, status, boundary, NULL);
+}
+
+void tto_transfer3(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                   const int32_t* target_off, const int32_t* map,
+                   const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                   const float* draft_probs, double T_d, int32_t top_k, double top_p,
+                   double* q_hat, int32_t* status, int32_t* boundary, int32_t* drow_bnd) {
+  transfer_impl(B, draft_off, draft_cols, target_off, map, draft_logits, dtype, row_stride, V,
+                draft_probs, T_d, top_k, top_p, q_hat, status, boundary, drow_bnd);
+}
+
 void tto_transfer(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
                   const int32_t* target_off, const int32_t* map,
                   const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
@@ -376,15 +401,24 @@ void tto_transfer(int32_t B, const int32_t* draft_off, const int32_t* draft_cols
 
 /* ------------------------------------------------------------------ verify */
 
-void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_cols,
-                 const double* q_hat, const void* target_logits, int32_t dtype_t,
-                 int64_t stride_t, int32_t V_t, double T_t,
-                 const int32_t* draft_off, const int32_t* map, const void* draft_logits,
-                 int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
-                 int32_t full_q, uint64_t seed, uint64_t request_base,
-                 int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
-                 int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
-                 int32_t* status, int32_t* boundary) {
+/* The verification; besides the request-wide boundary bits it can report
+ * where each one lies (all three may be NULL): row_bnd[r] for every target row
+ * r (indexed as lse) gets bit 1 when the accept decision of the position that
+ * row scores lay within 1e-6 of its threshold, bit 4 when the row's top-p cut
+ * is ambiguous, bit 8 (full-q) when the kept set of the draft row that the
+ * residual of this row subtracts is ambiguous; tok_lo[b] / tok_hi[b] are the
+ * first and last column of the drawn row whose running mass lies within
+ * 1e-6 Z of u' Z (-1 when none). None of these changes any result. */
+static void verify_impl(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                        const double* q_hat, const void* target_logits, int32_t dtype_t,
+                        int64_t stride_t, int32_t V_t, double T_t,
+                        const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                        int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                        int32_t full_q, uint64_t seed, uint64_t request_base,
+                        int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
+                        int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
+                        int32_t* status, int32_t* boundary, int32_t* row_bnd,
+                        int32_t* tok_lo, int32_t* tok_hi) {
   const int filt_t = top_k_t > 0 || (top_p_t > 0.0 && top_p_t < 1.0);
   const int filt_d = top_k_d > 0 || (top_p_d > 0.0 && top_p_d < 1.0);
   double* pf = filt_t ? (double*)malloc(sizeof(double) * (size_t)V_t) : NULL;
@@ -395,6 +429,8 @@ void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_col
     accepted[b] = 0;
     next_token[b] = -1;
     boundary[b] = 0;
+    if (tok_lo) tok_lo[b] = -1;
+    if (tok_hi) tok_hi[b] = -1;
     if (!offsets_ok(target_off, b)) {
       status[b] = ST_BAD_OFFSETS;
       continue;
@@ -425,8 +461,10 @@ void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_col
     for (int32_t j = 0; j <= m; ++j) {
       const void* row = row_ptr(target_logits, dtype_t, stride_t, row0 + j);
       if (filt_t) {
-        double l = tto_filtered_probs(row, dtype_t, V_t, T_t, top_k_t, top_p_t, pf,
-                                      &boundary[b]);
+        int32_t rb = 0;
+        double l = tto_filtered_probs(row, dtype_t, V_t, T_t, top_k_t, top_p_t, pf, &rb);
+        boundary[b] |= rb;
+        if (row_bnd) row_bnd[row0 + j] |= rb;
         if (lse) lse[row0 + j] = l;
         if (j < m) p_hat[t0 + j] = pf[target_cols[t0 + j]];
       } else {
@@ -443,7 +481,10 @@ void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_col
       double ph = p_hat[t0 + j], qh = q_hat[t0 + j];
       double ratio = qh > 0.0 ? ph / qh : (ph > 0.0 ? INFINITY : 0.0);
       double acc = ratio < 1.0 ? ratio : 1.0;
-      if (fabs(u - acc) < BOUNDARY_EPS) boundary[b] |= 1;
+      if (fabs(u - acc) < BOUNDARY_EPS) {
+        boundary[b] |= 1;
+        if (row_bnd) row_bnd[row0 + j] |= 1;
+      }
       if (u < acc) ++a;
       else break;
     }
@@ -457,8 +498,14 @@ void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_col
       if (full_q) {
         const void* qrow = row_ptr(draft_logits, dtype_d, stride_d,
                                    (int64_t)draft_off[b] + map[t0 + a]);
-        if (filt_d) tto_filtered_probs(qrow, dtype_d, V_d, T_d, top_k_d, top_p_d, q, &boundary[b]);
-        else tto_softmax(qrow, dtype_d, V_d, T_d, q);
+        if (filt_d) {
+          int32_t rb = 0;
+          tto_filtered_probs(qrow, dtype_d, V_d, T_d, top_k_d, top_p_d, q, &rb);
+          boundary[b] |= rb;
+          if (row_bnd && rb) row_bnd[row0 + a] |= 8;
+        } else {
+          tto_softmax(qrow, dtype_d, V_d, T_d, q);
+        }
         for (int32_t x = 0; x < V_t; ++x) r[x] = p[x] > q[x] ? p[x] - q[x] : 0.0;
       } else {
         int32_t t = target_cols[t0 + a];
@@ -482,7 +529,11 @@ void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_col
     for (int32_t x = 0; x < V_t; ++x) {
       cum += r[x];
       if (r[x] > 0.0) last_pos = x;
-      if (fabs(theta - cum) < BOUNDARY_EPS * Z) boundary[b] |= 2;
+      if (fabs(theta - cum) < BOUNDARY_EPS * Z) {
+        boundary[b] |= 2;
+        if (tok_lo && tok_lo[b] < 0) tok_lo[b] = x;
+        if (tok_hi) tok_hi[b] = x;
+      }
       if (pick < 0 && cum > theta) pick = x;
     }
     next_token[b] = pick >= 0 ? pick : last_pos;
@@ -491,6 +542,37 @@ void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_col
   free(q);
   free(r);
   free(pf);
+}
+
+void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                 const double* q_hat, const void* target_logits, int32_t dtype_t,
+                 int64_t stride_t, int32_t V_t, double T_t,
+                 const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                 int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                 int32_t full_q, uint64_t seed, uint64_t request_base,
+                 int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
+                 int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
+                 int32_t* status, int32_t* boundary) {
+  verify_impl(B, target_off, target_cols, q_hat, target_logits, dtype_t, stride_t, V_t, T_t,
+              draft_off, map, draft_logits, dtype_d, stride_d, V_d, T_d, full_q, seed,
+              request_base, top_k_t, top_p_t, top_k_d, top_p_d, accepted, next_token, p_hat,
+              lse, status, boundary, NULL, NULL, NULL);
+}
+
+void tto_verify3(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                 const double* q_hat, const void* target_logits, int32_t dtype_t,
+                 int64_t stride_t, int32_t V_t, double T_t,
+                 const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                 int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                 int32_t full_q, uint64_t seed, uint64_t request_base,
+                 int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
+                 int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
+                 int32_t* status, int32_t* boundary, int32_t* row_bnd, int32_t* tok_lo,
+                 int32_t* tok_hi) {
+  verify_impl(B, target_off, target_cols, q_hat, target_logits, dtype_t, stride_t, V_t, T_t,
+              draft_off, map, draft_logits, dtype_d, stride_d, V_d, T_d, full_q, seed,
+              request_base, top_k_t, top_p_t, top_k_d, top_p_d, accepted, next_token, p_hat,
+              lse, status, boundary, row_bnd, tok_lo, tok_hi);
 }
 
 void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols,

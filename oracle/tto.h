@@ -106,6 +106,35 @@ void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_col
                  int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
                  int32_t* status, int32_t* boundary);
 
+/* tto_transfer2 that also says which draft rows have an ambiguous top-p cut:
+ * drow_bnd[r] (n_draft entries, OR-ed into: the caller clears it) gets bit 4
+ * for each such row r. Results are those of tto_transfer2. */
+void tto_transfer3(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                   const int32_t* target_off, const int32_t* map,
+                   const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                   const float* draft_probs, double T_d, int32_t top_k, double top_p,
+                   double* q_hat, int32_t* status, int32_t* boundary, int32_t* drow_bnd);
+
+/* tto_verify2 that also says where each boundary case lies, so that a
+ * comparison can excuse a difference only at the decision it concerns.
+ * row_bnd (n_target + B entries, indexed as lse, OR-ed into: the caller clears
+ * it): bit 1 = the accept decision of the position this row scores lay within
+ * 1e-6 of min(1, p/q); bit 4 = this row's top-p cut is ambiguous; bit 8 =
+ * full-q, the kept set of the draft row the residual of this row subtracts is
+ * ambiguous. tok_lo[b] / tok_hi[b]: first and last column of the drawn row
+ * whose running mass lies within 1e-6 Z of u' Z, -1 when none. Results are
+ * those of tto_verify2. */
+void tto_verify3(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                 const double* q_hat, const void* target_logits, int32_t dtype_t,
+                 int64_t stride_t, int32_t V_t, double T_t,
+                 const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                 int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                 int32_t full_q, uint64_t seed, uint64_t request_base,
+                 int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
+                 int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
+                 int32_t* status, int32_t* boundary, int32_t* row_bnd, int32_t* tok_lo,
+                 int32_t* tok_hi);
+
 /* ------------------------------------------------------------ re-encoding */
 
 /* Re-encoding (§4.2; App. A.1, Lemma 1): T_b = encode_t(decode_d(D_b)).

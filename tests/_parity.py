@@ -1,9 +1,10 @@
 """Comparison of the CUDA path (through the C ABI) with the CPU oracle on the
 same seeded inputs. Tolerances follow the method's contract: alignment paths,
-costs, maps, statuses and accepted lengths bit-exact; probabilities and
-log-normalisers within 1e-5 absolute (fp32 accumulation); sampled tokens equal
-except where the oracle's uniform lay within 1e-6 of a decision boundary (those
-cases are counted, never hidden)."""
+costs, maps, statuses and accepted lengths bit-exact; probabilities within
+1e-5 absolute and 1e-4 relative, log-normalisers within 1e-5 absolute (fp32
+accumulation); sampled tokens equal except at the one decision where the
+oracle's uniform lay within 1e-6 of its boundary (those cases are counted,
+never hidden)."""
 from __future__ import annotations
 
 import numpy as np
@@ -11,9 +12,10 @@ import torch
 
 import oracle
 import paper_2510_15545_gb300 as tt
+from oracle.compare import compare_step
 from paper_2510_15545_gb300 import workload as W
 
-TOL = 1e-5
+TOL = 1e-5  # absolute bound on probabilities
 
 
 def to_np(out: dict) -> dict:
@@ -55,48 +57,13 @@ def sub_workload(wl, idx) -> W.Workload:
 
 
 def compare(wl, g: dict, o: dict, req_index=None, check_align=True, check_q=True) -> dict:
-    """Asserts parity of one step; returns counts of boundary cases.
-    ``req_index[b]`` maps the oracle's request b to the GPU's (sampled runs)."""
-    B = len(o["status"])
-    gi = np.arange(B) if req_index is None else np.asarray(req_index)
-    g_off_t = g.get("_target_off", wl.target_off)
-    g_off_d = g.get("_draft_off", wl.draft_off)
-    assert np.array_equal(g["status"][gi], o["status"]), (g["status"][gi], o["status"])
-    n_acc_b = n_tok_b = n_filt_b = 0
-    for b in range(B):
-        if o["status"][b] != 0:
-            assert g["accepted"][gi[b]] == 0 and g["next_token"][gi[b]] == -1
-            continue
-        gb = gi[b]
-        ot0, ot1 = int(wl.target_off[b]), int(wl.target_off[b + 1])
-        gt0, gt1 = int(g_off_t[gb]), int(g_off_t[gb + 1])
-        if check_align and "path_len" in g:
-            L = int(o["path_len"][b])
-            assert int(g["path_len"][gb]) == L, b
-            assert int(g["cost"][gb]) == int(o["cost"][b]), b
-            op = int(wl.draft_off[b]) + ot0
-            gp = int(g_off_d[gb]) + gt0
-            assert np.array_equal(g["path"][2 * gp:2 * (gp + L)], o["path"][op:op + L].ravel()), b
-            assert np.array_equal(g["map"][gt0:gt1], o["map"][ot0:ot1]), b
-        if int(o["boundary"][b]) & 4:
-            # a top-p cut within 1e-6 of the mass before some token: the kept
-            # sets may differ, so nothing downstream is compared
-            n_filt_b += 1
-            continue
-        if check_q and "q_hat" in g:
-            assert np.max(np.abs(g["q_hat"][gt0:gt1] - o["q_hat"][ot0:ot1]), initial=0) <= TOL, b
-        assert np.max(np.abs(g["p_hat"][gt0:gt1] - o["p_hat"][ot0:ot1]), initial=0) <= TOL, b
-        if "lse" in g:
-            gl = g["lse"][gt0 + gb:gt1 + gb + 1]
-            ol = o["lse"][ot0 + b:ot1 + b + 1]
-            assert np.max(np.abs(gl - ol)) <= TOL * max(1.0, float(np.max(np.abs(ol)))), b
-        bnd = int(o["boundary"][b])
-        if g["accepted"][gb] != o["accepted"][b]:
-            assert bnd & 1, (b, g["accepted"][gb], o["accepted"][b])
-            n_acc_b += 1
-            continue
-        if g["next_token"][gb] != o["next_token"][b]:
-            assert bnd & 2, (b, g["next_token"][gb], o["next_token"][b])
-            n_tok_b += 1
-    return dict(requests=B, accept_boundary=n_acc_b, token_boundary=n_tok_b,
-                filter_boundary=n_filt_b)
+    """Asserts parity of one step (the contract of ``oracle.compare``: exact
+    integers, 1e-5 absolute and 1e-4 relative probabilities, a sampled result
+    excused only at the decision the oracle flags as a boundary case); returns
+    the counts of excused cases. ``req_index[b]`` maps the oracle's request b to
+    the GPU's (sampled runs)."""
+    r = compare_step(g, o, wl.draft_off, wl.target_off, g_draft_off=g.get("_draft_off"),
+                     g_target_off=g.get("_target_off"), req_index=req_index,
+                     check_align=check_align, check_q=check_q)
+    assert not r["mismatches"], r["mismatches"][:8]
+    return r

@@ -22,7 +22,8 @@ def _lib():
     tt.load(build_if_missing=True)
 
 
-@pytest.mark.parametrize("name,n_sample", [("b64_g8_v152k", 10), ("b1024_g8_v201k_bf16", 6)])
+@pytest.mark.parametrize("name,n_sample", [("b64_g8_v152k", 10), ("b256_g16_v152k_bf16", 12),
+                                           ("b1024_g8_v201k_bf16", 6)])
 def test_full_size_step_sampled(name, n_sample):
     wl = W.make_workload(name, seed=0, device="cuda")
     inp = tt.device_inputs(wl, "cuda")
@@ -46,7 +47,7 @@ def test_full_size_step_sampled(name, n_sample):
     # a sample of requests, one by one, against the oracle
     rng = np.random.default_rng(1)
     idx = np.unique(np.concatenate([[0, B - 1], rng.choice(B, size=n_sample, replace=False)]))
-    total = dict(accept_boundary=0, token_boundary=0)
+    total = dict(accept_boundary=0, token_boundary=0, filter_boundary=0)
     for b in idx:
         sw = sub_workload(wl, [b])
         o = oracle_step(sw, request_base=int(b))
