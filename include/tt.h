@@ -234,24 +234,27 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
  * workspace and uses a fixed scratch array of TT_NOALLOC_SCRATCH_BYTES (16 MiB)
  * compiled into the library: every GPU that loads the library holds those
  * 16 MiB until the process exits. It allocates nothing.
- *  - Batches that need more scratch than that (tt_workspace_bytes) are refused
- *    with TT_ERR_UNSUPPORTED before anything touches the GPU; the five
- *    workloads the library is measured on all fit.
- *  - The first call on each device looks up the array's device address there
- *    (cudaGetSymbolAddress, with that device current); make that first call
- *    before any stream capture.
+ *  - Every argument check of tt_step runs first, on the host; a refused call
+ *    queues nothing on `stream`. Batches that need more scratch than the
+ *    array holds (tt_workspace_bytes_for with these params) are then refused
+ *    with TT_ERR_UNSUPPORTED; the five workloads the library is measured on
+ *    all fit.
+ *  - The scratch used is the current device's (devices 0..63; others get
+ *    TT_ERR_UNSUPPORTED): `stream` must belong to the current device. The
+ *    first call on each device looks up the array's device address there
+ *    (cudaGetSymbolAddress, once per device even with several host threads);
+ *    make that first call before any stream capture.
  *  - Every call on a device shares the one array, which keeps the last call's
- *    contents; each call clears the two words that must start at zero (the
- *    row pass's error report) on `stream`, and writes every other scratch
- *    value before reading it. Calls whose work overlaps on the GPU (two
- *    streams, or two host threads) race on the array: order them.
+ *    contents; nothing in it needs to start at zero (every value is written
+ *    before it is read, and the row pass's error report is tagged with the
+ *    call it belongs to). Calls whose work overlaps on the GPU (two streams,
+ *    or two host threads) race on the array: order them.
  * Results equal tt_step's for the same arguments. */
 tt_status tt_step_noalloc(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
                           const tt_logits* draft, const float* draft_probs,
                           const tt_logits* target, const tt_params* prm,
                           const tt_step_out* out, void* stream);
 
-/* Static text for a tt_status. */
 /* ------------------------------------------------------------------------
  * Re-encoding and its checks (§4.2; App. A.1, Lemma 1; §4.1 and App. K).
  * ---------------------------------------------------------------------- */
@@ -357,6 +360,7 @@ tt_status tt_verify_sharded(const tt_batch* batch, const float* q_hat, const tt_
                             int32_t* accepted, int32_t* next_token, float* p_hat, float* lse,
                             float* summaries, int32_t* status, void* stream);
 
+/* Static text for a tt_status. */
 const char* tt_status_string(tt_status s);
 
 /* cudaError_t of the last failed launch in this process (0 if none). */

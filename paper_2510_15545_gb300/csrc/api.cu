@@ -15,41 +15,46 @@ namespace {
 
 using namespace tt;
 
-int g_last_cuda_error = 0;
+std::atomic<int> g_last_cuda_error{0};
 std::atomic<int32_t> g_epoch{0x2b6f1000};  // tags each call's row-pass error word
 
 int32_t next_epoch() { return ++g_epoch; }
 
 tt_status cuda_fail(cudaError_t e) {
-  g_last_cuda_error = int(e);
+  g_last_cuda_error.store(int(e));
   return TT_ERR_CUDA;
 }
 
-// Loads all kernels on the current device once, before the first launch there.
+// Loads all kernels on the current device once, before the first launch there
+// (two threads that both find a device not yet done load it twice, which is
+// harmless: loading and setting attributes are idempotent).
 cudaError_t ensure_loaded() {
-  static bool done[64] = {false};
+  static std::atomic<bool> done[64];
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if (dev >= 0 && dev < 64 && done[dev]) return cudaSuccess;
+  if (dev >= 0 && dev < 64 && done[dev].load(std::memory_order_acquire)) return cudaSuccess;
   if ((e = preload_align()) != cudaSuccess) return e;
   if ((e = preload_rowpass()) != cudaSuccess) return e;
   if ((e = preload_decide()) != cudaSuccess) return e;
   if ((e = preload_filter()) != cudaSuccess) return e;
   if ((e = preload_shard()) != cudaSuccess) return e;
-  if (dev >= 0 && dev < 64) done[dev] = true;
+  if (dev >= 0 && dev < 64) done[dev].store(true, std::memory_order_release);
   return cudaSuccess;
 }
 
 int sm_count_current() {
-  static int cached[64] = {0};
+  static std::atomic<int> cached[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 148;
-  if (dev < 64 && cached[dev] > 0) return cached[dev];
+  if (dev < 64) {
+    const int c = cached[dev].load(std::memory_order_relaxed);
+    if (c > 0) return c;
+  }
   int n = 0;
   if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
     n = 148;
-  if (dev < 64) cached[dev] = n;
+  if (dev < 64) cached[dev].store(n, std::memory_order_relaxed);
   return n;
 }
 
@@ -212,6 +217,34 @@ tt_status fill_align_args(const tt_batch* bt, const tt_vocab* vd, const tt_vocab
 
 namespace tt {
 tt_status record_cuda_error(cudaError_t e) { return cuda_fail(e); }
+
+tt_status step_check(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
+                     const tt_logits* draft, const float* draft_probs, const tt_logits* target,
+                     const tt_params* prm, const tt_step_out* out, size_t* need) {
+  *need = 0;
+  if (!batch_ok(batch) || !params_ok(prm)) return TT_ERR_INVALID_ARG;
+  if (!out || !out->accepted || !out->next_token || !out->status) return TT_ERR_INVALID_ARG;
+  if (batch->B == 0) return TT_OK;
+  if (!vocab_ok(vd) || !vocab_ok(vt)) return TT_ERR_INVALID_ARG;
+  if ((batch->n_draft > 0 && !batch->draft_ids) || (batch->n_target > 0 && !batch->target_ids))
+    return TT_ERR_INVALID_ARG;
+  const bool full_q = prm->full_q != 0;
+  const bool from_logits = draft_probs == nullptr || full_q;
+  if (!logits_ok(target, int64_t(batch->n_target) + batch->B)) return TT_ERR_INVALID_ARG;
+  if (from_logits && !logits_ok(draft, batch->n_draft)) return TT_ERR_INVALID_ARG;
+  if (full_q && draft->n_cols != target->n_cols) return TT_ERR_INVALID_ARG;
+  if (!filters_supported(prm)) return TT_ERR_UNSUPPORTED;
+  // given draft probabilities are taken as they are (no draft filter)
+  const int kd = from_logits ? k_draft(prm) : 0, kt = k_target(prm);
+  if (full_q && (kd > 0) != (kt > 0)) return TT_ERR_UNSUPPORTED;
+  AlignArgs a;
+  const tt_status st = fill_align_args(batch, vd, vt, prm, a);
+  if (st != TT_OK) return st;
+  *need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target,
+                           from_logits ? draft->n_cols : 0, target->n_cols, kd, kt)
+              .bytes;
+  return TT_OK;
+}
 }  // namespace tt
 
 extern "C" {
@@ -448,27 +481,16 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
                   const tt_logits* draft, const float* draft_probs, const tt_logits* target,
                   const tt_params* prm, void* workspace, size_t workspace_bytes,
                   const tt_step_out* out, void* stream) {
-  if (!batch_ok(batch) || !params_ok(prm)) return TT_ERR_INVALID_ARG;
-  if (!out || !out->accepted || !out->next_token || !out->status) return TT_ERR_INVALID_ARG;
-  if (batch->B == 0) return TT_OK;
-  if (!vocab_ok(vd) || !vocab_ok(vt)) return TT_ERR_INVALID_ARG;
-  if ((batch->n_draft > 0 && !batch->draft_ids) || (batch->n_target > 0 && !batch->target_ids))
+  size_t need = 0;
+  const tt_status chk = step_check(batch, vd, vt, draft, draft_probs, target, prm, out, &need);
+  if (chk != TT_OK || batch->B == 0) return chk;
+  if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
     return TT_ERR_INVALID_ARG;
   const bool full_q = prm->full_q != 0;
   const bool from_logits = draft_probs == nullptr || full_q;
-  if (!logits_ok(target, int64_t(batch->n_target) + batch->B)) return TT_ERR_INVALID_ARG;
-  if (from_logits && !logits_ok(draft, batch->n_draft)) return TT_ERR_INVALID_ARG;
-  if (full_q && draft->n_cols != target->n_cols) return TT_ERR_INVALID_ARG;
-  if (!filters_supported(prm)) return TT_ERR_UNSUPPORTED;
-  // given draft probabilities are taken as they are (no draft filter)
   const int kd = from_logits ? k_draft(prm) : 0, kt = k_target(prm);
-  if (full_q && (kd > 0) != (kt > 0)) return TT_ERR_UNSUPPORTED;
   const bool filtered = kd > 0 || kt > 0;
   const int V_d = from_logits ? draft->n_cols : 0;
-  const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d,
-                                       target->n_cols, kd, kt).bytes;
-  if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
-    return TT_ERR_INVALID_ARG;
   const int32_t* dcols = batch->draft_cols ? batch->draft_cols : batch->draft_ids;
   const int32_t* tcols = batch->target_cols ? batch->target_cols : batch->target_ids;
   AlignArgs a;
@@ -703,7 +725,7 @@ const char* tt_status_string(tt_status s) {
   return "unknown status";
 }
 
-int32_t tt_last_cuda_error(void) { return g_last_cuda_error; }
+int32_t tt_last_cuda_error(void) { return g_last_cuda_error.load(); }
 
 int32_t tt_version(void) { return 110; }
 

@@ -8,7 +8,9 @@
 // tt_step needs, so this entry point brings its own: a fixed array in the
 // library's device image, set up once per device and reused by every call on
 // that device.
+#include <atomic>
 #include <cstdint>
+#include <mutex>
 
 #include "tt_device.cuh"
 #include "tt_launch.h"
@@ -19,9 +21,21 @@ namespace {
 // the library's module is loaded there until the process exits.
 static __device__ __align__(256) unsigned char tt_noalloc_scratch[TT_NOALLOC_SCRATCH_BYTES];
 
-// Device address of the scratch array per device; host code cannot use the
+constexpr int kMaxDevices = 64;
+
+// Device address of the scratch array per device, looked up once per device
+// (under its once-flag) with that device current: host code cannot use the
 // array's name as a device address, it is only a host-side stand-in.
-void* g_scratch_ptr[64] = {nullptr};
+std::once_flag g_once[kMaxDevices];
+std::atomic<void*> g_scratch_ptr[kMaxDevices];
+cudaError_t g_setup_error[kMaxDevices];
+
+void look_up_scratch(int dev) {
+  void* ptr = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&ptr, tt_noalloc_scratch);
+  g_setup_error[dev] = e == cudaSuccess && ptr == nullptr ? cudaErrorInvalidSymbol : e;
+  if (g_setup_error[dev] == cudaSuccess) g_scratch_ptr[dev].store(ptr, std::memory_order_release);
+}
 
 }  // namespace
 
@@ -30,31 +44,23 @@ extern "C" tt_status tt_step_noalloc(const tt_batch* batch, const tt_vocab* vd,
                                      const float* draft_probs, const tt_logits* target,
                                      const tt_params* prm, const tt_step_out* out,
                                      void* stream) {
-  if (!batch || !prm || !target || !out) return TT_ERR_INVALID_ARG;
-  if (batch->B < 0 || batch->n_draft < 0 || batch->n_target < 0) return TT_ERR_INVALID_ARG;
-  // size check first: nothing touches the GPU before it passes
-  const bool from_logits = draft_probs == nullptr || prm->full_q != 0;
-  if (from_logits && !draft) return TT_ERR_INVALID_ARG;
-  const int V_d = from_logits ? draft->n_cols : 0;
-  const size_t need = tt_workspace_bytes_for(batch, V_d, target->n_cols, prm);
-  if (need > size_t(TT_NOALLOC_SCRATCH_BYTES)) return TT_ERR_UNSUPPORTED;
+  // every check of tt_step first, on the host: a refused call queues nothing
+  size_t need = 0;
+  const tt_status chk =
+      tt::step_check(batch, vd, vt, draft, draft_probs, target, prm, out, &need);
+  if (chk != TT_OK) return chk;
   if (batch->B == 0) return TT_OK;
+  if (need == 0 || need > size_t(TT_NOALLOC_SCRATCH_BYTES)) return TT_ERR_UNSUPPORTED;
 
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return TT_ERR_CUDA;
-  if (g_scratch_ptr[dev] == nullptr) {  // set-up, once per device, on that device
-    void* ptr = nullptr;
-    if (cudaGetSymbolAddress(&ptr, tt_noalloc_scratch) != cudaSuccess || ptr == nullptr)
-      return TT_ERR_CUDA;
-    g_scratch_ptr[dev] = ptr;
-  }
-  void* ws = g_scratch_ptr[dev];
-  // the row-pass error words must not carry a previous call's flags
-  const tt::Workspace lay =
-      tt::workspace_layout(ws, batch->B, batch->n_draft, batch->n_target, V_d, target->n_cols);
-  if (cudaMemsetAsync(lay.err, 0, 2 * sizeof(int32_t), static_cast<cudaStream_t>(stream)) !=
-      cudaSuccess)
-    return TT_ERR_CUDA;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return tt::record_cuda_error(e);
+  if (dev < 0 || dev >= kMaxDevices) return TT_ERR_UNSUPPORTED;
+  std::call_once(g_once[dev], look_up_scratch, dev);  // set-up, once per device
+  void* ws = g_scratch_ptr[dev].load(std::memory_order_acquire);
+  if (ws == nullptr) return tt::record_cuda_error(g_setup_error[dev]);
+  // nothing in the scratch needs to start at zero: every value is written
+  // before it is read, and the row pass's error report carries the call's tag
   return tt_step(batch, vd, vt, draft, draft_probs, target, prm, ws,
                  size_t(TT_NOALLOC_SCRATCH_BYTES), out, stream);
 }

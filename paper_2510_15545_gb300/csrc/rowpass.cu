@@ -15,6 +15,7 @@
 // shared memory (no block barrier) and frees the stage. Every wait is bounded in time; on timeout the kernel sets
 // an error word that the decision kernel turns into a per-request status.
 #include <algorithm>
+#include <atomic>
 #include <cstdint>
 #include <cstdlib>
 
@@ -814,19 +815,47 @@ cudaError_t preload_rowpass() {
   return preload_pair<TT_BF16, TT_BF16>();
 }
 
-// Test hooks, read from the environment at each launch (off unless set):
-// TT_TEST_STALL_STAGE=n makes CTA 0 hold the stage of its n-th consumer step, and
-// TT_TEST_WAIT_MS=t sets the limit of every pipeline wait, so that a test can
-// watch the bounded waits run out and the call report TT_REQ_TIMEOUT.
+namespace {
+
+// Test hook of the bounded waits, read from the environment once per process
+// (off unless set): TT_TEST_STALL_STAGE=n makes CTA 0 of the first
+// TT_TEST_STALL_LAUNCHES row-pass launches (default 1) hold the stage of its
+// n-th consumer step, with every pipeline wait of those launches limited to
+// TT_TEST_WAIT_MS milliseconds, so that a test can watch the waits run out and
+// the call report TT_REQ_TIMEOUT, then see the next launches run normally.
+struct StallHook {
+  int stall_stage = -1;
+  uint64_t wait_ns = kWaitLimitNs;
+  std::atomic<int> launches_left{0};
+  StallHook() {
+    if (const char* v = std::getenv("TT_TEST_STALL_STAGE")) stall_stage = std::atoi(v);
+    if (stall_stage < 0) return;
+    if (const char* v = std::getenv("TT_TEST_WAIT_MS")) {
+      const long long ms = std::atoll(v);
+      if (ms > 0) wait_ns = uint64_t(ms) * 1000000ull;
+    }
+    int n = 1;
+    if (const char* v = std::getenv("TT_TEST_STALL_LAUNCHES")) n = std::atoi(v);
+    launches_left.store(n > 0 ? n : 0);
+  }
+};
+
+StallHook& stall_hook() {
+  static StallHook hook;  // initialised once, thread-safe
+  return hook;
+}
+
+}  // namespace
+
 cudaError_t launch_rowpass(const RowPassArgs& args, int dt_d, int dt_t, cudaStream_t stream,
                            int sm_count, bool pdl) {
   RowPassArgs a = args;
   a.stall_stage = -1;
   a.wait_ns = kWaitLimitNs;
-  if (const char* v = std::getenv("TT_TEST_STALL_STAGE")) a.stall_stage = std::atoi(v);
-  if (const char* v = std::getenv("TT_TEST_WAIT_MS")) {
-    const long long ms = std::atoll(v);
-    if (ms > 0) a.wait_ns = uint64_t(ms) * 1000000ull;
+  StallHook& hook = stall_hook();
+  if (hook.stall_stage >= 0 && hook.launches_left.fetch_sub(1) > 0) {
+    a.stall_stage = hook.stall_stage;
+    a.wait_ns = hook.wait_ns;
   }
   if (dt_d == TT_F32 && dt_t == TT_F32) return launch_pair<TT_F32, TT_F32>(a, stream, sm_count, pdl);
   if (dt_d == TT_F32 && dt_t == TT_BF16) return launch_pair<TT_F32, TT_BF16>(a, stream, sm_count, pdl);

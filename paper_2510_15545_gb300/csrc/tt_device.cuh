@@ -258,10 +258,21 @@ __device__ __forceinline__ double philox_uniform(uint64_t seed, uint64_t pos, ui
 }
 
 // Records a failure of call `epoch` (TT_REQ_TIMEOUT / TT_REQ_INTERNAL bits).
+// Error report of a call: err[0] = the reporting call's epoch, err[1] = its
+// TT_REQ_* bits, updated together as one 64-bit word, so that a report of a
+// new call replaces an earlier call's bits instead of adding to them (the
+// words never need clearing). The compare-and-swap retries only while other
+// reporters of the same call change the word.
 __device__ __forceinline__ void report_error(int32_t* err, int32_t epoch, int32_t bits) {
   if (!err) return;
-  atomicOr(&err[1], bits);
-  atomicExch(&err[0], epoch);
+  unsigned long long* w = reinterpret_cast<unsigned long long*>(err);
+  unsigned long long seen = __ldcg(w), want;
+  do {
+    want = seen;
+    const uint32_t old_bits = int32_t(uint32_t(want)) == epoch ? uint32_t(want >> 32) : 0u;
+    seen = atomicCAS(w, want,
+                     (uint64_t(old_bits | uint32_t(bits)) << 32) | uint64_t(uint32_t(epoch)));
+  } while (seen != want);
 }
 
 // ------------------------------------------------------------ warp sorting

@@ -150,4 +150,11 @@ cudaError_t preload_filter();
 // Records a failed CUDA call for tt_last_cuda_error() and returns TT_ERR_CUDA.
 tt_status record_cuda_error(cudaError_t e);
 
+// Every argument check of tt_step, on the host only (nothing is queued on a
+// stream): TT_OK and the workspace bytes the step needs (0 for an empty batch),
+// or the status tt_step would return for these arguments.
+tt_status step_check(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
+                     const tt_logits* draft, const float* draft_probs, const tt_logits* target,
+                     const tt_params* prm, const tt_step_out* out, size_t* need);
+
 }  // namespace tt

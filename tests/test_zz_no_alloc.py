@@ -35,6 +35,24 @@ def test_batch_beyond_the_scratch_is_refused_on_the_host():
     assert code == binding.TT_ERR_UNSUPPORTED
 
 
+def test_invalid_params_are_refused_before_the_size_check():
+    # an invalid top-k (-1) must not slip past the size check: tt_step's own
+    # checks run first and refuse the call before anything touches the GPU
+    lib = tt.load(build_if_missing=True)
+    b = binding._Batch(1, 1, 10_000_000, 1, 1, 16, 16, None, 16, 16, None)
+    v = binding._Vocab(16, 16, 1, 1)
+    lg = binding._Logits(256, binding.TT_F32, 151936, 151936, 10_000_001)
+    out = binding._StepOut(16, 16, 16, None, None, None, None, None, None, None)
+    keep = []
+    for bad in (dict(top_k_target=-1), dict(top_k_draft=-1), dict(top_k_target=33),
+                dict(temp_target=0.0)):
+        prm = binding.Params(**bad)._c(keep)
+        code = lib.tt_step_noalloc(ctypes.byref(b), ctypes.byref(v), ctypes.byref(v),
+                                   ctypes.byref(lg), None, ctypes.byref(lg), ctypes.byref(prm),
+                                   ctypes.byref(out), None)
+        assert code == binding.TT_ERR_INVALID_ARG, bad
+
+
 def _check_same(wl, ref, got):
     for k in ("status", "accepted", "next_token", "path_len", "cost", "map"):
         assert torch.equal(ref[k], got[k]), k
@@ -55,13 +73,24 @@ def test_noalloc_step_equals_step_on_two_calls_in_a_row():
     workloads = [W.make_workload("b64_g8_v152k", B=16, seed=3, vocab_cache=_CACHE),
                  W.make_workload("b1024_g8_v201k_bf16", B=8, seed=4, vocab_cache=_CACHE),
                  W.make_workload("dtw_4096x64", B=24, seed=5, vocab_cache=_CACHE)]
-    for wl in workloads:
+    filters = dict(temp_draft=0.7, temp_target=0.7, top_k_draft=20, top_p_draft=0.8,
+                   top_k_target=20, top_p_target=0.8)
+    cases = [(wl, {}, False) for wl in workloads]
+    cases.append((workloads[0], filters, False))  # kept sets and lists in the scratch
+    cases.append((workloads[1], {}, True))        # caller-given draft probabilities
+    for wl, f, given in cases:
         inp = tt.device_inputs(wl, "cuda")
+        prm = inp["params"]
+        for k, v in f.items():
+            setattr(prm, k, v)
+        probs = None
+        if given:
+            probs = torch.rand(wl.n_draft, device="cuda") * 0.9 + 0.05
         args = (inp["batch"], inp["vd"], inp["vt"], inp["draft_logits"], inp["target_logits"],
-                inp["params"])
-        ref = tt.tt_step(*args)
-        first = tt.tt_step_noalloc(*args)
-        second = tt.tt_step_noalloc(*args)
+                prm)
+        ref = tt.tt_step(*args, draft_probs=probs)
+        first = tt.tt_step_noalloc(*args, draft_probs=probs)
+        second = tt.tt_step_noalloc(*args, draft_probs=probs)
         torch.cuda.synchronize()
         assert int((ref["status"] != 0).sum()) == 0
         _check_same(wl, ref, first)
