@@ -29,7 +29,7 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-DEFAULT_WORKLOAD = "b64_g8_v152k"
+DEFAULT_WORKLOAD = "b1024_g8_v201k_bf16"
 METRIC = "verified draft positions/sec (batch×γ) and HBM GB/s vs 8 TB/s; DTW pairs/sec"
 UNIT = "positions/s"
 L2_BYTES = 129 * 1024 * 1024
@@ -51,6 +51,8 @@ def parse_args(argv=None):
                          "batches are for profiler captures, not bench lines")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-extra", action="store_true",
+                    help="time only --workload, not also the other workloads")
     ap.add_argument("--temp", type=float, default=None,
                     help="temperature of draft and target rows (default: the workload's)")
     ap.add_argument("--top-k", type=int, default=0,
@@ -253,26 +255,32 @@ def step_kwargs(args) -> dict:
     return kw
 
 
-def oracle_sample_rate(wl, budget_s: float, step_kw=None):
+def oracle_sample_rate(wl, budget_s: float, step_kw=None, keep: bool = False):
     """Times the oracle (as it stands) over requests of the workload, cycling
-    through them until the CPU budget is spent; returns positions/s and a note."""
+    through them until the CPU budget is spent; returns positions/s, a note,
+    the requests and seconds, and (keep=True) each request's first oracle
+    result with its one-request workload."""
     import oracle
     oracle.build()
     order = list(range(wl.B))
-    subs = {}
-    done_req, positions, elapsed, passes = 0, 0, 0.0, 0
+    subs, outs = {}, {}
+    done_req, positions, elapsed = 0, 0, 0.0
     while elapsed < budget_s:
         b = order[done_req % wl.B]
         if b not in subs:
             subs[b] = wl.subset([b])
         sw = subs[b]
         t = time.perf_counter()
-        oracle.step(sw, request_base=b, **(step_kw or {}))
+        o = oracle.step(sw, request_base=b, **(step_kw or {}))
         elapsed += time.perf_counter() - t
+        if keep and b not in outs:
+            outs[b] = (sw, o)
         positions += int(sw.draft_off[-1])
         done_req += 1
     sample = ("%d requests of the %s batch (cycling from request 0), oracle single-threaded, "
               "fp64, %.1f s of CPU time" % (done_req, wl.spec.name, elapsed))
+    if keep:
+        return positions / elapsed, sample, done_req, elapsed, outs
     return positions / elapsed, sample, done_req, elapsed
 
 
@@ -329,23 +337,13 @@ def oracle_all_cores_rate(wl, budget_s: float, per_worker: int = 2, step_kw=None
 
 # -------------------------------------------------------------- my arm
 
-def run_mine(args):
-    import numpy as np
-    import torch
+EXTRA_WORKLOADS = ("b64_g8_v152k", "b256_g16_v152k_bf16", "dtw_4096x64", "b1_g4_v32k")
 
-    rank, ws, local = dist_env()
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    dist_init(ws, "nccl")
-    import paper_2510_15545_gb300 as tt
-    from paper_2510_15545_gb300 import workload as W
-    tt.load(build_if_missing=(rank == 0 or ws == 1))
-    barrier(ws)
-    tt.load()
 
-    name = args.workload
-    K = args.steps if args.steps is not None else default_steps(name)
-    Wm = max(3, args.warmup)
+def prepare_step(tt, W, name, args, rank, dev, stream):
+    """The workload's inputs on the device, its step parameters, one untimed
+    step with every output (mapped draft rows, acceptance, the parity sample),
+    and a prepared call for the timed loop."""
     wl = W.make_workload(name, B=args.batch, seed=rank, device=str(dev))
     inp = tt.device_inputs(wl, dev)
     prm = inp["params"]
@@ -354,24 +352,24 @@ def run_mine(args):
         prm.temp_draft = prm.temp_target = args.temp
     prm.top_k_draft = prm.top_k_target = args.top_k
     prm.top_p_draft = prm.top_p_target = args.top_p
-    filtered = args.top_k > 0
-    batch, vd, vt = inp["batch"], inp["vd"], inp["vt"]
-    dl, tl = inp["draft_logits"], inp["target_logits"]
-    stream = torch.cuda.current_stream(dev)
-
-    # one untimed step with every output: mapped draft rows, acceptance
-    full = tt.tt_step(batch, vd, vt, dl, tl, prm)
+    full = tt.tt_step(inp["batch"], inp["vd"], inp["vt"], inp["draft_logits"],
+                      inp["target_logits"], prm)
+    import torch
     torch.cuda.synchronize(dev)
-    mp = full["map"].cpu().numpy()
-    acc = full["accepted"].cpu().numpy()
     assert int((full["status"] != 0).sum()) == 0, "a request failed"
-    ab = algorithmic_bytes(wl, mp)
-    m = np.diff(wl.target_off)
+    call = tt.StepCall(inp["batch"], inp["vd"], inp["vt"], inp["draft_logits"],
+                       inp["target_logits"], prm,
+                       out=tt.step_outputs(inp["batch"], dev, full=False), stream=stream)
+    return wl, inp, prm, full, call
 
-    call = tt.StepCall(batch, vd, vt, dl, tl, prm, out=tt.step_outputs(batch, dev, full=False),
-                       stream=stream)
-    # stage events on a strided subset of the timed steps: at most one step in
-    # ten (events between the kernels break their dependent-launch overlap)
+
+def time_steps(call, K, Wm, stream, dev, ws):
+    """W untimed steps, then exactly K steps bracketed by a barrier and a device
+    synchronise on both sides, timed with CUDA events on the launching stream.
+    Stage events sit on at most one timed step in ten (events between the
+    kernels break their dependent-launch overlap). Returns the time of the K
+    steps (seconds, this rank), the host interval and the mean stage times."""
+    import torch
     stride = max(10, math.ceil(K / 2000))
     sampled = list(range(0, K, stride))
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in sampled]
@@ -379,13 +377,9 @@ def run_mine(args):
         for e in e4:
             e.record(stream)
     handles = [[e.cuda_event for e in e4] for e4 in ev]
-
     for _ in range(Wm):
         call()
     torch.cuda.synchronize(dev)
-
-    clocks = ClockSampler(local)
-    time.sleep(0.3)
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     barrier(ws)
@@ -403,13 +397,112 @@ def run_mine(args):
     torch.cuda.synchronize(dev)
     h1 = time.perf_counter()
     barrier(ws)
-    time.sleep(0.2)
-    clocks.stop()
     sec = t_start.elapsed_time(t_end) / 1e3
+    stages = {"align": statistics.mean(e4[0].elapsed_time(e4[1]) for e4 in ev),
+              "rowpass": statistics.mean(e4[1].elapsed_time(e4[2]) for e4 in ev),
+              "decide": statistics.mean(e4[2].elapsed_time(e4[3]) for e4 in ev),
+              "sampled_steps": len(sampled)}
+    return sec, (h0, h1), stages
+
+
+def extra_workload(tt, W, name, args, rank, ws, dev, stream, clocks, peak):
+    """Another workload, timed in the same run as the headline one and with the
+    same rules (its own K steps after W warm-up steps, inputs resident in HBM):
+    the step time, the metric, the step's and the row pass's HBM rate, and the
+    DTW alignment's pairs per second alone."""
+    import numpy as np
+    import torch
+    wl, inp, prm, full, call = prepare_step(tt, W, name, args, rank, dev, stream)
+    K = args.steps if args.steps is not None else min(default_steps(name), 2000)
+    Wm = max(3, args.warmup)
+    ab = algorithmic_bytes(wl, full["map"].cpu().numpy())
+    sec, (h0, h1), st = time_steps(call, K, Wm, stream, dev, ws)
     sec_max = max_over_ranks(sec, ws, dev)
-    align_ms = statistics.mean(e4[0].elapsed_time(e4[1]) for e4 in ev)
-    row_ms = statistics.mean(e4[1].elapsed_time(e4[2]) for e4 in ev)
-    dec_ms = statistics.mean(e4[2].elapsed_time(e4[3]) for e4 in ev)
+    align_alone_ms = run_align_alone(tt, wl, inp, prm, dev, stream)
+    acc = full["accepted"].cpu().numpy()
+    m = np.diff(wl.target_off)
+    row_gbs = ab["total"] / (st["rowpass"] / 1e3) / 1e9
+    r = {"workload": name, "batch_per_gpu": wl.B, "gamma": wl.spec.k,
+         "dtype": "bf16" if wl.target_logits.element_size() == 2 else "f32", "steps": K,
+         "ms_per_step": sec_max * 1e3 / K, "value": wl.n_draft * K * ws / sec_max,
+         "unit": UNIT, "algorithmic_bytes": ab["total"],
+         "hbm_gbs_step": ab["total"] / (sec / K) / 1e9,
+         "step_frac_of_8tbs": ab["total"] / (sec / K) / 8e12,
+         "rowpass_gbs": row_gbs, "rowpass_frac": row_gbs / peak,
+         "rowpass_traffic": profiled_traffic(name, args.top_k),
+         "stage_ms": st, "dtw_pairs_per_s": wl.B / (align_alone_ms / 1e3),
+         "accept_rate": float(acc.sum() / max(1, m.sum())), "clocks": clocks.summary(h0, h1)}
+    del wl, inp, full, call
+    torch.cuda.empty_cache()
+    return r
+
+
+def cpu_baseline_leg(wl, full, args, step_kw):
+    """The oracle, as it stands, on the host: one core over a bounded sample of
+    the workload's requests (cycling from request 0), then one process per
+    host core. The single-core sample's oracle outputs are also compared with
+    the device step's outputs for the same requests (the untimed full step,
+    launched as the timed ones), which gives the boundary-case counts the
+    parity contract reports: accept decisions, drawn tokens and top-p cuts that
+    differ within 1e-6 of their boundary, and any difference outside it."""
+    from oracle.compare import compare_step
+    rate, sample, nreq, el, outs = oracle_sample_rate(wl, args.cpu_seconds, step_kw,
+                                                      keep=True)
+    cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
+    g = {k: v.cpu().numpy() for k, v in full.items()}
+    tot = {"requests_compared": 0, "accept_boundary": 0, "token_boundary": 0,
+           "filter_boundary": 0, "mismatches": 0}
+    first = []
+    for b, (sw, o) in sorted(outs.items()):
+        r = compare_step(g, o, sw.draft_off, sw.target_off, g_draft_off=wl.draft_off,
+                         g_target_off=wl.target_off, req_index=[b])
+        tot["requests_compared"] += 1
+        for k in ("accept_boundary", "token_boundary", "filter_boundary"):
+            tot[k] += r[k]
+        tot["mismatches"] += len(r["mismatches"])
+        first += r["mismatches"][:2]
+    tot["first_mismatches"] = first[:4]
+    tot["note"] = ("requests %s of the full-size step compared with the oracle: integers "
+                   "exact, probabilities 1e-5 absolute and 1e-4 relative, a sampled result "
+                   "excused only at the decision within 1e-6 of its boundary"
+                   % ("0..%d" % (tot["requests_compared"] - 1)))
+    rate, sample, n = oracle_all_cores_rate(wl, min(args.cpu_seconds, 8.0), step_kw=step_kw)
+    cpu_all = {"value": rate, "unit": UNIT, "cores": n, "kind": "oracle", "sample": sample}
+    return cpu, cpu_all, tot
+
+
+def run_mine(args):
+    import numpy as np
+    import torch
+
+    rank, ws, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist_init(ws, "nccl")
+    import paper_2510_15545_gb300 as tt
+    from paper_2510_15545_gb300 import workload as W
+    tt.load(build_if_missing=(rank == 0 or ws == 1))
+    barrier(ws)
+    tt.load()
+
+    name = args.workload
+    K = args.steps if args.steps is not None else default_steps(name)
+    Wm = max(3, args.warmup)
+    stream = torch.cuda.current_stream(dev)
+    wl, inp, prm, full, call = prepare_step(tt, W, name, args, rank, dev, stream)
+    filtered = args.top_k > 0
+    dl, tl = inp["draft_logits"], inp["target_logits"]
+    mp = full["map"].cpu().numpy()
+    acc = full["accepted"].cpu().numpy()
+    ab = algorithmic_bytes(wl, mp)
+    m = np.diff(wl.target_off)
+
+    clocks = ClockSampler(local)
+    time.sleep(0.3)
+    sec, (h0, h1), st = time_steps(call, K, Wm, stream, dev, ws)
+    sec_max = max_over_ranks(sec, ws, dev)
+    clk = clocks.summary(h0, h1)
+    align_ms, row_ms = st["align"], st["rowpass"]
 
     positions = wl.n_draft  # verified draft positions per step (batch x gamma)
     value = positions * K * ws / sec_max
@@ -432,43 +525,54 @@ def run_mine(args):
     if args.shards > 0 and not filtered and not prm.full_q:
         sharded = run_sharded(tt, wl, inp, prm, full["q_hat"], dev, stream, args.shards)
 
-    cpu = cpu_all = None
+    cpu = cpu_all = bnd = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        rate, sample, nreq, el = oracle_sample_rate(wl, args.cpu_seconds, step_kwargs(args))
-        cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
-        rate, sample, n = oracle_all_cores_rate(wl, min(args.cpu_seconds, 8.0),
-                                                step_kw=step_kwargs(args))
-        cpu_all = {"value": rate, "unit": UNIT, "cores": n, "kind": "oracle", "sample": sample}
+        cpu, cpu_all, bnd = cpu_baseline_leg(wl, full, args, step_kwargs(args))
 
-    clk = clocks.summary(h0, h1)
+    extras = {}
+    if not args.no_extra and args.batch is None:
+        keep = dict(wl=wl, dl_shape=list(dl.shape), tl_shape=list(tl.shape),
+                    in_bytes=dl.numel() * dl.element_size() + tl.numel() * tl.element_size())
+        del inp, full, call, dl, tl
+        torch.cuda.empty_cache()
+        for x in EXTRA_WORKLOADS:
+            if x != name:
+                extras[x] = extra_workload(tt, W, x, args, rank, ws, dev, stream, clocks, peak)
+        wl = keep["wl"]
+        dl_shape, tl_shape, in_bytes = keep["dl_shape"], keep["tl_shape"], keep["in_bytes"]
+    else:
+        dl_shape, tl_shape = list(dl.shape), list(tl.shape)
+        in_bytes = dl.numel() * dl.element_size() + tl.numel() * tl.element_size()
+    time.sleep(0.2)
+    clocks.stop()
+
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": K,
         "warmup": Wm, "ms_per_step": sec_max * 1e3 / K, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": wl.spec.dtype.__repr__().split(".")[-1]
-        .replace("float32", "f32").replace("bfloat16", "bf16"),
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if wl.target_logits.element_size() == 2 else "f32",
         "data": "synthetic (seeded byte-string vocabularies, greedy re-encoding, Zipf logits)",
         "config": {"workload": name, "batch_per_gpu": wl.B, "gamma": wl.spec.k,
                    "V_d": wl.spec.V_d, "V_t": wl.spec.V_t,
-                   "logits_cols": [int(dl.shape[1]), int(tl.shape[1])],
+                   "logits_cols": [int(dl_shape[1]), int(tl_shape[1])],
                    "target_tokens_per_gpu": wl.n_target, "window": prm.window,
                    "temperature": [prm.temp_draft, prm.temp_target],
                    "filters": ({"top_k": args.top_k, "top_p": args.top_p} if filtered
                                else None),
                    "parallelism": "dp%d (independent requests per GPU)" % ws,
                    "l2": "inputs %.0f MB exceed the 129 MB L2; no flush between steps"
-                         % ((dl.numel() * dl.element_size() + tl.numel() * tl.element_size()) / 1e6)
-                   if ab["total"] > L2_BYTES else "inputs fit in L2",
+                         % (in_bytes / 1e6) if ab["total"] > L2_BYTES else "inputs fit in L2",
                    "accept_rate": float(acc.sum() / max(1, m.sum())),
                    "mean_accepted": float(acc.mean())},
         "hbm_gbs_step": step_gbs,
+        "step_frac_of_8tbs": step_gbs / 8000.0,
         "dtw_pairs_per_s": wl.B / (align_alone_ms / 1e3),
         "dtw": {"ms_alone": align_alone_ms, "ms_in_step": align_ms,
                 "pairs_per_s_in_step": wl.B / (align_ms / 1e3),
                 "band_cells": cells, "band_cells_per_s": cells / (align_alone_ms / 1e3),
                 "note": "dtw_pairs_per_s: tt_align alone (one warp per pair), 200 calls; in "
                         "the step the alignment takes one CTA per SM beside the row pass"},
-        "stage_ms": {"align": align_ms, "rowpass": row_ms, "decide": dec_ms,
-                     "sampled_steps": len(sampled)},
+        "stage_ms": st,
         "roofline": {"bound": "hbm", "kernel": "rowpass_kernel", "achieved": achieved,
                      "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                      "peak_kind": "%s copy bandwidth (hbm_gbs)" % peak_kind,
@@ -489,6 +593,10 @@ def run_mine(args):
         line["cpu_baseline"] = cpu
     if cpu_all is not None:
         line["cpu_baseline_all_cores"] = cpu_all
+    if bnd is not None:
+        line["boundary_cases"] = bnd
+    if extras:
+        line["workloads"] = extras
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:

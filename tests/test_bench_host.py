@@ -138,3 +138,25 @@ def test_oracle_legs_run_the_step_parameters_of_the_run(monkeypatch):
     # a worker job carries the same parameters
     pos, sec, done = bench._oracle_job(([(0, wl.subset([0]))], 0.0, bench.step_kwargs(args)))
     assert done == 1 and pos == 4 and seen[-1]["top_k_target"] == 20
+
+
+def test_cpu_leg_counts_boundary_cases_and_mismatches(monkeypatch):
+    """The CPU-baseline leg compares its oracle sample with the device step's
+    outputs for the same requests: the oracle against itself gives no
+    mismatch; a planted wrong next token is counted as one."""
+    import oracle
+    import torch
+    from paper_2510_15545_gb300 import workload as W
+    monkeypatch.setattr(bench, "oracle_all_cores_rate", lambda wl, b, step_kw=None: (1.0, "-", 1))
+    wl = W.make_workload("b1_g4_v32k", B=3, seed=2)
+    o = oracle.step(wl)
+    keys = ("status", "accepted", "next_token", "path_len", "cost", "map", "q_hat", "p_hat", "lse")
+    full = {k: torch.as_tensor(np.asarray(o[k])) for k in keys}
+    full["path"] = torch.as_tensor(np.asarray(o["path"]).ravel())
+    args = bench.parse_args(["--cpu-seconds", "0.05"])
+    cpu, cpu_all, bnd = bench.cpu_baseline_leg(wl, full, args, bench.step_kwargs(args))
+    assert cpu["cores"] == 1 and cpu["kind"] == "oracle"
+    assert bnd["requests_compared"] == 3 and bnd["mismatches"] == 0
+    full["next_token"][1] = (int(o["next_token"][1]) + 7) % wl.target_logits.shape[1]
+    cpu, cpu_all, bnd = bench.cpu_baseline_leg(wl, full, args, bench.step_kwargs(args))
+    assert bnd["mismatches"] == 1 and bnd["first_mismatches"]
