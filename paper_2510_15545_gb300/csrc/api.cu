@@ -180,6 +180,15 @@ void attach_kept(DecideArgs& d, const Workspace& ws) {
   d.head_t = ws.head_t;
 }
 
+// Share of the target rows the step's row pass streams before it waits for
+// the alignment (in eighths): half, or seven eighths when the batch holds so
+// many draft tokens (B x max_k of 32768 and more, each a row of the DTW tile)
+// that the alignment outlasts half of the target rows; the rest is drawn
+// dynamically after the wait.
+int pre_wait_eighths(const tt_batch* b) {
+  return int64_t(b->B) * b->max_k >= 32768 ? 7 : 4;
+}
+
 void record(const tt_params* p, int i, cudaStream_t s) {
   if (p->events && p->events[i]) cudaEventRecord(static_cast<cudaEvent_t>(p->events[i]), s);
 }
@@ -353,6 +362,7 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
     r.err = ws.err;
     r.epoch = next_epoch();
     r.work = ws.work;
+    r.pre_eighths = 4;
     d.err = ws.err;
     d.epoch = r.epoch;
     // (the absent family's type is a placeholder: the draft's, one kernel variant)
@@ -432,6 +442,7 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   r.err = ws.err;
   r.epoch = next_epoch();
   r.work = full_q ? ws.work : nullptr;  // zeroed by the prep kernel
+  r.pre_eighths = 4;
   // the first kernel of the chain starts only after the caller's work is
   // complete: it reads the logits before its grid-dependency wait
   if ((e = launch_rowpass(r, full_q ? draft->dtype : target->dtype, target->dtype, s,
@@ -534,6 +545,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   r.err = ws.err;
   r.epoch = next_epoch();
   r.work = ws.work;       // zeroed by the alignment kernel
+  r.pre_eighths = pre_wait_eighths(batch);
   r.excl_late = ws.excl;  // written by the alignment kernel
   // programmatic dependent launch: target rows stream while the alignment runs
   // (unless stage events sit between the kernels)
@@ -699,6 +711,7 @@ tt_status tt_verify_sharded(const tt_batch* batch, const float* q_hat, const tt_
     r.target_cols = tcols;
     r.err = ws.err;
     r.epoch = a.epoch;
+    r.pre_eighths = 4;
     r.work = reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(ws.work) +
                                                    size_t(k) * kWorkShards * kWorkStride *
                                                        sizeof(unsigned long long));

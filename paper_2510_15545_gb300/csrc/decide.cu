@@ -251,7 +251,12 @@ struct DecShared {
 // stream: 256 threads, shared memory sized by the batch, and at most 56
 // registers, since registers come from each SM sub-partition's own file and one
 // that holds 7 row-pass warps (56 registers each) has room for 2 more such warps.
+// LPR lanes work on one row in the rows and coarse phases (a power of two from 2
+// to 16, at least the row's chunk count where that is below 16), so that short
+// rows do not leave most lanes of their group idle: 32 / LPR rows per warp.
+template <int LPR>
 __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
+  constexpr int G = 32 / LPR;  // row groups per warp
   extern __shared__ __align__(16) char dsm[];
   __shared__ DecShared sh;
   __shared__ int s_bad;
@@ -259,7 +264,7 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
   const DecSmem sm = dec_smem(dsm, MX, dec_kx(a), dec_nr(a));
 
   const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int half = lane >> 4, hl = lane & 15;
+  const int grp = lane / LPR, hl = lane % LPR;
   const bool want_draft = a.full_q || a.q_hat_in == nullptr;
   const bool q_from_logits = a.q_hat_in == nullptr && a.draft_probs == nullptr;
   const bool draft_rows = q_from_logits || a.full_q;  // draft normalisers needed
@@ -388,11 +393,11 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
       err1 = __ldcg(a.err + 1);
     }
     // ------ row normalisers: target rows 0..m, then the first row of each run
-    // of equal map entries (the copy rule reuses it); a half-warp per row
+    // of equal map entries (the copy rule reuses it); LPR lanes per row
     int nonfinite = 0;
     const int n_tasks = m + 1 + sh.nd;
-    for (int base = 2 * warp; base < n_tasks; base += 2 * kWarps) {
-      const int task = base + half;
+    for (int base = G * warp; base < n_tasks; base += G * kWarps) {
+      const int task = base + grp;
       const bool valid = task < n_tasks;
       const bool tgt = task <= m;
       int j = 0;
@@ -413,35 +418,36 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
       }
       const int nch = valid ? R->nch : 0;
       const Partial* part = R->part + row * R->nch;
-      const bool cached = nch <= 128;
-      Partial c8[8];
+      constexpr int kCache = LPR >= 8 ? 8 : 4;  // partials per lane held in registers
+      const bool cached = nch <= kCache * LPR;
+      Partial c8[kCache];
   #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int c = hl + 16 * i;
+      for (int i = 0; i < kCache; ++i) {
+        const int c = hl + LPR * i;
         c8[i] = (cached && c < nch) ? part[c] : Partial{-INFINITY, 0.f};
       }
       float lmx = -INFINITY;
       if (cached) {
   #pragma unroll
-        for (int i = 0; i < 8; ++i) lmx = fmaxf(lmx, c8[i].m);
+        for (int i = 0; i < kCache; ++i) lmx = fmaxf(lmx, c8[i].m);
       } else {
-        for (int c = hl; c < nch; c += 16) lmx = fmaxf(lmx, part[c].m);
+        for (int c = hl; c < nch; c += LPR) lmx = fmaxf(lmx, part[c].m);
       }
-      const float mx = group_max<16>(lmx);
+      const float mx = group_max<LPR>(lmx);
       F2 acc = {0.f, 0.f};
       if (mx != -INFINITY) {
         if (cached) {
   #pragma unroll
-          for (int i = 0; i < 8; ++i)
+          for (int i = 0; i < kCache; ++i)
             if (c8[i].m != -INFINITY) acc = f2_add(acc, F2{c8[i].s * ex2_approx(c8[i].m - mx), 0.f});
         } else {
-          for (int c = hl; c < nch; c += 16) {
+          for (int c = hl; c < nch; c += LPR) {
             const Partial q = part[c];
             if (q.m != -INFINITY) acc = f2_add(acc, F2{q.s * ex2_approx(q.m - mx), 0.f});
           }
         }
       }
-      const F2 Ssum = group_sum<16>(acc);
+      const F2 Ssum = group_sum<LPR>(acc);
       const float S = __fadd_rn(Ssum.hi, Ssum.lo);
       if (valid && hl == 0) {
         if (tgt) {
@@ -490,8 +496,8 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
     // accept test: one-hot q puts r_t = max(0, p_j - q_j) on t_j and p elsewhere
     // (the row itself when that residual has no mass, and for the bonus row m)
     if (!a.full_q) {
-      for (int base = 2 * warp; base <= m; base += 2 * kWarps) {
-        const int j0 = base + half;
+      for (int base = G * warp; base <= m; base += G * kWarps) {
+        const int j0 = base + grp;
         const bool valid = j0 <= m;
         const int j = valid ? j0 : m;
         const int64_t row = int64_t(t0) + b + j;
@@ -507,7 +513,7 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
         int chunk;
         F2 rel, Z;
         bool main_used;
-        coarse_pick<16>(base_mass, nch, lane, sm.u2[j], ct, rt, pj, chunk, rel, Z, main_used);
+        coarse_pick<LPR>(base_mass, nch, lane, sm.u2[j], ct, rt, pj, chunk, rel, Z, main_used);
         if (valid && hl == 0) {
           sm.cchunk[j] = chunk;
           sm.crel[j] = rel;
@@ -770,19 +776,38 @@ cudaError_t launch_pdl(K kernel, const DecideArgs& args, unsigned grid, unsigned
   return cudaLaunchKernelEx(&cfg, kernel, args);
 }
 
+template <int LPR>
+cudaError_t preload_decide_lpr() {
+  cudaFuncAttributes fa;
+  cudaError_t e;
+  if ((e = cudaFuncGetAttributes(&fa, decide_kernel<LPR>)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(decide_kernel<LPR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kDecSmemMax)) != cudaSuccess)
+    return e;
+  // the same shared-memory split as the row pass, so that CTAs of both fit on one SM
+  return cudaFuncSetAttribute(decide_kernel<LPR>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                              int(cudaSharedmemCarveoutMaxShared));
+}
+
+// Lanes per row of the decision kernel: the smallest power of two from 2 to 16
+// that covers the chunks of every row it normalises.
+int decide_lpr(const DecideArgs& a) {
+  const bool draft_rows = (a.q_hat_in == nullptr && a.draft_probs == nullptr) || a.full_q;
+  const int nch = draft_rows ? max(a.t.nch, a.d.nch) : a.t.nch;
+  int l = 2;
+  while (l < 16 && l < nch) l *= 2;
+  return l;
+}
+
 }  // namespace
 
 cudaError_t preload_decide() {
   cudaFuncAttributes fa;
   cudaError_t e;
-  if ((e = cudaFuncGetAttributes(&fa, decide_kernel)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(decide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kDecSmemMax)) != cudaSuccess)
-    return e;
-  // the same shared-memory split as the row pass, so that CTAs of both fit on one SM
-  if ((e = cudaFuncSetAttribute(decide_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                int(cudaSharedmemCarveoutMaxShared))) != cudaSuccess)
-    return e;
+  if ((e = preload_decide_lpr<2>()) != cudaSuccess) return e;
+  if ((e = preload_decide_lpr<4>()) != cudaSuccess) return e;
+  if ((e = preload_decide_lpr<8>()) != cudaSuccess) return e;
+  if ((e = preload_decide_lpr<16>()) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, transfer_kernel)) != cudaSuccess) return e;
   return cudaFuncGetAttributes(&fa, prep_kernel);
 }
@@ -796,7 +821,13 @@ cudaError_t launch_decide(const DecideArgs& args, cudaStream_t stream, bool pdl)
   DecideArgs a = args;
   // a warming pass is free only for CTAs that start beside the row pass
   if (!pdl || smem > size_t(kDecSmemBeside)) a.warm_ctas = 0;
-  return launch_pdl(decide_kernel, a, unsigned(a.B), kDecThreads, smem, stream, pdl);
+  switch (decide_lpr(a)) {
+    case 2: return launch_pdl(decide_kernel<2>, a, unsigned(a.B), kDecThreads, smem, stream, pdl);
+    case 4: return launch_pdl(decide_kernel<4>, a, unsigned(a.B), kDecThreads, smem, stream, pdl);
+    case 8: return launch_pdl(decide_kernel<8>, a, unsigned(a.B), kDecThreads, smem, stream, pdl);
+    default:
+      return launch_pdl(decide_kernel<16>, a, unsigned(a.B), kDecThreads, smem, stream, pdl);
+  }
 }
 
 cudaError_t launch_prep(const PrepArgs& args, cudaStream_t stream) {

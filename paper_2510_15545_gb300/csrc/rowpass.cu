@@ -122,22 +122,44 @@ __device__ __forceinline__ void grid_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
-// Scored column of target row r (-1 for a bonus row or an unusable entry):
-// request b owns rows target_off[b] + b .. target_off[b+1] + b.
-__device__ int target_excl(const RowPassArgs& a, int64_t r) {
+// The scored columns of target rows visited mostly in increasing order: the
+// request of the last row looked up is kept, so that the next row of the same
+// request, or the first row of the next request, needs no search. The
+// producer keeps it in shared memory, off its register budget.
+struct ExclCursor {
+  int b;           // request of the cached range (-1: none)
+  int t0;          // its first target position
+  int64_t r0, r1;  // its rows: r0 .. r1 (r1 is the bonus row)
+};
+
+__device__ __forceinline__ int excl_lookup(const RowPassArgs& a, ExclCursor* cur, int64_t r) {
   if (!a.target_off || a.B <= 0) return -1;
-  int lo = 0, hi = a.B - 1;
-  while (lo < hi) {  // largest b with target_off[b] + b <= r
-    const int mid = (lo + hi + 1) >> 1;
-    if (int64_t(a.target_off[mid]) + mid <= r) lo = mid;
-    else hi = mid - 1;
+  int b = cur->b;
+  if (!(b >= 0 && r >= cur->r0 && r <= cur->r1)) {
+    if (b >= 0 && r == cur->r1 + 1 && b + 1 < a.B) {
+      ++b;
+    } else {
+      int lo = 0, hi = a.B - 1;
+      while (lo < hi) {  // largest b with target_off[b] + b <= r
+        const int mid = (lo + hi + 1) >> 1;
+        if (int64_t(a.target_off[mid]) + mid <= r) lo = mid;
+        else hi = mid - 1;
+      }
+      b = lo;
+    }
+    const int t0 = a.target_off[b], t1 = a.target_off[b + 1];
+    if (t0 < 0 || t1 < t0 || t1 > a.n_target) {
+      cur->b = -1;
+      return -1;
+    }
+    cur->b = b;
+    cur->t0 = t0;
+    cur->r0 = int64_t(t0) + b;
+    cur->r1 = int64_t(t1) + b;
   }
-  const int b = lo;
-  const int t0 = a.target_off[b], t1 = a.target_off[b + 1];
-  if (t0 < 0 || t1 < t0 || t1 > a.n_target) return -1;
-  const int64_t j = r - (int64_t(t0) + b);
-  if (j < 0 || j >= t1 - t0) return -1;
-  const int c = a.target_cols[t0 + j];
+  const int64_t j = r - cur->r0;
+  if (j < 0 || j >= cur->r1 - cur->r0) return -1;  // the bonus row
+  const int c = a.target_cols[cur->t0 + j];
   return (c >= 0 && c < a.t.V) ? c : -1;
 }
 
@@ -522,6 +544,8 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       int it = 0;
       int64_t cached_row = -1, cached_drow = -1;
       int cached_excl = -1;
+      __shared__ ExclCursor cursor;
+      cursor.b = -1;
       bool cached_need = true;
       // Queues chunk `chunk` of row `row` (tgt: a target row, else a draft
       // row) on the next stage; false once a wait has run out.
@@ -540,7 +564,7 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
             cached_row = row;
             cached_excl = a.excl                ? a.excl[row]
                           : (late && a.excl_late) ? a.excl_late[row]
-                                                  : target_excl(a, row);
+                                                  : excl_lookup(a, &cursor, row);
           }
           const int ex = cached_excl - unit * cps * kChunk;
           d.excl = (cached_excl >= 0 && ex >= 0 && ex < cps * kChunk) ? ex : -1;
@@ -614,11 +638,12 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
         grid_launch_dependents();
         walk(false, d_lo, d_hi);
       } else {
-        // A fixed block of the first half of the target items, streamed while
-        // the alignment may still run; then batches of the rest (target items,
-        // then draft items) from the work counter, so that CTAs that started
-        // late or drew less bandwidth take fewer and all finish together.
-        const int64_t per = items_t / 2 / G;
+        // A fixed block of a.pre_eighths / 8 of the target items, streamed
+        // while the alignment may still run (target rows do not depend on
+        // it); then batches of the rest (target items, then draft items) from
+        // the work counter, so that CTAs that started late or drew less
+        // bandwidth take fewer and all finish together.
+        const int64_t per = items_t * a.pre_eighths / 8 / G;
         walk(true, g * per, (g + 1) * per);
         grid_dependency_wait();  // the counters, flags and scored columns are ready
         late = true;

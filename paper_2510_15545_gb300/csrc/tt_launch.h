@@ -67,6 +67,8 @@ struct RowPassArgs {
   // this one depends on and read only after the grid-dependency wait; NULL:
   // every item belongs to a fixed share.
   unsigned long long* work;
+  int32_t pre_eighths;       // with work: eighths of the target items streamed in fixed
+                             // blocks before the grid-dependency wait (1..7)
   int32_t stall_stage;       // test hook (-1 = off): in CTA 0 the stage consumed at
                              // consumer step stall_stage is never freed, so the
                              // bounded waits run out
