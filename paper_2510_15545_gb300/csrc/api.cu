@@ -320,6 +320,7 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
 
   DecideArgs d;
   std::memset(&d, 0, sizeof d);
+  d.sm_count = sm_count_current();
   d.B = batch->B;
   d.n_draft = batch->n_draft;
   d.n_target = batch->n_target;
@@ -451,6 +452,7 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
 
   DecideArgs d;
   std::memset(&d, 0, sizeof d);
+  d.sm_count = sm_count_current();
   d.B = batch->B;
   d.n_draft = batch->n_draft;
   d.n_target = batch->n_target;
@@ -557,6 +559,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
 
   DecideArgs d;
   std::memset(&d, 0, sizeof d);
+  d.sm_count = sm_count_current();
   d.B = batch->B;
   d.n_draft = batch->n_draft;
   d.n_target = batch->n_target;

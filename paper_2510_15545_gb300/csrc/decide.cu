@@ -2,7 +2,8 @@
 // accept loop, Alg. 4 residual) and the standalone transfer (Alg. 2
 // MapProbabilities, App. A.2).
 //
-// One CTA per request. From the row-pass partials it rebuilds the
+// One CTA per request (256 threads, or 128 when the batch has more requests
+// than fit on the GPU at once). From the row-pass partials it rebuilds the
 // log2-normaliser of each of the m+1 target rows (adding back the scored
 // token's term) and of each mapped draft row, giving p(t_j) and the
 // transferred q(t_j); fp32 with compensated sums and exactly split exponents,
@@ -20,8 +21,8 @@ namespace tt {
 
 namespace {
 
-constexpr int kDecThreads = 256;
-constexpr int kWarps = kDecThreads / 32;
+constexpr int kDecThreads = 256;            // threads of the transfer kernel, most of a decision CTA
+constexpr int kWarps = kDecThreads / 32;  // most warps of a decision CTA
 constexpr int kDecSmemMax = 64 * 1024;  // largest dynamic shared memory of a decision CTA
 // Dynamic shared memory up to which a decision CTA fits beside three row-pass
 // CTAs on one SM (3 x 66 KB of the 228 KB, less per-CTA reservations).
@@ -239,24 +240,27 @@ struct DecShared {
   int a, pick, last, nd, err;
 };
 
-// One CTA (8 warps) per request.
+// One CTA of NT threads (256, or 128 for batches larger than the GPU holds at
+// once) per request.
 //  before the grid-dependency wait: checks of the caller's inputs, the map,
 //  the scored logits and both uniforms of every position;
-//  after it: one half-warp per row rebuilds the normaliser of
-//  each target row and each mapped draft row from the row-pass partials; the
-//  accept test and, for every candidate row, the coarse level of its residual
-//  (one half-warp per row) run side by side; the whole CTA then re-reads the
-//  chosen chunk of the accepted row (fine level).
+//  after it: LPR lanes per row rebuild the normaliser of each target row and
+//  each mapped draft row from the row-pass partials; the accept test and, for
+//  every candidate row, the coarse level of its residual (LPR lanes per row)
+//  run side by side; the whole CTA then re-reads the chosen chunk of the
+//  accepted row (fine level).
+// LPR is a power of two from 2 to 16, at least the row's chunk count where that
+// is below 16, so that short rows do not leave most lanes of their group idle:
+// 32 / LPR rows per warp.
 // Small enough to sit beside the row pass's CTAs, so it starts while they
-// stream: 256 threads, shared memory sized by the batch, and at most 56
-// registers, since registers come from each SM sub-partition's own file and one
-// that holds 7 row-pass warps (56 registers each) has room for 2 more such warps.
-// LPR lanes work on one row in the rows and coarse phases (a power of two from 2
-// to 16, at least the row's chunk count where that is below 16), so that short
-// rows do not leave most lanes of their group idle: 32 / LPR rows per warp.
-template <int LPR>
+// stream: shared memory sized by the batch, and at most 56 registers, since
+// registers come from each SM sub-partition's own file and one that holds 7
+// row-pass warps (56 registers each) has room for 2 more such warps.
+template <int NT, int LPR>
 __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
+  constexpr int NW = NT / 32;  // warps of the CTA
   constexpr int G = 32 / LPR;  // row groups per warp
+  static_assert(NW <= kWarps, "shared scan buffers hold kWarps warps");
   extern __shared__ __align__(16) char dsm[];
   __shared__ DecShared sh;
   __shared__ int s_bad;
@@ -300,7 +304,7 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
   // are read through L2 only).
   int bad = 0;
   if (st == 0) {
-    for (int j = tid; j < m; j += kDecThreads) {
+    for (int j = tid; j < m; j += NT) {
       const int col = a.target_cols[t0 + j];
       sm.col[j] = col;
       if (col < 0 || col >= a.t.V) bad |= 1;
@@ -312,7 +316,7 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
       sm.map[j] = i;
     }
     if (q_from_logits)
-      for (int i = tid; i < k; i += kDecThreads) {
+      for (int i = tid; i < k; i += NT) {
         const int col = a.draft_cols[d0 + i];
         sm.dcol[i] = col;
         if (col < 0 || col >= a.d.V) bad |= 1;
@@ -330,7 +334,7 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
 
   const uint64_t req = a.request_base + uint64_t(b);
   if (st == 0) {
-    for (int j = tid; j <= m; j += kDecThreads) {
+    for (int j = tid; j <= m; j += NT) {
       sm.u2[j] = float(philox_uniform(a.seed, uint64_t(j), 1, req));
       if (j == m) continue;
       int f = j;  // first position of this run of equal map entries
@@ -396,7 +400,7 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
     // of equal map entries (the copy rule reuses it); LPR lanes per row
     int nonfinite = 0;
     const int n_tasks = m + 1 + sh.nd;
-    for (int base = G * warp; base < n_tasks; base += G * kWarps) {
+    for (int base = G * warp; base < n_tasks; base += G * NW) {
       const int task = base + grp;
       const bool valid = task < n_tasks;
       const bool tgt = task <= m;
@@ -483,7 +487,7 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
     }
 
     // --------------------------- accept while u_j q_j < p_j (u < 1 exactly)
-    for (int j = tid; j < m; j += kDecThreads) {
+    for (int j = tid; j < m; j += NT) {
       const float qh = sm.q[sm.qi[j]];
       if (a.q_hat_out && !dry) a.q_hat_out[t0 + j] = qh;
       if (!(sm.u[j] * qh < sm.p[j])) atomicMin(&sh.a, j);
@@ -496,7 +500,7 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
     // accept test: one-hot q puts r_t = max(0, p_j - q_j) on t_j and p elsewhere
     // (the row itself when that residual has no mass, and for the bonus row m)
     if (!a.full_q) {
-      for (int base = G * warp; base <= m; base += G * kWarps) {
+      for (int base = G * warp; base <= m; base += G * NW) {
         const int j0 = base + grp;
         const bool valid = j0 <= m;
         const int j = valid ? j0 : m;
@@ -552,7 +556,7 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
       const Partial* part = a.t.part + row * nch;
       int md = acc < m ? 2 : 0;
       if (md == 2) {
-        for (int c = warp; c < nch; c += kWarps) {
+        for (int c = warp; c < nch; c += NW) {
           F2 acc2 = {0.f, 0.f};
           const int hi_c = min(V, (c + 1) * kChunk);
           for (int x = c * kChunk + lane; x < hi_c; x += 32)
@@ -590,87 +594,98 @@ __global__ void __maxnreg__(56) decide_kernel(DecideArgs a) {
     const F2 rel = sm.crel[acc];
     const int mode = sm.cmode[acc];
 
-    // ------------------------------------------ fine level: one chunk re-read
-    constexpr int kPer = kChunk / kDecThreads;  // 8 consecutive columns per thread
-    const int x0 = chunk * kChunk + tid * kPer;
-    float r[kPer];
-    if (x0 + kPer <= V) {
-      if (a.dt_t == TT_F32) {
-        const float4 w0 = __ldg(reinterpret_cast<const float4*>(trow + size_t(x0) * 4));
-        const float4 w1 = __ldg(reinterpret_cast<const float4*>(trow + size_t(x0) * 4 + 16));
-        r[0] = w0.x;
-        r[1] = w0.y;
-        r[2] = w0.z;
-        r[3] = w0.w;
-        r[4] = w1.x;
-        r[5] = w1.y;
-        r[6] = w1.z;
-        r[7] = w1.w;
+    // ------------------------------------------ fine level: one chunk re-read,
+    // in slabs of NT x 8 consecutive columns (8 per thread) taken in column
+    // order; each slab is scanned as a block prefix in pairs, and the draw
+    // minus the mass of the slabs before it is looked for in the next one
+    constexpr int kPer = 8;
+    constexpr int kSlabs = kChunk / (NT * kPer);
+    F2 rel_s = rel;  // the draw relative to the current slab's start
+#pragma unroll 1
+    for (int slab = 0; slab < kSlabs; ++slab) {
+      const int x0 = chunk * kChunk + slab * NT * kPer + tid * kPer;
+      float r[kPer];
+      if (x0 + kPer <= V) {
+        if (a.dt_t == TT_F32) {
+          const float4 w0 = __ldg(reinterpret_cast<const float4*>(trow + size_t(x0) * 4));
+          const float4 w1 = __ldg(reinterpret_cast<const float4*>(trow + size_t(x0) * 4 + 16));
+          r[0] = w0.x;
+          r[1] = w0.y;
+          r[2] = w0.z;
+          r[3] = w0.w;
+          r[4] = w1.x;
+          r[5] = w1.y;
+          r[6] = w1.z;
+          r[7] = w1.w;
+        } else {
+          const uint4 w = __ldg(reinterpret_cast<const uint4*>(trow + size_t(x0) * 2));
+          const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+    #pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            r[2 * q] = __uint_as_float(ww[q] << 16);
+            r[2 * q + 1] = __uint_as_float(ww[q] & 0xffff0000u);
+          }
+        }
       } else {
-        const uint4 w = __ldg(reinterpret_cast<const uint4*>(trow + size_t(x0) * 2));
-        const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-  #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          r[2 * q] = __uint_as_float(ww[q] << 16);
-          r[2 * q + 1] = __uint_as_float(ww[q] & 0xffff0000u);
-        }
+    #pragma unroll
+        for (int q = 0; q < kPer; ++q) r[q] = x0 + q < V ? load_dt(trow, a.dt_t, x0 + q) : 0.f;
       }
-    } else {
-  #pragma unroll
-      for (int q = 0; q < kPer; ++q) r[q] = x0 + q < V ? load_dt(trow, a.dt_t, x0 + q) : 0.f;
-    }
-    F2 run = {0.f, 0.f};
-    int last_pos = -1;
-  #pragma unroll
-    for (int q = 0; q < kPer; ++q) {
-      const int x = x0 + q;
-      const float v = x < V ? r_of(x, r[q], mode) : 0.f;
-      if (v > 0.f) last_pos = x;
-      r[q] = v;
-      run = f2_add(run, F2{v, 0.f});
-    }
-    // block prefix in pairs: scan within each warp, warp totals scanned by
-    // warp 0; a warp's last interval ends where the next warp's first begins
-    F2 incl = run;
-  #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const F2 n = shfl_up_f2(incl, o, 32);
-      if (lane >= o) incl = f2_add(n, incl);
-    }
-    const F2 prev = shfl_up_f2(incl, 1, 32);
-    F2 excl = lane == 0 ? F2{0.f, 0.f} : prev;
-    if (lane == 31) sh.wtot[warp] = incl;
-    __syncthreads();
-    if (warp == 0) {
-      const F2 t = lane < kWarps ? sh.wtot[lane] : F2{0.f, 0.f};
-      F2 wi = t;
-  #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const F2 n = shfl_up_f2(wi, o, 32);
-        if (lane >= o) wi = f2_add(n, wi);
-      }
-      const F2 wp = shfl_up_f2(wi, 1, 32);
-      if (lane <= kWarps) sh.wpre[lane] = lane == 0 ? F2{0.f, 0.f} : wp;
-    }
-    __syncthreads();
-    const F2 base = sh.wpre[warp];
-    incl = lane == 31 ? sh.wpre[warp + 1] : f2_add(base, incl);
-    excl = f2_add(base, excl);
-    if (f2_le(excl, rel) && f2_lt(rel, incl)) {
-      F2 c = excl;
-      int pick = last_pos;
-  #pragma unroll
+      F2 run = {0.f, 0.f};
+      int last_pos = -1;
+    #pragma unroll
       for (int q = 0; q < kPer; ++q) {
-        c = f2_add(c, F2{r[q], 0.f});
-        if (r[q] > 0.f && f2_lt(rel, c)) {
-          pick = x0 + q;
-          break;
-        }
+        const int x = x0 + q;
+        const float v = x < V ? r_of(x, r[q], mode) : 0.f;
+        if (v > 0.f) last_pos = x;
+        r[q] = v;
+        run = f2_add(run, F2{v, 0.f});
       }
-      atomicMax(&sh.pick, pick);
+      // block prefix in pairs: scan within each warp, warp totals scanned by
+      // warp 0; a warp's last interval ends where the next warp's first begins
+      F2 incl = run;
+    #pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const F2 n = shfl_up_f2(incl, o, 32);
+        if (lane >= o) incl = f2_add(n, incl);
+      }
+      const F2 prev = shfl_up_f2(incl, 1, 32);
+      F2 excl = lane == 0 ? F2{0.f, 0.f} : prev;
+      if (lane == 31) sh.wtot[warp] = incl;
+      __syncthreads();
+      if (warp == 0) {
+        const F2 t = lane < NW ? sh.wtot[lane] : F2{0.f, 0.f};
+        F2 wi = t;
+    #pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const F2 n = shfl_up_f2(wi, o, 32);
+          if (lane >= o) wi = f2_add(n, wi);
+        }
+        const F2 wp = shfl_up_f2(wi, 1, 32);
+        if (lane <= NW) sh.wpre[lane] = lane == 0 ? F2{0.f, 0.f} : wp;
+      }
+      __syncthreads();
+      const F2 base = sh.wpre[warp];
+      const F2 slab_total = sh.wpre[NW];
+      incl = lane == 31 ? sh.wpre[warp + 1] : f2_add(base, incl);
+      excl = f2_add(base, excl);
+      if (f2_le(excl, rel_s) && f2_lt(rel_s, incl)) {
+        F2 c = excl;
+        int pick = last_pos;
+    #pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+          c = f2_add(c, F2{r[q], 0.f});
+          if (r[q] > 0.f && f2_lt(rel_s, c)) {
+            pick = x0 + q;
+            break;
+          }
+        }
+        atomicMax(&sh.pick, pick);
+      }
+      if (last_pos >= 0) atomicMax(&sh.last, last_pos);
+      __syncthreads();
+      if (sh.pick >= 0) break;  // the same for every thread (read past the barrier)
+      rel_s = f2_add(rel_s, f2_neg(slab_total));
     }
-    if (last_pos >= 0) atomicMax(&sh.last, last_pos);
-    __syncthreads();
     if (tid == 0 && !dry) {
       a.accepted[b] = acc;
       a.next_token[b] = sh.pick >= 0 ? sh.pick : sh.last;
@@ -776,19 +791,6 @@ cudaError_t launch_pdl(K kernel, const DecideArgs& args, unsigned grid, unsigned
   return cudaLaunchKernelEx(&cfg, kernel, args);
 }
 
-template <int LPR>
-cudaError_t preload_decide_lpr() {
-  cudaFuncAttributes fa;
-  cudaError_t e;
-  if ((e = cudaFuncGetAttributes(&fa, decide_kernel<LPR>)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(decide_kernel<LPR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kDecSmemMax)) != cudaSuccess)
-    return e;
-  // the same shared-memory split as the row pass, so that CTAs of both fit on one SM
-  return cudaFuncSetAttribute(decide_kernel<LPR>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                              int(cudaSharedmemCarveoutMaxShared));
-}
-
 // Lanes per row of the decision kernel: the smallest power of two from 2 to 16
 // that covers the chunks of every row it normalises.
 int decide_lpr(const DecideArgs& a) {
@@ -799,15 +801,47 @@ int decide_lpr(const DecideArgs& a) {
   return l;
 }
 
+template <int NT, int LPR>
+cudaError_t preload_decide_variant() {
+  cudaFuncAttributes fa;
+  cudaError_t e;
+  if ((e = cudaFuncGetAttributes(&fa, decide_kernel<NT, LPR>)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(decide_kernel<NT, LPR>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, kDecSmemMax)) !=
+      cudaSuccess)
+    return e;
+  // the same shared-memory split as the row pass, so that CTAs of both fit on one SM
+  return cudaFuncSetAttribute(decide_kernel<NT, LPR>,
+                              cudaFuncAttributePreferredSharedMemoryCarveout,
+                              int(cudaSharedmemCarveoutMaxShared));
+}
+
+template <int NT>
+cudaError_t preload_decide_nt() {
+  cudaError_t e;
+  if ((e = preload_decide_variant<NT, 2>()) != cudaSuccess) return e;
+  if ((e = preload_decide_variant<NT, 4>()) != cudaSuccess) return e;
+  if ((e = preload_decide_variant<NT, 8>()) != cudaSuccess) return e;
+  return preload_decide_variant<NT, 16>();
+}
+
+template <int NT>
+cudaError_t launch_decide_nt(const DecideArgs& a, size_t smem, cudaStream_t stream, bool pdl) {
+  switch (decide_lpr(a)) {
+    case 2: return launch_pdl(decide_kernel<NT, 2>, a, unsigned(a.B), NT, smem, stream, pdl);
+    case 4: return launch_pdl(decide_kernel<NT, 4>, a, unsigned(a.B), NT, smem, stream, pdl);
+    case 8: return launch_pdl(decide_kernel<NT, 8>, a, unsigned(a.B), NT, smem, stream, pdl);
+    default: return launch_pdl(decide_kernel<NT, 16>, a, unsigned(a.B), NT, smem, stream, pdl);
+  }
+}
+
 }  // namespace
 
 cudaError_t preload_decide() {
   cudaFuncAttributes fa;
   cudaError_t e;
-  if ((e = preload_decide_lpr<2>()) != cudaSuccess) return e;
-  if ((e = preload_decide_lpr<4>()) != cudaSuccess) return e;
-  if ((e = preload_decide_lpr<8>()) != cudaSuccess) return e;
-  if ((e = preload_decide_lpr<16>()) != cudaSuccess) return e;
+  if ((e = preload_decide_nt<128>()) != cudaSuccess) return e;
+  if ((e = preload_decide_nt<256>()) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, transfer_kernel)) != cudaSuccess) return e;
   return cudaFuncGetAttributes(&fa, prep_kernel);
 }
@@ -821,13 +855,11 @@ cudaError_t launch_decide(const DecideArgs& args, cudaStream_t stream, bool pdl)
   DecideArgs a = args;
   // a warming pass is free only for CTAs that start beside the row pass
   if (!pdl || smem > size_t(kDecSmemBeside)) a.warm_ctas = 0;
-  switch (decide_lpr(a)) {
-    case 2: return launch_pdl(decide_kernel<2>, a, unsigned(a.B), kDecThreads, smem, stream, pdl);
-    case 4: return launch_pdl(decide_kernel<4>, a, unsigned(a.B), kDecThreads, smem, stream, pdl);
-    case 8: return launch_pdl(decide_kernel<8>, a, unsigned(a.B), kDecThreads, smem, stream, pdl);
-    default:
-      return launch_pdl(decide_kernel<16>, a, unsigned(a.B), kDecThreads, smem, stream, pdl);
-  }
+  // 256 threads while the batch's CTAs all fit on the GPU at once (four per
+  // SM: 56 registers x 256 threads), else 128 (nine per SM), which keeps more
+  // requests in flight and fewer threads waiting at the CTA's barriers
+  if (int64_t(a.B) > int64_t(4) * a.sm_count) return launch_decide_nt<128>(a, smem, stream, pdl);
+  return launch_decide_nt<256>(a, smem, stream, pdl);
 }
 
 cudaError_t launch_prep(const PrepArgs& args, cudaStream_t stream) {

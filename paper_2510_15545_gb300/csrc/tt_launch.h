@@ -97,6 +97,7 @@ struct DecideArgs {
   float* p_hat;
   float* lse;
   int warm_ctas;  // CTAs b < warm_ctas run a warming pass before the wait (see decide.cu)
+  int sm_count;   // SMs of the device (sizes the decision kernel's CTAs)
   float top_p_d, top_p_t;    // top-p of filtered families (d.top_k / t.top_k > 0)
   const int32_t* status_q;   // status of the kernel that produced q_hat_in, or NULL
   const Cand* kept_d;        // kept sets of filtered families (written by the kept kernel)
