@@ -58,7 +58,8 @@ def parse_args(argv=None):
     ap.add_argument("--top-k", type=int, default=0,
                     help="top-k filter of draft and target rows (0 = off)")
     ap.add_argument("--top-p", type=float, default=1.0,
-                    help="top-p filter after the top-k (1 = off)")
+                    help="top-p filter (after the top-k when --top-k is set; over the whole row "
+                         "when it is not; 1 = off)")
     ap.add_argument("--shards", type=int, default=0,
                     help="also time the vocabulary-sharded verification with the target "
                          "rows split into this many column slices (1-8), against the "
@@ -243,6 +244,17 @@ def algorithmic_bytes(wl, mp) -> dict:
 def default_steps(name: str) -> int:
     return {"b1_g4_v32k": 20000, "b64_g8_v152k": 20000, "b256_g16_v152k_bf16": 3000,
             "dtw_4096x64": 1000, "b1024_g8_v201k_bf16": 1000}.get(name, 1000)
+
+
+def step_launches(args) -> int:
+    """Kernels one tt_step launches: alignment, row pass and decision; with
+    filters also the kept sets of top-k families, the nucleus kernel of
+    top-p-only families and the transfer of q_hat before the decision."""
+    if args.top_k > 0:
+        return 5
+    if args.top_p < 1.0:
+        return 5
+    return 3
 
 
 def step_kwargs(args) -> dict:
@@ -490,7 +502,7 @@ def run_mine(args):
     Wm = max(3, args.warmup)
     stream = torch.cuda.current_stream(dev)
     wl, inp, prm, full, call = prepare_step(tt, W, name, args, rank, dev, stream)
-    filtered = args.top_k > 0
+    filtered = args.top_k > 0 or args.top_p < 1.0
     dl, tl = inp["draft_logits"], inp["target_logits"]
     mp = full["map"].cpu().numpy()
     acc = full["accepted"].cpu().numpy()
@@ -578,7 +590,7 @@ def run_mine(args):
                      "peak_kind": "%s copy bandwidth (hbm_gbs)" % peak_kind,
                      "traffic": traffic, "algorithmic_bytes": ab["total"],
                      "vs_nominal_8tbs": achieved / 8000.0},
-        "gpu_launches": (5 if filtered else 3) * K,
+        "gpu_launches": step_launches(args) * K,
         "clocks": clk,
     }
     if e2e is not None:

@@ -38,6 +38,7 @@ cudaError_t ensure_loaded() {
   if ((e = preload_rowpass()) != cudaSuccess) return e;
   if ((e = preload_decide()) != cudaSuccess) return e;
   if ((e = preload_filter()) != cudaSuccess) return e;
+  if ((e = preload_nucleus()) != cudaSuccess) return e;
   if ((e = preload_shard()) != cudaSuccess) return e;
   if (dev >= 0 && dev < 64) done[dev].store(true, std::memory_order_release);
   return cudaSuccess;
@@ -92,16 +93,11 @@ bool params_ok(const tt_params* p) {
   return true;
 }
 
-// Filters the kernels take: top-p only after a top-k (a nucleus over the whole
-// vocabulary is not built).
-bool filters_supported(const tt_params* p) {
-  if (p->top_p_draft < 1.f && p->top_k_draft == 0) return false;
-  if (p->top_p_target < 1.f && p->top_k_target == 0) return false;
-  return true;
-}
-
 int k_draft(const tt_params* p) { return p->top_k_draft; }
 int k_target(const tt_params* p) { return p->top_k_target; }
+// Nucleus families: top-p without top-k (a kept set over the whole row).
+bool nuc_draft(const tt_params* p) { return p->top_k_draft == 0 && p->top_p_draft < 1.f; }
+bool nuc_target(const tt_params* p) { return p->top_k_target == 0 && p->top_p_target < 1.f; }
 
 // Shards usable by tt_verify_sharded: 1..TT_MAX_SHARDS logits arrays of
 // rows_needed rows that tile the row in order from column 0; V = the row width.
@@ -143,6 +139,7 @@ RowSet rowset(const tt_logits* L, Partial* part, const uint8_t* need, float T) {
   r.top_k = 0;
   r.cand = nullptr;
   r.nlist = L->dtype == TT_F32 ? r.nch : (r.nch + 1) / 2;
+  r.nucleus = 0;
   return r;
 }
 
@@ -173,11 +170,39 @@ cudaError_t launch_kept_sets(const RowSet& d, int64_t rows_d, const RowSet& t, i
   return launch_kept(k, s, sm_count_current(), pdl);
 }
 
+// Kept sets of the nucleus families among d and t (top-p without top-k).
+cudaError_t launch_nucleus_sets(const RowSet& d, int64_t rows_d, const RowSet& t, int64_t rows_t,
+                                const tt_params* prm, const Workspace& ws, int dt_d, int dt_t,
+                                const tt_batch* batch, const int32_t* tcols, cudaStream_t s,
+                                bool pdl) {
+  KeptArgs k;
+  std::memset(&k, 0, sizeof k);
+  k.d = d;
+  k.t = t;
+  k.rows_d = d.nucleus ? rows_d : 0;
+  k.rows_t = t.nucleus ? rows_t : 0;
+  k.top_p_d = prm->top_p_draft;
+  k.top_p_t = prm->top_p_target;
+  k.head_d = ws.head_d;
+  k.head_t = ws.head_t;
+  k.um_d = ws.um_d;
+  k.um_t = ws.um_t;
+  k.dt_d = dt_d;
+  k.dt_t = dt_t;
+  k.B = batch->B;
+  k.n_target = batch->n_target;
+  k.target_off = batch->target_off;
+  k.target_cols = tcols;
+  return launch_nucleus(k, s, sm_count_current(), pdl);
+}
+
 void attach_kept(DecideArgs& d, const Workspace& ws) {
   d.kept_d = ws.kept_d;
   d.kept_t = ws.kept_t;
   d.head_d = ws.head_d;
   d.head_t = ws.head_t;
+  d.um_d = ws.um_d;
+  d.um_t = ws.um_t;
 }
 
 // Share of the target rows the step's row pass streams before it waits for
@@ -242,15 +267,16 @@ tt_status step_check(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* 
   if (!logits_ok(target, int64_t(batch->n_target) + batch->B)) return TT_ERR_INVALID_ARG;
   if (from_logits && !logits_ok(draft, batch->n_draft)) return TT_ERR_INVALID_ARG;
   if (full_q && draft->n_cols != target->n_cols) return TT_ERR_INVALID_ARG;
-  if (!filters_supported(prm)) return TT_ERR_UNSUPPORTED;
   // given draft probabilities are taken as they are (no draft filter)
   const int kd = from_logits ? k_draft(prm) : 0, kt = k_target(prm);
-  if (full_q && (kd > 0) != (kt > 0)) return TT_ERR_UNSUPPORTED;
+  const bool nd = from_logits && nuc_draft(prm), nt = nuc_target(prm);
+  // full-q: both families filtered or neither, and no nucleus family
+  if (full_q && ((kd > 0 || nd) != (kt > 0 || nt) || nd || nt)) return TT_ERR_UNSUPPORTED;
   AlignArgs a;
   const tt_status st = fill_align_args(batch, vd, vt, prm, a);
   if (st != TT_OK) return st;
   *need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target,
-                           from_logits ? draft->n_cols : 0, target->n_cols, kd, kt)
+                           from_logits ? draft->n_cols : 0, target->n_cols, kd, kt, nd, nt)
               .bytes;
   return TT_OK;
 }
@@ -263,8 +289,9 @@ size_t tt_workspace_bytes_for(const tt_batch* batch, int32_t V_d, int32_t V_t,
   if (!batch || batch->B < 0 || batch->n_draft < 0 || batch->n_target < 0) return 0;
   const int kd = prm ? prm->top_k_draft : 0, kt = prm ? prm->top_k_target : 0;
   if (kd < 0 || kd > TT_MAX_TOP_K || kt < 0 || kt > TT_MAX_TOP_K) return 0;
+  const bool nd = prm && nuc_draft(prm), nt = prm && nuc_target(prm);
   return workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d < 0 ? 0 : V_d,
-                          V_t < 0 ? 0 : V_t, kd, kt)
+                          V_t < 0 ? 0 : V_t, kd, kt, nd, nt)
       .bytes;
 }
 
@@ -306,17 +333,18 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   if (from_logits && !logits_ok(draft, batch->n_draft)) return TT_ERR_INVALID_ARG;
   const int32_t* cols = batch->draft_cols ? batch->draft_cols : batch->draft_ids;
   if (from_logits && batch->n_draft > 0 && !cols) return TT_ERR_INVALID_ARG;
-  if (!filters_supported(prm)) return TT_ERR_UNSUPPORTED;
   const int kd = from_logits ? k_draft(prm) : 0;  // given probabilities are taken as they are
+  const bool nd = from_logits && nuc_draft(prm);
   const int V_d = from_logits ? draft->n_cols : 0;
-  const size_t need =
-      workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d, 0, kd, 0).bytes;
+  const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d,
+                                       0, kd, 0, nd, false)
+                          .bytes;
   if (from_logits && (!workspace || workspace_bytes < need ||
                       (reinterpret_cast<uintptr_t>(workspace) & 255) != 0))
     return TT_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  Workspace ws =
-      workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d, 0, kd, 0);
+  Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d, 0,
+                                  kd, 0, nd, false);
 
   DecideArgs d;
   std::memset(&d, 0, sizeof d);
@@ -335,6 +363,7 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   d.d = from_logits ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
   d.d.top_k = kd;
   d.d.cand = ws.cand_d;
+  d.d.nucleus = nd ? 1 : 0;
   d.top_p_d = prm->top_p_draft;
   d.t = no_rows();
   d.dt_d = from_logits ? draft->dtype : TT_F32;
@@ -371,9 +400,13 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
         cudaSuccess)
       return cuda_fail(e);
   }
-  if (kd > 0) {
+  if (kd > 0 || nd) {
     attach_kept(d, ws);
-    if ((e = launch_kept_sets(d.d, batch->n_draft, no_rows(), 0, prm, ws, s, true)) != cudaSuccess)
+    if (kd > 0 &&
+        (e = launch_kept_sets(d.d, batch->n_draft, no_rows(), 0, prm, ws, s, true)) != cudaSuccess)
+      return cuda_fail(e);
+    if (nd && (e = launch_nucleus_sets(d.d, batch->n_draft, no_rows(), 0, prm, ws, draft->dtype,
+                                       draft->dtype, batch, nullptr, s, true)) != cudaSuccess)
       return cuda_fail(e);
     if ((e = launch_filter_q(d, s, true)) != cudaSuccess) return cuda_fail(e);
   } else if ((e = launch_decide(d, s, from_logits)) != cudaSuccess) {
@@ -399,18 +432,19 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
     if (!logits_ok(draft, batch->n_draft) || draft->n_cols != target->n_cols) return TT_ERR_INVALID_ARG;
     if (batch->n_target > 0 && !map) return TT_ERR_INVALID_ARG;
   }
-  if (!filters_supported(prm)) return TT_ERR_UNSUPPORTED;
   // q_hat is given; the draft rows' filter matters only to the full-q residual
   const int kt = k_target(prm), kd = full_q ? k_draft(prm) : 0;
-  if (full_q && (kd > 0) != (kt > 0)) return TT_ERR_UNSUPPORTED;
+  const bool nt = nuc_target(prm), nd = full_q && nuc_draft(prm);
+  // full-q: both families filtered or neither, and no nucleus family
+  if (full_q && ((kd > 0 || nd) != (kt > 0 || nt) || nd || nt)) return TT_ERR_UNSUPPORTED;
   const int V_d = full_q ? draft->n_cols : 0;
   const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d,
-                                       target->n_cols, kd, kt).bytes;
+                                       target->n_cols, kd, kt, false, nt).bytes;
   if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
     return TT_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d,
-                                  target->n_cols, kd, kt);
+                                  target->n_cols, kd, kt, false, nt);
   cudaError_t e = ensure_loaded();
   if (e != cudaSuccess) return cuda_fail(e);
   if (full_q) {  // the residual needs the mapped draft rows' normalisers
@@ -431,6 +465,7 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   r.t = rowset(target, ws.part_t, nullptr, prm->temp_target);
   r.t.top_k = kt;
   r.t.cand = ws.cand_t;
+  r.t.nucleus = nt ? 1 : 0;
   r.rows_t = int64_t(batch->n_target) + batch->B;
   r.d = full_q ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
   r.d.top_k = kd;
@@ -484,6 +519,12 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
     if ((e = launch_kept_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, s, true)) != cudaSuccess)
       return cuda_fail(e);
     if ((e = launch_decide_filtered(d, s, true)) != cudaSuccess) return cuda_fail(e);
+  } else if (nt) {
+    attach_kept(d, ws);
+    if ((e = launch_nucleus_sets(no_rows(), 0, r.t, r.rows_t, prm, ws, target->dtype,
+                                 target->dtype, batch, tcols, s, true)) != cudaSuccess)
+      return cuda_fail(e);
+    if ((e = launch_decide_nucleus(d, s, true)) != cudaSuccess) return cuda_fail(e);
   } else if ((e = launch_decide(d, s, true)) != cudaSuccess) {
     return cuda_fail(e);
   }
@@ -502,7 +543,8 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   const bool full_q = prm->full_q != 0;
   const bool from_logits = draft_probs == nullptr || full_q;
   const int kd = from_logits ? k_draft(prm) : 0, kt = k_target(prm);
-  const bool filtered = kd > 0 || kt > 0;
+  const bool nd = from_logits && nuc_draft(prm), nt = nuc_target(prm);
+  const bool filtered = kd > 0 || kt > 0 || nd || nt;
   const int V_d = from_logits ? draft->n_cols : 0;
   const int32_t* dcols = batch->draft_cols ? batch->draft_cols : batch->draft_ids;
   const int32_t* tcols = batch->target_cols ? batch->target_cols : batch->target_ids;
@@ -512,7 +554,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d,
-                                  target->n_cols, kd, kt);
+                                  target->n_cols, kd, kt, nd, nt);
   int32_t* map = out->map ? out->map : ws.map;
   a.path = out->path;
   a.path_len = out->path_len;
@@ -538,8 +580,10 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   r.rows_d = from_logits ? batch->n_draft : 0;
   r.t.top_k = kt;
   r.t.cand = ws.cand_t;
+  r.t.nucleus = nt ? 1 : 0;
   r.d.top_k = kd;
   r.d.cand = ws.cand_d;
+  r.d.nucleus = nd ? 1 : 0;
   r.B = batch->B;
   r.n_target = batch->n_target;
   r.target_off = batch->target_off;
@@ -596,19 +640,25 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
     record(prm, 3, s);
     return TT_OK;
   }
-  // Filtered: q_hat first (from the draft rows' top-k lists, or as without
-  // filters), into out->q_hat or the workspace with its own status; then the
-  // decision over the target rows (their top-k lists, or the partials).
+  // Filtered: the kept sets (top-k families from their lists, nucleus families
+  // from their partials and logits); q_hat (from the draft rows' kept sets, or
+  // as without filters), into out->q_hat or the workspace with its own status;
+  // then the decision over the target rows (their kept sets, or the partials).
   float* qbuf = out->q_hat ? out->q_hat : ws.q_hat;
   attach_kept(d, ws);
-  if ((e = launch_kept_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, s, pdl)) != cudaSuccess)
+  if ((kd > 0 || kt > 0) &&
+      (e = launch_kept_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, s, pdl)) != cudaSuccess)
+    return cuda_fail(e);
+  if ((nd || nt) &&
+      (e = launch_nucleus_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, d.dt_d, d.dt_t, batch, tcols,
+                               s, pdl)) != cudaSuccess)
     return cuda_fail(e);
   DecideArgs q = d;
   q.mode_transfer_only = 1;
   q.status = ws.status;
   q.q_hat_out = qbuf;
   q.draft_probs = full_q ? nullptr : draft_probs;
-  if (kd > 0) {
+  if (kd > 0 || nd) {
     if ((e = launch_filter_q(q, s, pdl)) != cudaSuccess) return cuda_fail(e);
   } else if ((e = launch_decide(q, s, pdl)) != cudaSuccess) {
     return cuda_fail(e);
@@ -619,6 +669,8 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   d.status_q = ws.status;
   if (kt > 0) {
     if ((e = launch_decide_filtered(d, s, pdl)) != cudaSuccess) return cuda_fail(e);
+  } else if (nt) {
+    if ((e = launch_decide_nucleus(d, s, pdl)) != cudaSuccess) return cuda_fail(e);
   } else if ((e = launch_decide(d, s, false)) != cudaSuccess) {
     // (this decision kernel reads q_hat before its grid-dependency wait)
     return cuda_fail(e);

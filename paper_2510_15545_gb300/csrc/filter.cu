@@ -3,6 +3,9 @@
 // whose rows the row pass reduced to top-k lists (one sorted list of k
 // candidates per row unit: 2048 fp32 or 4096 bf16 columns).
 //
+// (Nucleus rows, top-p without top-k, are found in nucleus.cu; filter_q_kernel
+// takes both kinds of draft rows.)
+//
 // A filtered row's distribution is fixed by its top k logits: kept_kernel
 // merges the row's unit lists into its top-k (one warp per row, every
 // filtered row of the call at once), then softmax at temperature, the top-p
@@ -35,6 +38,10 @@ __device__ __forceinline__ F2 warp_scan_f2(F2 v, int lane) {
     if (lane >= o) v = f2_add(n, v);
   }
   return v;
+}
+
+__device__ __forceinline__ float load_logit_dt(const char* row, int dt, int64_t col) {
+  return dt == TT_F32 ? load_logit<TT_F32>(row, col) : load_logit<TT_BF16>(row, col);
 }
 
 __device__ __forceinline__ bool cand_before(float v1, int c1, float v2, int c2) {
@@ -476,11 +483,21 @@ __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
   for (int j = warp; j < m; j += kFWarps) {
     if (j > 0 && s_map[j] == s_map[j - 1]) continue;
     const int64_t row = int64_t(d0) + s_map[j];
-    int col;
-    float prob, lse;
-    const int n = load_kept(a.kept_d, a.head_d, row, K, lane, col, prob, lse);
-    if (n == 0) nonfinite = 1;
-    const float q = kept_prob(col, prob, a.draft_cols[row]);
+    float q;
+    if (a.d.nucleus) {  // kept when ranked at or before (tau, tau_col)
+      const KeptHead h = a.head_d[row];
+      if (h.n == 0) nonfinite = 1;
+      const int c = a.draft_cols[row];
+      const float z = load_logit_dt(a.d.data + row * a.d.stride_bytes, a.dt_d, c);
+      const bool kept = z > h.tau || (z == h.tau && c <= h.tau_col);
+      q = kept ? exp2_scaled(z, a.d.scale, h.M) * h.inv_s : 0.f;
+    } else {
+      int col;
+      float prob, lse;
+      const int n = load_kept(a.kept_d, a.head_d, row, K, lane, col, prob, lse);
+      if (n == 0) nonfinite = 1;
+      q = kept_prob(col, prob, a.draft_cols[row]);
+    }
     if (lane == 0) s_q[j] = q;
   }
   const int nf = __syncthreads_or(nonfinite);

@@ -38,12 +38,20 @@ struct Cand {
 // an even count, so that every list starts on a 16-byte boundary.
 __host__ __device__ inline int cand_stride(int k) { return k + (k & 1); }
 
-// Header of a filtered row's kept set (the set itself is k Cand entries
-// holding (probability, column), larger logit first, unused entries (0, -1)):
-// natural log of the kept normaliser, and the kept count (0: not finite).
+// Header of a filtered row's kept set: natural log of the kept normaliser and
+// the kept count (0: not finite). A top-k row's set itself is k Cand entries
+// holding (probability, column), larger logit first, unused entries (0, -1).
+// A nucleus row (top-p without top-k) keeps every column ranked at or before
+// (tau, tau_col) in the order larger logit first, then smaller column; its
+// kept probabilities are 2^(z * scale - M) * inv_s, and its per-chunk kept
+// masses sit in the workspace's um arrays.
 struct KeptHead {
   float lse;
   int32_t n;
+  float tau;       // nucleus rows: raw logit of the last kept column
+  int32_t tau_col; // and that column
+  float M;         // nucleus rows: the row's largest z * scale
+  float inv_s;     // 1 / (sum over kept columns of 2^(z * scale - M))
 };
 
 // The row pass hands out work from kWorkShards counters, each on its own
@@ -68,12 +76,17 @@ struct Workspace {
   Cand* kept_t;      // [(n_target + B) * k_t] kept sets of filtered target rows
   KeptHead* head_d;  // [n_draft] their headers
   KeptHead* head_t;  // [n_target + B]
+  float* um_d;       // [n_draft * nch_d] kept probability mass per chunk of nucleus draft rows
+  float* um_t;       // [(n_target + B) * nch_t] the same for nucleus target rows
   size_t bytes;
 };
 
+// Workspace of a call: k_d / k_t > 0 for families with top-k lists, nuc_d /
+// nuc_t for nucleus families (top-p without top-k).
 __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_draft, int n_target,
                                                       int V_d, int V_t, int k_d = 0,
-                                                      int k_t = 0) {
+                                                      int k_t = 0, bool nuc_d = false,
+                                                      bool nuc_t = false) {
   Workspace w;
   char* p = static_cast<char*>(base);
   size_t off = 0;
@@ -82,26 +95,27 @@ __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_d
     off = align256(off + n);
     return r;
   };
+  const size_t rows_t = size_t(n_target) + B;
   w.part_d = reinterpret_cast<Partial*>(take(sizeof(Partial) * size_t(n_draft) * n_chunks(V_d)));
-  w.part_t = reinterpret_cast<Partial*>(
-      take(sizeof(Partial) * size_t(n_target + B) * n_chunks(V_t)));
+  w.part_t = reinterpret_cast<Partial*>(take(sizeof(Partial) * rows_t * n_chunks(V_t)));
   w.need_d = reinterpret_cast<uint8_t*>(take(size_t(n_draft)));
   w.map = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * size_t(n_target)));
   w.q_hat = reinterpret_cast<float*>(take(sizeof(float) * size_t(n_target)));
   w.status = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * size_t(B)));
-  w.excl = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (size_t(n_target) + B)));
+  w.excl = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * rows_t));
   w.err = reinterpret_cast<int32_t*>(take(2 * sizeof(int32_t)));
   w.work = reinterpret_cast<unsigned long long*>(take(kWorkShards * kWorkStride * sizeof(unsigned long long)));
   w.cand_d = reinterpret_cast<Cand*>(
       take(sizeof(Cand) * size_t(n_draft) * n_chunks(V_d) * size_t(k_d > 0 ? cand_stride(k_d) : 0)));
   w.cand_t = reinterpret_cast<Cand*>(
-      take(sizeof(Cand) * size_t(n_target + B) * n_chunks(V_t) * size_t(k_t > 0 ? cand_stride(k_t) : 0)));
+      take(sizeof(Cand) * rows_t * n_chunks(V_t) * size_t(k_t > 0 ? cand_stride(k_t) : 0)));
   w.kept_d = reinterpret_cast<Cand*>(take(sizeof(Cand) * size_t(n_draft) * size_t(k_d > 0 ? k_d : 0)));
-  w.kept_t = reinterpret_cast<Cand*>(
-      take(sizeof(Cand) * size_t(n_target + B) * size_t(k_t > 0 ? k_t : 0)));
-  w.head_d = reinterpret_cast<KeptHead*>(take(k_d > 0 ? sizeof(KeptHead) * size_t(n_draft) : 0));
-  w.head_t = reinterpret_cast<KeptHead*>(
-      take(k_t > 0 ? sizeof(KeptHead) * (size_t(n_target) + B) : 0));
+  w.kept_t = reinterpret_cast<Cand*>(take(sizeof(Cand) * rows_t * size_t(k_t > 0 ? k_t : 0)));
+  const bool hd = k_d > 0 || nuc_d, ht = k_t > 0 || nuc_t;
+  w.head_d = reinterpret_cast<KeptHead*>(take(hd ? sizeof(KeptHead) * size_t(n_draft) : 0));
+  w.head_t = reinterpret_cast<KeptHead*>(take(ht ? sizeof(KeptHead) * rows_t : 0));
+  w.um_d = reinterpret_cast<float*>(take(nuc_d ? sizeof(float) * size_t(n_draft) * n_chunks(V_d) : 0));
+  w.um_t = reinterpret_cast<float*>(take(nuc_t ? sizeof(float) * rows_t * n_chunks(V_t) : 0));
   w.bytes = off;
   return w;
 }

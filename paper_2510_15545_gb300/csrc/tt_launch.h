@@ -49,6 +49,8 @@ struct RowSet {
   int top_k;            // > 0: filtered rows, the row pass writes top-k lists to cand
   Cand* cand;           // [n_rows * nlist * cand_stride(top_k)]: one list per row unit
   int nlist;            // units (8 KB stages: 2048 fp32 or 4096 bf16 columns) per row
+  int nucleus;          // 1: top-p without top-k (the row pass writes partials, as for
+                        // unfiltered rows; the nucleus kernel finds each row's kept set)
 };
 
 struct RowPassArgs {
@@ -104,18 +106,27 @@ struct DecideArgs {
   const Cand* kept_t;
   const KeptHead* head_d;
   const KeptHead* head_t;
+  const float* um_d;         // per-chunk kept masses of nucleus families
+  const float* um_t;
 };
 
 // The kept-set stage of filtered families: one warp per row merges the row's
 // unit lists into its top-k and applies temperature and top-p.
 struct KeptArgs {
-  RowSet d, t;             // families with top_k > 0 are done, the others skipped
+  RowSet d, t;             // families with top_k > 0 (kept_kernel) or nucleus (nucleus_kernel)
+                           // are done, the others skipped
   int64_t rows_d, rows_t;  // rows of each family (draft rows with d.need[row] == 0 skipped)
   float top_p_d, top_p_t;
   Cand* kept_d;
   Cand* kept_t;
   KeptHead* head_d;
   KeptHead* head_t;
+  float* um_d;             // nucleus families: kept probability mass per chunk
+  float* um_t;
+  int dt_d, dt_t;          // logits types (nucleus rows are read again)
+  int B, n_target;         // the batch, to find a nucleus target row's scored column
+  const int32_t* target_off;
+  const int32_t* target_cols;
 };
 
 struct PrepArgs {
@@ -140,6 +151,11 @@ cudaError_t launch_prep(const PrepArgs& args, cudaStream_t stream);
 // mapped draft rows, and the decision over filtered target rows
 // (args.t.top_k > 0) with q_hat_in given.
 cudaError_t launch_kept(const KeptArgs& args, cudaStream_t stream, int sm_count, bool pdl);
+// Nucleus families (top-p without top-k, App. F): the exact kept set of every
+// nucleus row from its logits and the row pass's partials, and the decision
+// over nucleus target rows.
+cudaError_t launch_nucleus(const KeptArgs& args, cudaStream_t stream, int sm_count, bool pdl);
+cudaError_t launch_decide_nucleus(const DecideArgs& args, cudaStream_t stream, bool pdl);
 cudaError_t launch_filter_q(const DecideArgs& args, cudaStream_t stream, bool pdl);
 cudaError_t launch_decide_filtered(const DecideArgs& args, cudaStream_t stream, bool pdl);
 
@@ -149,6 +165,7 @@ cudaError_t preload_align();
 cudaError_t preload_rowpass();
 cudaError_t preload_decide();
 cudaError_t preload_filter();
+cudaError_t preload_nucleus();
 
 // Records a failed CUDA call for tt_last_cuda_error() and returns TT_ERR_CUDA.
 tt_status record_cuda_error(cudaError_t e);

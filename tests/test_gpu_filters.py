@@ -1,5 +1,6 @@
 """GPU parity of the sampling filters (temperature, top-k, top-p; the paper's
-generation hyperparameter table) against the oracle, through the C ABI:
+generation hyperparameter table) against the oracle, through the C ABI
+(top-p without top-k in test_gpu_nucleus.py):
 tt_step in one-hot and full-q mode, tt_transfer and tt_verify alone, rows with
 many equal logits (the exact fallback of the candidate selection), and the
 argument rules."""
@@ -148,9 +149,6 @@ def test_filter_argument_rules():
     call = lambda **f: tt.tt_step(inp["batch"], inp["vd"], inp["vt"], inp["draft_logits"],
                                   inp["target_logits"], tt.Params(**f))
     with pytest.raises(tt.TTError) as e:
-        call(top_p_target=0.9)  # top-p without top-k
-    assert e.value.code == tt.binding.TT_ERR_UNSUPPORTED
-    with pytest.raises(tt.TTError) as e:
         call(top_k_target=33)
     assert e.value.code == tt.binding.TT_ERR_INVALID_ARG
     with pytest.raises(tt.TTError) as e:
@@ -161,4 +159,9 @@ def test_filter_argument_rules():
     with pytest.raises(tt.TTError) as e:
         tt.tt_step(hin["batch"], hin["vd"], hin["vt"], hin["draft_logits"], hin["target_logits"],
                    tt.Params(full_q=True, top_k_target=4))
+    assert e.value.code == tt.binding.TT_ERR_UNSUPPORTED
+    # full-q has no nucleus rows (top-p without top-k): one-hot transfer only
+    with pytest.raises(tt.TTError) as e:
+        tt.tt_step(hin["batch"], hin["vd"], hin["vt"], hin["draft_logits"], hin["target_logits"],
+                   tt.Params(full_q=True, top_p_draft=0.9, top_p_target=0.9))
     assert e.value.code == tt.binding.TT_ERR_UNSUPPORTED
