@@ -22,6 +22,12 @@ _SRC = os.path.join(_HERE, "tto.c")
 _LIB = os.path.join(_HERE, "libtto.so")
 _lib = None
 
+
+class _Pen(ctypes.Structure):
+    """tto_penalty: the repetition penalty of one family (tto.h)."""
+    _fields_ = [("hist_off", ctypes.c_void_p), ("hist_cols", ctypes.c_void_p),
+                ("theta", ctypes.c_float)]
+
 # Status bits (shared meaning with the CUDA library, defined independently).
 ST_ID_RANGE, ST_TOO_LONG, ST_EMPTY, ST_BAD_OFFSETS = 1, 2, 4, 8
 ST_NO_MATCH, ST_INCONSISTENT = 128, 256
@@ -80,6 +86,13 @@ def lib():
                                   f64, i32, u64, u64, i32, f64, i32, f64, P, P, P, P, P, P, P, P,
                                   P]
         L.tto_verify3.restype = None
+        L.tto_transfer_pen.argtypes = [i32, P, P, P, P, P, i32, i64, i32, P, f64, i32, f64, P, P,
+                                       P, P, P]
+        L.tto_transfer_pen.restype = None
+        L.tto_verify_pen.argtypes = [i32, P, P, P, P, i32, i64, i32, f64, P, P, P, i32, i64, i32,
+                                     f64, i32, u64, u64, i32, f64, i32, f64, P, P, P, P, P, P, P,
+                                     P, P, P]
+        L.tto_verify_pen.restype = None
         L.tto_encode.argtypes = [i32, P, P, P, P, i32, P, P, i32, i32, i32, i32, P, P, P]
         L.tto_encode.restype = None
         L.tto_consistency.argtypes = [i32, P, P, P, P, P, P, i32, P, P, i32, i32, i32, P]
@@ -189,8 +202,20 @@ def filtered_probs(row, temp: float = 1.0, top_k: int = 0, top_p: float = 1.0):
     return out, lse, int(bnd[0])
 
 
+def _penalty(theta, hist_off, hist_cols, keep: list):
+    """(pointer to a tto_penalty or None) for a family's repetition penalty."""
+    if theta is None or float(np.float32(theta)) == 1.0:
+        return None
+    ho = None if hist_off is None else _i32(hist_off)
+    hc = None if hist_cols is None else _i32(hist_cols if len(hist_cols) else np.zeros(1))
+    pen = _Pen(_p(ho), _p(hc), float(theta))
+    keep += [ho, hc, pen]
+    return ctypes.addressof(pen)
+
+
 def transfer(draft_off, draft_cols, target_off, mp, draft_logits, temp_draft: float = 1.0,
-             draft_probs=None, top_k: int = 0, top_p: float = 1.0) -> dict:
+             draft_probs=None, top_k: int = 0, top_p: float = 1.0, rep_penalty: float = 1.0,
+             hist_off=None, hist_cols=None) -> dict:
     draft_off, target_off, mp = _i32(draft_off), _i32(target_off), _i32(mp)
     draft_cols = _i32(draft_cols)
     B = len(draft_off) - 1
@@ -205,16 +230,19 @@ def transfer(draft_off, draft_cols, target_off, mp, draft_logits, temp_draft: fl
     bnd = np.zeros(max(B, 1), np.int32)
     nd = max(int(draft_off[-1]), 0)
     drow = np.zeros(max(nd, 1), np.int32)
-    lib().tto_transfer3(B, _p(draft_off), _p(draft_cols), _p(target_off), _p(mp), _p(buf), dt,
-                        stride, V, _p(probs), float(temp_draft), int(top_k), float(top_p), _p(q),
-                        _p(status), _p(bnd), _p(drow))
+    keep = []
+    pen = _penalty(rep_penalty, hist_off, hist_cols, keep)
+    lib().tto_transfer_pen(B, _p(draft_off), _p(draft_cols), _p(target_off), _p(mp), _p(buf), dt,
+                           stride, V, _p(probs), float(temp_draft), int(top_k), float(top_p), pen,
+                           _p(q), _p(status), _p(bnd), _p(drow))
     return dict(q_hat=q[:nt], status=status, boundary=bnd[:B], drow_bnd=drow[:nd])
 
 
 def verify(target_off, target_cols, q_hat, target_logits, *, temp_target: float = 1.0,
            seed: int = 1234, request_base: int = 0, full_q: bool = False, draft_off=None,
            mp=None, draft_logits=None, temp_draft: float = 1.0, top_k_target: int = 0,
-           top_p_target: float = 1.0, top_k_draft: int = 0, top_p_draft: float = 1.0) -> dict:
+           top_p_target: float = 1.0, top_k_draft: int = 0, top_p_draft: float = 1.0,
+           rep_penalty_target: float = 1.0, hist_off_t=None, hist_cols_t=None) -> dict:
     target_off, target_cols = _i32(target_off), _i32(target_cols)
     q_hat = np.ascontiguousarray(q_hat, dtype=np.float64)
     B = len(target_off) - 1
@@ -234,13 +262,15 @@ def verify(target_off, target_cols, q_hat, target_logits, *, temp_target: float 
     row_bnd = np.zeros(max(nt + B, 1), np.int32)
     tok_lo = np.full(max(B, 1), -1, np.int32)
     tok_hi = np.full(max(B, 1), -1, np.int32)
-    lib().tto_verify3(B, _p(target_off), _p(target_cols), _p(q_hat), _p(tbuf), tdt, tstride, Vt,
-                      float(temp_target), _p(draft_off) if full_q else None,
-                      _p(mp) if full_q else None, _p(dbuf), ddt, dstride, Vd, float(temp_draft),
-                      int(bool(full_q)), int(seed), int(request_base), int(top_k_target),
-                      float(top_p_target), int(top_k_draft), float(top_p_draft), _p(acc),
-                      _p(nxt), _p(p_hat), _p(lse), _p(status), _p(bnd), _p(row_bnd), _p(tok_lo),
-                      _p(tok_hi))
+    keep = []
+    pen = _penalty(rep_penalty_target, hist_off_t, hist_cols_t, keep)
+    lib().tto_verify_pen(B, _p(target_off), _p(target_cols), _p(q_hat), _p(tbuf), tdt, tstride,
+                         Vt, float(temp_target), _p(draft_off) if full_q else None,
+                         _p(mp) if full_q else None, _p(dbuf), ddt, dstride, Vd,
+                         float(temp_draft), int(bool(full_q)), int(seed), int(request_base),
+                         int(top_k_target), float(top_p_target), int(top_k_draft),
+                         float(top_p_draft), pen, _p(acc), _p(nxt), _p(p_hat), _p(lse),
+                         _p(status), _p(bnd), _p(row_bnd), _p(tok_lo), _p(tok_hi))
     return dict(accepted=acc, next_token=nxt, p_hat=p_hat[:nt], lse=lse, status=status,
                 boundary=bnd, row_bnd=row_bnd[:nt + B], tok_lo=tok_lo[:B], tok_hi=tok_hi[:B])
 
@@ -248,8 +278,10 @@ def verify(target_off, target_cols, q_hat, target_logits, *, temp_target: float 
 def step(wl, *, window: Optional[int] = None, temp_draft: Optional[float] = None,
          temp_target: Optional[float] = None, seed: Optional[int] = None,
          request_base: int = 0, full_q: bool = False, draft_probs=None, top_k_draft: int = 0,
-         top_p_draft: float = 1.0, top_k_target: int = 0, top_p_target: float = 1.0) -> dict:
-    """The whole verification path for a workload (align -> transfer -> verify)."""
+         top_p_draft: float = 1.0, top_k_target: int = 0, top_p_target: float = 1.0,
+         rep_penalty_draft: float = 1.0, rep_penalty_target: float = 1.0) -> dict:
+    """The whole verification path for a workload (align -> transfer -> verify);
+    the repetition penalties use the workload's histories (hist_*_d / hist_*_t)."""
     spec = wl.spec
     window = spec.window if window is None else window
     temp_draft = spec.temp_draft if temp_draft is None else temp_draft
@@ -257,13 +289,18 @@ def step(wl, *, window: Optional[int] = None, temp_draft: Optional[float] = None
     seed = spec.seed if seed is None else seed
     al = align(wl.draft_off, wl.draft_ids, wl.target_off, wl.target_ids, wl.vd.blob, wl.vd.off,
                wl.vt.blob, wl.vt.off, window)
+    hist = lambda name: getattr(wl, name, None)
     tr = transfer(wl.draft_off, wl.draft_cols, wl.target_off, al["map"], wl.draft_logits,
-                  temp_draft, draft_probs, top_k=top_k_draft, top_p=top_p_draft)
+                  temp_draft, draft_probs, top_k=top_k_draft, top_p=top_p_draft,
+                  rep_penalty=rep_penalty_draft, hist_off=hist("hist_off_d"),
+                  hist_cols=hist("hist_cols_d"))
     ve = verify(wl.target_off, wl.target_cols, tr["q_hat"], wl.target_logits,
                 temp_target=temp_target, seed=seed, request_base=request_base, full_q=full_q,
                 draft_off=wl.draft_off, mp=al["map"], draft_logits=wl.draft_logits,
                 temp_draft=temp_draft, top_k_target=top_k_target, top_p_target=top_p_target,
-                top_k_draft=top_k_draft, top_p_draft=top_p_draft)
+                top_k_draft=top_k_draft, top_p_draft=top_p_draft,
+                rep_penalty_target=rep_penalty_target, hist_off_t=hist("hist_off_t"),
+                hist_cols_t=hist("hist_cols_t"))
     # the fused step reports the alignment's problems first, else the later stages'
     status = np.where(al["status"] != 0, al["status"], tr["status"] | ve["status"])
     out = dict(al)

@@ -259,6 +259,50 @@ static int32_t offsets_ok(const int32_t* off, int32_t b) {
   return off[b] >= 0 && off[b + 1] >= off[b];
 }
 
+/* ------------------------------------------------------ repetition penalty */
+
+/* The repetition penalty of the generation hyperparameters (App. F; the
+ * Hugging Face default the paper says it keeps): every column of the row's
+ * penalized set -- the request's history and the sequence tokens before the
+ * row's position -- has its logit z replaced by z * theta when z < 0 and by
+ * z / theta otherwise, once however often the column occurs, in fp32
+ * arithmetic (the logits' own type); temperature and the filters then act on
+ * the penalized row. Returns the row to use: `row` itself when there is no
+ * penalty, else `buf` (V floats) holding the penalized copy. */
+static const void* penalized_row(const void* row, int32_t dtype, int64_t V,
+                                 const tto_penalty* pen, int32_t b, const int32_t* seq,
+                                 int32_t n_seq, float* buf, uint8_t* mark, int32_t* out_dtype) {
+  if (!pen || pen->theta == 1.0f) {
+    *out_dtype = dtype;
+    return row;
+  }
+  for (int64_t x = 0; x < V; ++x) {
+    buf[x] = (float)load_logit(row, dtype, x);
+    mark[x] = 0;
+  }
+  if (pen->hist_off)
+    for (int32_t h = pen->hist_off[b]; h < pen->hist_off[b + 1]; ++h) {
+      const int32_t c = pen->hist_cols[h];
+      if (c >= 0 && c < V) mark[c] = 1;
+    }
+  for (int32_t i = 0; i < n_seq; ++i)
+    if (seq[i] >= 0 && seq[i] < V) mark[seq[i]] = 1;
+  const float theta = pen->theta;
+  for (int64_t x = 0; x < V; ++x)
+    if (mark[x]) buf[x] = buf[x] < 0.0f ? buf[x] * theta : buf[x] / theta;
+  *out_dtype = 0;
+  return buf;
+}
+
+/* Status of a request's history under a penalty: its CSR range and columns. */
+static int32_t history_status(const tto_penalty* pen, int32_t b, int64_t V) {
+  if (!pen || pen->theta == 1.0f || !pen->hist_off) return 0;
+  if (!offsets_ok(pen->hist_off, b)) return ST_BAD_OFFSETS;
+  for (int32_t h = pen->hist_off[b]; h < pen->hist_off[b + 1]; ++h)
+    if (pen->hist_cols[h] < 0 || pen->hist_cols[h] >= V) return ST_ID_RANGE;
+  return 0;
+}
+
 void tto_align(int32_t B, const int32_t* draft_off, const int32_t* draft_ids,
                const int32_t* target_off, const int32_t* target_ids,
                const uint8_t* vd_bytes, const int64_t* vd_off, int32_t Vd,
@@ -327,9 +371,12 @@ static void transfer_impl(int32_t B, const int32_t* draft_off, const int32_t* dr
                           const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
                           const float* draft_probs, double T_d, int32_t top_k, double top_p,
                           double* q_hat, int32_t* status, int32_t* boundary,
-                          int32_t* drow_bnd) {
+                          int32_t* drow_bnd, const tto_penalty* pen) {
   const int filtered = top_k > 0 || (top_p > 0.0 && top_p < 1.0);
   double* qf = filtered ? (double*)malloc(sizeof(double) * (size_t)(V > 0 ? V : 1)) : NULL;
+  const int penal = pen && pen->theta != 1.0f && !draft_probs;
+  float* pbuf = penal ? (float*)malloc(sizeof(float) * (size_t)(V > 0 ? V : 1)) : NULL;
+  uint8_t* mark = penal ? (uint8_t*)malloc((size_t)(V > 0 ? V : 1)) : NULL;
   for (int32_t b = 0; b < B; ++b) {
     if (boundary) boundary[b] = 0;
     if (!offsets_ok(draft_off, b) || !offsets_ok(target_off, b)) {
@@ -345,6 +392,7 @@ static void transfer_impl(int32_t B, const int32_t* draft_off, const int32_t* dr
       if (map[t0 + j] < 0 || map[t0 + j] >= k) st |= ST_ID_RANGE;
     for (int32_t i = 0; i < k && !skip_tokens && !draft_probs; ++i)
       if (draft_cols[d0 + i] < 0 || draft_cols[d0 + i] >= V) st |= ST_ID_RANGE;
+    if (!st && penal) st |= history_status(pen, b, V);
     status[b] = st;
     for (int32_t j = 0; j < m; ++j) q_hat[t0 + j] = 0.0;
     if (st) continue;
@@ -353,24 +401,31 @@ static void transfer_impl(int32_t B, const int32_t* draft_off, const int32_t* dr
       int64_t r = (int64_t)d0 + map[t0 + j];
       if (draft_probs) {
         q_hat[t0 + j] = (double)draft_probs[r];
-      } else if (filtered) {
-        const void* row = row_ptr(draft_logits, dtype, row_stride, r);
+        continue;
+      }
+      /* draft row map[j] scores d_{map[j]+1}: the draft tokens before it are penalized */
+      int32_t rdt = dtype;
+      const void* row = penalized_row(row_ptr(draft_logits, dtype, row_stride, r), dtype, V,
+                                      penal ? pen : NULL, b, draft_cols + d0, map[t0 + j], pbuf,
+                                      mark, &rdt);
+      if (filtered) {
         if (r != have) {
           int32_t rb = 0;
-          tto_filtered_probs(row, dtype, V, T_d, top_k, top_p, qf, &rb);
+          tto_filtered_probs(row, rdt, V, T_d, top_k, top_p, qf, &rb);
           if (boundary) boundary[b] |= rb;
           if (drow_bnd) drow_bnd[r] |= rb;
           have = r;
         }
         q_hat[t0 + j] = qf[draft_cols[r]];
       } else {
-        const void* row = row_ptr(draft_logits, dtype, row_stride, r);
-        double lse = tto_logsumexp(row, dtype, V, T_d);
-        q_hat[t0 + j] = exp(load_logit(row, dtype, draft_cols[r]) / T_d - lse);
+        double lse = tto_logsumexp(row, rdt, V, T_d);
+        q_hat[t0 + j] = exp(load_logit(row, rdt, draft_cols[r]) / T_d - lse);
       }
     }
   }
   free(qf);
+  free(pbuf);
+  free(mark);
 }
 
 void tto_transfer2(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
@@ -379,7 +434,7 @@ void tto_transfer2(int32_t B, const int32_t* draft_off, const int32_t* draft_col
                    const float* draft_probs, double T_d, int32_t top_k, double top_p,
                    double* q_hat, int32_t* status, int32_t* boundary) {
   transfer_impl(B, draft_off, draft_cols, target_off, map, draft_logits, dtype, row_stride, V,
-                draft_probs, T_d, top_k, top_p, q_hat, status, boundary, NULL);
+                draft_probs, T_d, top_k, top_p, q_hat, status, boundary, NULL, NULL);
 }
 
 void tto_transfer3(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
@@ -388,7 +443,17 @@ void tto_transfer3(int32_t B, const int32_t* draft_off, const int32_t* draft_col
                    const float* draft_probs, double T_d, int32_t top_k, double top_p,
                    double* q_hat, int32_t* status, int32_t* boundary, int32_t* drow_bnd) {
   transfer_impl(B, draft_off, draft_cols, target_off, map, draft_logits, dtype, row_stride, V,
-                draft_probs, T_d, top_k, top_p, q_hat, status, boundary, drow_bnd);
+                draft_probs, T_d, top_k, top_p, q_hat, status, boundary, drow_bnd, NULL);
+}
+
+void tto_transfer_pen(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                      const int32_t* target_off, const int32_t* map,
+                      const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                      const float* draft_probs, double T_d, int32_t top_k, double top_p,
+                      const tto_penalty* pen, double* q_hat, int32_t* status, int32_t* boundary,
+                      int32_t* drow_bnd) {
+  transfer_impl(B, draft_off, draft_cols, target_off, map, draft_logits, dtype, row_stride, V,
+                draft_probs, T_d, top_k, top_p, q_hat, status, boundary, drow_bnd, pen);
 }
 
 void tto_transfer(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
@@ -418,9 +483,12 @@ static void verify_impl(int32_t B, const int32_t* target_off, const int32_t* tar
                         int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
                         int32_t* accepted, int32_t* next_token, double* p_hat, double* lse,
                         int32_t* status, int32_t* boundary, int32_t* row_bnd,
-                        int32_t* tok_lo, int32_t* tok_hi) {
+                        int32_t* tok_lo, int32_t* tok_hi, const tto_penalty* pen_t) {
   const int filt_t = top_k_t > 0 || (top_p_t > 0.0 && top_p_t < 1.0);
   const int filt_d = top_k_d > 0 || (top_p_d > 0.0 && top_p_d < 1.0);
+  const int penal = pen_t && pen_t->theta != 1.0f;
+  float* pbuf = penal ? (float*)malloc(sizeof(float) * (size_t)V_t) : NULL;
+  uint8_t* mark = penal ? (uint8_t*)malloc((size_t)V_t) : NULL;
   double* pf = filt_t ? (double*)malloc(sizeof(double) * (size_t)V_t) : NULL;
   double* p = (double*)malloc(sizeof(double) * (size_t)V_t);
   double* q = full_q ? (double*)malloc(sizeof(double) * (size_t)V_d) : NULL;
@@ -453,24 +521,29 @@ static void verify_impl(int32_t B, const int32_t* target_off, const int32_t* tar
           if (map[t0 + j] < 0 || map[t0 + j] >= k) st |= ST_ID_RANGE;
       }
     }
+    if (!st && penal) st |= history_status(pen_t, b, V_t);
     status[b] = st;
     if (st) continue;
 
     /* p_hat_j = p_j(t_j) for every target position; lse of all m+1 rows
-       (with filters: of the kept set) */
+       (with filters: of the kept set); row j scores t_{j+1}, so with a
+       penalty the proxy tokens t_1..t_j join the request's history */
     for (int32_t j = 0; j <= m; ++j) {
-      const void* row = row_ptr(target_logits, dtype_t, stride_t, row0 + j);
+      int32_t rdt = dtype_t;
+      const void* row = penalized_row(row_ptr(target_logits, dtype_t, stride_t, row0 + j),
+                                      dtype_t, V_t, pen_t, b, target_cols + t0, j, pbuf, mark,
+                                      &rdt);
       if (filt_t) {
         int32_t rb = 0;
-        double l = tto_filtered_probs(row, dtype_t, V_t, T_t, top_k_t, top_p_t, pf, &rb);
+        double l = tto_filtered_probs(row, rdt, V_t, T_t, top_k_t, top_p_t, pf, &rb);
         boundary[b] |= rb;
         if (row_bnd) row_bnd[row0 + j] |= rb;
         if (lse) lse[row0 + j] = l;
         if (j < m) p_hat[t0 + j] = pf[target_cols[t0 + j]];
       } else {
-        double l = tto_logsumexp(row, dtype_t, V_t, T_t);
+        double l = tto_logsumexp(row, rdt, V_t, T_t);
         if (lse) lse[row0 + j] = l;
-        if (j < m) p_hat[t0 + j] = exp(load_logit(row, dtype_t, target_cols[t0 + j]) / T_t - l);
+        if (j < m) p_hat[t0 + j] = exp(load_logit(row, rdt, target_cols[t0 + j]) / T_t - l);
       }
     }
 
@@ -491,9 +564,12 @@ static void verify_impl(int32_t B, const int32_t* target_off, const int32_t* tar
     accepted[b] = a;
 
     /* the residual (or bonus) row a */
-    const void* prow = row_ptr(target_logits, dtype_t, stride_t, row0 + a);
-    if (filt_t) tto_filtered_probs(prow, dtype_t, V_t, T_t, top_k_t, top_p_t, p, &boundary[b]);
-    else tto_softmax(prow, dtype_t, V_t, T_t, p);
+    int32_t pdt = dtype_t;
+    const void* prow = penalized_row(row_ptr(target_logits, dtype_t, stride_t, row0 + a),
+                                     dtype_t, V_t, pen_t, b, target_cols + t0, a, pbuf, mark,
+                                     &pdt);
+    if (filt_t) tto_filtered_probs(prow, pdt, V_t, T_t, top_k_t, top_p_t, p, &boundary[b]);
+    else tto_softmax(prow, pdt, V_t, T_t, p);
     if (a < m) {
       if (full_q) {
         const void* qrow = row_ptr(draft_logits, dtype_d, stride_d,
@@ -542,6 +618,8 @@ static void verify_impl(int32_t B, const int32_t* target_off, const int32_t* tar
   free(q);
   free(r);
   free(pf);
+  free(pbuf);
+  free(mark);
 }
 
 void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_cols,
@@ -556,7 +634,7 @@ void tto_verify2(int32_t B, const int32_t* target_off, const int32_t* target_col
   verify_impl(B, target_off, target_cols, q_hat, target_logits, dtype_t, stride_t, V_t, T_t,
               draft_off, map, draft_logits, dtype_d, stride_d, V_d, T_d, full_q, seed,
               request_base, top_k_t, top_p_t, top_k_d, top_p_d, accepted, next_token, p_hat,
-              lse, status, boundary, NULL, NULL, NULL);
+              lse, status, boundary, NULL, NULL, NULL, NULL);
 }
 
 void tto_verify3(int32_t B, const int32_t* target_off, const int32_t* target_cols,
@@ -572,7 +650,23 @@ void tto_verify3(int32_t B, const int32_t* target_off, const int32_t* target_col
   verify_impl(B, target_off, target_cols, q_hat, target_logits, dtype_t, stride_t, V_t, T_t,
               draft_off, map, draft_logits, dtype_d, stride_d, V_d, T_d, full_q, seed,
               request_base, top_k_t, top_p_t, top_k_d, top_p_d, accepted, next_token, p_hat,
-              lse, status, boundary, row_bnd, tok_lo, tok_hi);
+              lse, status, boundary, row_bnd, tok_lo, tok_hi, NULL);
+}
+
+void tto_verify_pen(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                    const double* q_hat, const void* target_logits, int32_t dtype_t,
+                    int64_t stride_t, int32_t V_t, double T_t,
+                    const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                    int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                    int32_t full_q, uint64_t seed, uint64_t request_base,
+                    int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
+                    const tto_penalty* pen_t, int32_t* accepted, int32_t* next_token,
+                    double* p_hat, double* lse, int32_t* status, int32_t* boundary,
+                    int32_t* row_bnd, int32_t* tok_lo, int32_t* tok_hi) {
+  verify_impl(B, target_off, target_cols, q_hat, target_logits, dtype_t, stride_t, V_t, T_t,
+              draft_off, map, draft_logits, dtype_d, stride_d, V_d, T_d, full_q, seed,
+              request_base, top_k_t, top_p_t, top_k_d, top_p_d, accepted, next_token, p_hat,
+              lse, status, boundary, row_bnd, tok_lo, tok_hi, pen_t);
 }
 
 void tto_verify(int32_t B, const int32_t* target_off, const int32_t* target_cols,

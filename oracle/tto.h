@@ -135,6 +135,43 @@ void tto_verify3(int32_t B, const int32_t* target_off, const int32_t* target_col
                  int32_t* status, int32_t* boundary, int32_t* row_bnd, int32_t* tok_lo,
                  int32_t* tok_hi);
 
+/* ------------------------------------------------------ repetition penalty */
+
+/* The repetition penalty of the generation hyperparameters (App. F): a request's
+ * history of logits columns (hist_cols[hist_off[b] .. hist_off[b+1]), CSR; NULL
+ * hist_off = empty histories) and the penalty theta (1 = off). A row's
+ * penalized set is the history plus the sequence tokens before the row's
+ * position (target row j: t_1..t_j; draft row i: d_1..d_i, 0-based rows);
+ * each of its columns has z replaced by z * theta when z < 0, else by
+ * z / theta, in fp32, before temperature and the filters. A history column
+ * out of range gives status 1, a bad history range status 8. */
+typedef struct {
+  const int32_t* hist_off;
+  const int32_t* hist_cols;
+  float theta;
+} tto_penalty;
+
+/* tto_transfer3 with a penalty on the draft rows (NULL: none; ignored with
+ * given draft probabilities). */
+void tto_transfer_pen(int32_t B, const int32_t* draft_off, const int32_t* draft_cols,
+                      const int32_t* target_off, const int32_t* map,
+                      const void* draft_logits, int32_t dtype, int64_t row_stride, int32_t V,
+                      const float* draft_probs, double T_d, int32_t top_k, double top_p,
+                      const tto_penalty* pen, double* q_hat, int32_t* status, int32_t* boundary,
+                      int32_t* drow_bnd);
+
+/* tto_verify3 with a penalty on the target rows (NULL: none). */
+void tto_verify_pen(int32_t B, const int32_t* target_off, const int32_t* target_cols,
+                    const double* q_hat, const void* target_logits, int32_t dtype_t,
+                    int64_t stride_t, int32_t V_t, double T_t,
+                    const int32_t* draft_off, const int32_t* map, const void* draft_logits,
+                    int32_t dtype_d, int64_t stride_d, int32_t V_d, double T_d,
+                    int32_t full_q, uint64_t seed, uint64_t request_base,
+                    int32_t top_k_t, double top_p_t, int32_t top_k_d, double top_p_d,
+                    const tto_penalty* pen_t, int32_t* accepted, int32_t* next_token,
+                    double* p_hat, double* lse, int32_t* status, int32_t* boundary,
+                    int32_t* row_bnd, int32_t* tok_lo, int32_t* tok_hi);
+
 /* ------------------------------------------------------------ re-encoding */
 
 /* Re-encoding (§4.2; App. A.1, Lemma 1): T_b = encode_t(decode_d(D_b)).
