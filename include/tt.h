@@ -79,6 +79,7 @@ typedef enum {
 #define TT_MAX_ENCODE_BYTES 2048 /* longest decoded draft string tt_encode takes per request */
 #define TT_MAX_TOP_K 32          /* largest top-k of the sampling filters */
 #define TT_MAX_DPOS_BINS 4096    /* most bins of tt_dpos_hist */
+#define TT_MAX_HISTORY 3072      /* longest repetition-penalty history per request */
 
 typedef enum { TT_F32 = 0, TT_BF16 = 1 } tt_dtype;
 
@@ -129,6 +130,15 @@ typedef struct {
   float top_p_draft;
   int32_t top_k_target;
   float top_p_target;
+  /* Repetition penalty of the same table, per family (1 = off, else > 0): in
+     a row, every column of the request's history (tt_batch hist_*) and of the
+     sequence tokens before the row's position (target row j: t_1..t_j; draft
+     row i: d_1..d_i) has its logit z replaced by z * theta when z < 0, else by
+     z / theta (fp32, once per column), before temperature and the filters.
+     A penalized family needs top_k >= 1 (TT_ERR_UNSUPPORTED otherwise, and in
+     full-q mode). */
+  float rep_penalty_draft;
+  float rep_penalty_target;
 } tt_params;
 
 typedef struct {
@@ -143,6 +153,16 @@ typedef struct {
   const int32_t* target_off;  /* [B+1] */
   const int32_t* target_ids;  /* [n_target] ids into the target vocab table */
   const int32_t* target_cols; /* [n_target] column of t_j in its logits row; NULL = target_ids */
+  /* Histories of the repetition penalty (read only when that family's penalty
+     is on): request b's earlier tokens as logits columns,
+     hist_cols[hist_off[b] .. hist_off[b+1]), at most TT_MAX_HISTORY per request
+     (TT_REQ_TOO_LONG beyond); NULL hist_off = empty histories. */
+  const int32_t* hist_off_d;  /* [B+1] draft family (draft logits columns) */
+  const int32_t* hist_cols_d; /* [n_hist_d] */
+  const int32_t* hist_off_t;  /* [B+1] target family (target logits columns) */
+  const int32_t* hist_cols_t; /* [n_hist_t] */
+  int32_t n_hist_d;           /* hist_off_d[B] (sizes the workspace) */
+  int32_t n_hist_t;           /* hist_off_t[B] */
 } tt_batch;
 
 /* Outputs of tt_step. accepted, next_token and status are required; the rest

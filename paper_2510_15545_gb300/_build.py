@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libtt.so")
 SOURCES = ["api.cu", "align.cu", "rowpass.cu", "decide.cu", "noalloc.cu", "encode.cu", "shard.cu",
-           "filter.cu", "nucleus.cu"]
+           "filter.cu", "nucleus.cu", "pen.cu"]
 HEADERS = ["tt_device.cuh", "tt_launch.h", "tt_shard.h", "tt_f2.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

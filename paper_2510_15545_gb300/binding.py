@@ -10,6 +10,7 @@ import dataclasses
 import os
 from typing import Optional, Sequence
 
+import numpy as np
 import torch
 
 from . import _build
@@ -49,13 +50,16 @@ class _Params(ctypes.Structure):
     _fields_ = [("window", c_i32), ("temp_draft", c_f32), ("temp_target", c_f32),
                 ("full_q", c_i32), ("seed", c_u64), ("request_base", c_u64), ("events", c_p),
                 ("top_k_draft", c_i32), ("top_p_draft", c_f32), ("top_k_target", c_i32),
-                ("top_p_target", c_f32)]
+                ("top_p_target", c_f32), ("rep_penalty_draft", c_f32),
+                ("rep_penalty_target", c_f32)]
 
 
 class _Batch(ctypes.Structure):
     _fields_ = [("B", c_i32), ("n_draft", c_i32), ("n_target", c_i32), ("max_k", c_i32),
                 ("max_m", c_i32), ("draft_off", c_p), ("draft_ids", c_p), ("draft_cols", c_p),
-                ("target_off", c_p), ("target_ids", c_p), ("target_cols", c_p)]
+                ("target_off", c_p), ("target_ids", c_p), ("target_cols", c_p),
+                ("hist_off_d", c_p), ("hist_cols_d", c_p), ("hist_off_t", c_p),
+                ("hist_cols_t", c_p), ("n_hist_d", c_i32), ("n_hist_t", c_i32)]
 
 
 class _StepOut(ctypes.Structure):
@@ -161,6 +165,26 @@ class Batch:
     n_target: int = 0
     max_k: int = 1
     max_m: int = 1
+    # repetition-penalty histories (logits columns, CSR per request); None = empty
+    hist_off_d: Optional[torch.Tensor] = None
+    hist_cols_d: Optional[torch.Tensor] = None
+    hist_off_t: Optional[torch.Tensor] = None
+    hist_cols_t: Optional[torch.Tensor] = None
+    n_hist_d: int = 0
+    n_hist_t: int = 0
+
+    def with_history(self, hist_off_d=None, hist_cols_d=None, hist_off_t=None,
+                     hist_cols_t=None) -> "Batch":
+        """This batch with repetition-penalty histories (host or device arrays)."""
+        dev = self.target_off.device
+
+        def d(x):
+            return None if x is None else torch.as_tensor(x, dtype=torch.int32).to(dev).contiguous()
+        b = dataclasses.replace(self, hist_off_d=d(hist_off_d), hist_cols_d=d(hist_cols_d),
+                                hist_off_t=d(hist_off_t), hist_cols_t=d(hist_cols_t))
+        b.n_hist_d = 0 if hist_off_d is None else int(np.asarray(hist_off_d)[-1])
+        b.n_hist_t = 0 if hist_off_t is None else int(np.asarray(hist_off_t)[-1])
+        return b
 
     @staticmethod
     def from_host(draft_off, draft_ids, target_off, target_ids, draft_cols=None,
@@ -185,7 +209,9 @@ class Batch:
     def _c(self) -> _Batch:
         return _Batch(self.B, self.n_draft, self.n_target, self.max_k, self.max_m,
                       _ptr(self.draft_off), _ptr(self.draft_ids), _ptr(self.draft_cols),
-                      _ptr(self.target_off), _ptr(self.target_ids), _ptr(self.target_cols))
+                      _ptr(self.target_off), _ptr(self.target_ids), _ptr(self.target_cols),
+                      _ptr(self.hist_off_d), _ptr(self.hist_cols_d), _ptr(self.hist_off_t),
+                      _ptr(self.hist_cols_t), int(self.n_hist_d), int(self.n_hist_t))
 
 
 @dataclasses.dataclass
@@ -222,6 +248,9 @@ class Params:
     top_p_draft: float = 1.0
     top_k_target: int = 0
     top_p_target: float = 1.0
+    # repetition penalty per family (1.0 = off); needs that family's top_k >= 1
+    rep_penalty_draft: float = 1.0
+    rep_penalty_target: float = 1.0
 
     def _c(self, keep: list) -> _Params:
         ev = None
@@ -232,7 +261,8 @@ class Params:
         return _Params(int(self.window), float(self.temp_draft), float(self.temp_target),
                        int(bool(self.full_q)), int(self.seed), int(self.request_base), ev,
                        int(self.top_k_draft), float(self.top_p_draft), int(self.top_k_target),
-                       float(self.top_p_target))
+                       float(self.top_p_target), float(self.rep_penalty_draft),
+                       float(self.rep_penalty_target))
 
 
 def _logits(t: Optional[torch.Tensor]) -> Optional[_Logits]:
@@ -525,6 +555,8 @@ def device_inputs(wl, device="cuda") -> dict:
     arguments: batch, vocab tables and logits."""
     batch = Batch.from_host(wl.draft_off, wl.draft_ids, wl.target_off, wl.target_ids,
                             wl.draft_cols, wl.target_cols, device=device)
+    if getattr(wl, "hist_off_d", None) is not None or getattr(wl, "hist_off_t", None) is not None:
+        batch = batch.with_history(wl.hist_off_d, wl.hist_cols_d, wl.hist_off_t, wl.hist_cols_t)
     return dict(batch=batch, vd=VocabTable.from_host(wl.vd.blob, wl.vd.off, device),
                 vt=VocabTable.from_host(wl.vt.blob, wl.vt.off, device),
                 draft_logits=wl.draft_logits.to(device), target_logits=wl.target_logits.to(device),

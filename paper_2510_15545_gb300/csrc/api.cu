@@ -39,6 +39,7 @@ cudaError_t ensure_loaded() {
   if ((e = preload_decide()) != cudaSuccess) return e;
   if ((e = preload_filter()) != cudaSuccess) return e;
   if ((e = preload_nucleus()) != cudaSuccess) return e;
+  if ((e = preload_pen()) != cudaSuccess) return e;
   if ((e = preload_shard()) != cudaSuccess) return e;
   if (dev >= 0 && dev < 64) done[dev].store(true, std::memory_order_release);
   return cudaSuccess;
@@ -90,7 +91,77 @@ bool params_ok(const tt_params* p) {
   if (p->top_k_target < 0 || p->top_k_target > TT_MAX_TOP_K) return false;
   if (!(p->top_p_draft > 0.f) || std::isnan(p->top_p_draft)) return false;
   if (!(p->top_p_target > 0.f) || std::isnan(p->top_p_target)) return false;
+  if (!(p->rep_penalty_draft > 0.f) || !std::isfinite(p->rep_penalty_draft)) return false;
+  if (!(p->rep_penalty_target > 0.f) || !std::isfinite(p->rep_penalty_target)) return false;
   return true;
+}
+
+// Repetition penalties on: per family, and the batch's histories usable.
+bool pen_draft(const tt_params* p) { return p->rep_penalty_draft != 1.f; }
+bool pen_target(const tt_params* p) { return p->rep_penalty_target != 1.f; }
+bool history_ok(const int32_t* off, const int32_t* cols, int32_t n) {
+  return n >= 0 && (off == nullptr ? n == 0 : (n == 0 || cols != nullptr));
+}
+
+PenSizes pen_sizes(const tt_batch* b, bool on_d, bool on_t) {
+  PenSizes p;
+  p.on_d = on_d;
+  p.on_t = on_t;
+  p.n_hist_d = on_d && b->hist_off_d ? b->n_hist_d : 0;
+  p.n_hist_t = on_t && b->hist_off_t ? b->n_hist_t : 0;
+  return p;
+}
+
+// The per-request sets of the penalized families (one small kernel).
+cudaError_t launch_pen_sets(const tt_batch* batch, const RowSet& d, const RowSet& t, bool on_d,
+                            bool on_t, const int32_t* dcols, const int32_t* tcols,
+                            const Workspace& ws, cudaStream_t s) {
+  PenArgs a;
+  std::memset(&a, 0, sizeof a);
+  a.B = batch->B;
+  a.on_d = on_d;
+  a.on_t = on_t;
+  a.V_d = d.V;
+  a.V_t = t.V;
+  a.nch_d = d.nch;
+  a.nch_t = t.nch;
+  a.unit_d = d.unit_cols;
+  a.unit_t = t.unit_cols;
+  a.nlist_d = d.nlist;
+  a.nlist_t = t.nlist;
+  a.n_draft = batch->n_draft;
+  a.n_target = batch->n_target;
+  a.n_hist_d = batch->hist_off_d ? batch->n_hist_d : 0;
+  a.n_hist_t = batch->hist_off_t ? batch->n_hist_t : 0;
+  a.hist_off_d = batch->hist_off_d;
+  a.hist_cols_d = batch->hist_cols_d;
+  a.hist_off_t = batch->hist_off_t;
+  a.hist_cols_t = batch->hist_cols_t;
+  a.draft_off = batch->draft_off;
+  a.draft_cols = dcols;
+  a.target_off = batch->target_off;
+  a.target_cols = tcols;
+  a.pen_d = ws.pen_d;
+  a.pbase_d = ws.pbase_d;
+  a.pcnt_d = ws.pcnt_d;
+  a.pstart_d = ws.pstart_d;
+  a.pen_t = ws.pen_t;
+  a.pbase_t = ws.pbase_t;
+  a.pcnt_t = ws.pcnt_t;
+  a.pstart_t = ws.pstart_t;
+  a.pstatus = ws.pstatus;
+  return launch_pen_prep(a, s);
+}
+
+// A family's row set sees its penalty arrays.
+void attach_pen(RowSet& r, bool on, float theta, PenEntry* pen, const int32_t* pbase,
+                const int32_t* pcnt, const int32_t* pstart) {
+  if (!on) return;
+  r.pen = pen;
+  r.pbase = pbase;
+  r.pcnt = pcnt;
+  r.pstart = pstart;
+  r.penalty = theta;
 }
 
 int k_draft(const tt_params* p) { return p->top_k_draft; }
@@ -140,6 +211,10 @@ RowSet rowset(const tt_logits* L, Partial* part, const uint8_t* need, float T) {
   r.cand = nullptr;
   r.nlist = L->dtype == TT_F32 ? r.nch : (r.nch + 1) / 2;
   r.nucleus = 0;
+  r.pen = nullptr;
+  r.pbase = r.pcnt = r.pstart = nullptr;
+  r.penalty = 1.f;
+  r.unit_cols = L->dtype == TT_F32 ? kChunk : 2 * kChunk;
   return r;
 }
 
@@ -151,12 +226,23 @@ RowSet no_rows() {
   return r;
 }
 
-// Kept sets of the filtered families among d (rows_d rows) and t (rows_t).
+// Kept sets of the filtered families among d (rows_d rows) and t (rows_t);
+// penalized families find each row's request and position from the batch.
 cudaError_t launch_kept_sets(const RowSet& d, int64_t rows_d, const RowSet& t, int64_t rows_t,
                              const tt_params* prm, const Workspace& ws, cudaStream_t s,
-                             bool pdl) {
+                             bool pdl, const tt_batch* batch = nullptr, int dt_d = TT_F32,
+                             int dt_t = TT_F32) {
   KeptArgs k;
   std::memset(&k, 0, sizeof k);
+  if (batch) {
+    k.B = batch->B;
+    k.n_target = batch->n_target;
+    k.n_draft = batch->n_draft;
+    k.target_off = batch->target_off;
+    k.draft_off = batch->draft_off;
+  }
+  k.dt_d = dt_d;
+  k.dt_t = dt_t;
   k.d = d;
   k.t = t;
   k.rows_d = d.top_k > 0 ? rows_d : 0;
@@ -193,6 +279,8 @@ cudaError_t launch_nucleus_sets(const RowSet& d, int64_t rows_d, const RowSet& t
   k.n_target = batch->n_target;
   k.target_off = batch->target_off;
   k.target_cols = tcols;
+  k.draft_off = batch->draft_off;
+  k.n_draft = batch->n_draft;
   return launch_nucleus(k, s, sm_count_current(), pdl);
 }
 
@@ -272,11 +360,18 @@ tt_status step_check(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* 
   const bool nd = from_logits && nuc_draft(prm), nt = nuc_target(prm);
   // full-q: both families filtered or neither, and no nucleus family
   if (full_q && ((kd > 0 || nd) != (kt > 0 || nt) || nd || nt)) return TT_ERR_UNSUPPORTED;
+  // a repetition penalty needs its family's top-k, and one-hot transfer
+  const bool pd = from_logits && pen_draft(prm), pt = pen_target(prm);
+  if ((pd && kd == 0) || (pt && kt == 0) || (full_q && (pd || pt))) return TT_ERR_UNSUPPORTED;
+  if ((pd && !history_ok(batch->hist_off_d, batch->hist_cols_d, batch->n_hist_d)) ||
+      (pt && !history_ok(batch->hist_off_t, batch->hist_cols_t, batch->n_hist_t)))
+    return TT_ERR_INVALID_ARG;
   AlignArgs a;
   const tt_status st = fill_align_args(batch, vd, vt, prm, a);
   if (st != TT_OK) return st;
   *need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target,
-                           from_logits ? draft->n_cols : 0, target->n_cols, kd, kt, nd, nt)
+                           from_logits ? draft->n_cols : 0, target->n_cols, kd, kt, nd, nt,
+                           pen_sizes(batch, pd, pt))
               .bytes;
   return TT_OK;
 }
@@ -290,8 +385,9 @@ size_t tt_workspace_bytes_for(const tt_batch* batch, int32_t V_d, int32_t V_t,
   const int kd = prm ? prm->top_k_draft : 0, kt = prm ? prm->top_k_target : 0;
   if (kd < 0 || kd > TT_MAX_TOP_K || kt < 0 || kt > TT_MAX_TOP_K) return 0;
   const bool nd = prm && nuc_draft(prm), nt = prm && nuc_target(prm);
+  const bool pd = prm && pen_draft(prm), pt = prm && pen_target(prm);
   return workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d < 0 ? 0 : V_d,
-                          V_t < 0 ? 0 : V_t, kd, kt, nd, nt)
+                          V_t < 0 ? 0 : V_t, kd, kt, nd, nt, pen_sizes(batch, pd, pt))
       .bytes;
 }
 
@@ -335,16 +431,20 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   if (from_logits && batch->n_draft > 0 && !cols) return TT_ERR_INVALID_ARG;
   const int kd = from_logits ? k_draft(prm) : 0;  // given probabilities are taken as they are
   const bool nd = from_logits && nuc_draft(prm);
+  const bool pd = from_logits && pen_draft(prm);
+  if (pd && kd == 0) return TT_ERR_UNSUPPORTED;
+  if (pd && !history_ok(batch->hist_off_d, batch->hist_cols_d, batch->n_hist_d))
+    return TT_ERR_INVALID_ARG;
   const int V_d = from_logits ? draft->n_cols : 0;
   const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d,
-                                       0, kd, 0, nd, false)
+                                       0, kd, 0, nd, false, pen_sizes(batch, pd, false))
                           .bytes;
   if (from_logits && (!workspace || workspace_bytes < need ||
                       (reinterpret_cast<uintptr_t>(workspace) & 255) != 0))
     return TT_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d, 0,
-                                  kd, 0, nd, false);
+                                  kd, 0, nd, false, pen_sizes(batch, pd, false));
 
   DecideArgs d;
   std::memset(&d, 0, sizeof d);
@@ -364,6 +464,8 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   d.d.top_k = kd;
   d.d.cand = ws.cand_d;
   d.d.nucleus = nd ? 1 : 0;
+  attach_pen(d.d, pd, prm->rep_penalty_draft, ws.pen_d, ws.pbase_d, ws.pcnt_d, ws.pstart_d);
+  d.status_p = pd ? ws.pstatus : nullptr;
   d.top_p_d = prm->top_p_draft;
   d.t = no_rows();
   d.dt_d = from_logits ? draft->dtype : TT_F32;
@@ -383,12 +485,18 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
     p.need = ws.need_d;
     p.work = ws.work;
     if ((e = launch_prep(p, s)) != cudaSuccess) return cuda_fail(e);
+    if (pd && (e = launch_pen_sets(batch, d.d, no_rows(), true, false, cols, nullptr, ws, s)) !=
+                  cudaSuccess)
+      return cuda_fail(e);
     RowPassArgs r;
     std::memset(&r, 0, sizeof r);
     r.d = d.d;
     r.t = no_rows();
     r.rows_d = batch->n_draft;
     r.rows_t = 0;
+    r.B = batch->B;
+    r.n_draft = batch->n_draft;
+    r.draft_off = batch->draft_off;
     r.err = ws.err;
     r.epoch = next_epoch();
     r.work = ws.work;
@@ -402,8 +510,8 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   }
   if (kd > 0 || nd) {
     attach_kept(d, ws);
-    if (kd > 0 &&
-        (e = launch_kept_sets(d.d, batch->n_draft, no_rows(), 0, prm, ws, s, true)) != cudaSuccess)
+    if (kd > 0 && (e = launch_kept_sets(d.d, batch->n_draft, no_rows(), 0, prm, ws, s, true,
+                                        batch, draft->dtype, draft->dtype)) != cudaSuccess)
       return cuda_fail(e);
     if (nd && (e = launch_nucleus_sets(d.d, batch->n_draft, no_rows(), 0, prm, ws, draft->dtype,
                                        draft->dtype, batch, nullptr, s, true)) != cudaSuccess)
@@ -437,14 +545,20 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   const bool nt = nuc_target(prm), nd = full_q && nuc_draft(prm);
   // full-q: both families filtered or neither, and no nucleus family
   if (full_q && ((kd > 0 || nd) != (kt > 0 || nt) || nd || nt)) return TT_ERR_UNSUPPORTED;
+  // a target penalty needs the target's top-k, and one-hot transfer
+  const bool pt = pen_target(prm);
+  if ((pt && kt == 0) || (full_q && (pt || pen_draft(prm)))) return TT_ERR_UNSUPPORTED;
+  if (pt && !history_ok(batch->hist_off_t, batch->hist_cols_t, batch->n_hist_t))
+    return TT_ERR_INVALID_ARG;
   const int V_d = full_q ? draft->n_cols : 0;
   const size_t need = workspace_layout(nullptr, batch->B, batch->n_draft, batch->n_target, V_d,
-                                       target->n_cols, kd, kt, false, nt).bytes;
+                                       target->n_cols, kd, kt, false, nt,
+                                       pen_sizes(batch, false, pt)).bytes;
   if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
     return TT_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d,
-                                  target->n_cols, kd, kt, false, nt);
+                                  target->n_cols, kd, kt, false, nt, pen_sizes(batch, false, pt));
   cudaError_t e = ensure_loaded();
   if (e != cudaSuccess) return cuda_fail(e);
   if (full_q) {  // the residual needs the mapped draft rows' normalisers
@@ -466,6 +580,10 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   r.t.top_k = kt;
   r.t.cand = ws.cand_t;
   r.t.nucleus = nt ? 1 : 0;
+  attach_pen(r.t, pt, prm->rep_penalty_target, ws.pen_t, ws.pbase_t, ws.pcnt_t, ws.pstart_t);
+  if (pt && (e = launch_pen_sets(batch, no_rows(), r.t, false, true, nullptr, tcols, ws, s)) !=
+                cudaSuccess)
+    return cuda_fail(e);
   r.rows_t = int64_t(batch->n_target) + batch->B;
   r.d = full_q ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
   r.d.top_k = kd;
@@ -514,9 +632,11 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   d.epoch = r.epoch;
   d.top_p_d = prm->top_p_draft;
   d.top_p_t = prm->top_p_target;
+  d.status_p = pt ? ws.pstatus : nullptr;
   if (kt > 0) {
     attach_kept(d, ws);
-    if ((e = launch_kept_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, s, true)) != cudaSuccess)
+    if ((e = launch_kept_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, s, true, batch, d.dt_d,
+                              d.dt_t)) != cudaSuccess)
       return cuda_fail(e);
     if ((e = launch_decide_filtered(d, s, true)) != cudaSuccess) return cuda_fail(e);
   } else if (nt) {
@@ -544,6 +664,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   const bool from_logits = draft_probs == nullptr || full_q;
   const int kd = from_logits ? k_draft(prm) : 0, kt = k_target(prm);
   const bool nd = from_logits && nuc_draft(prm), nt = nuc_target(prm);
+  const bool pd = from_logits && pen_draft(prm), pt = pen_target(prm);
   const bool filtered = kd > 0 || kt > 0 || nd || nt;
   const int V_d = from_logits ? draft->n_cols : 0;
   const int32_t* dcols = batch->draft_cols ? batch->draft_cols : batch->draft_ids;
@@ -554,7 +675,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Workspace ws = workspace_layout(workspace, batch->B, batch->n_draft, batch->n_target, V_d,
-                                  target->n_cols, kd, kt, nd, nt);
+                                  target->n_cols, kd, kt, nd, nt, pen_sizes(batch, pd, pt));
   int32_t* map = out->map ? out->map : ws.map;
   a.path = out->path;
   a.path_len = out->path_len;
@@ -565,12 +686,6 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   a.work = ws.work;
   a.target_cols = tcols;
   a.excl = ws.excl;
-
-  cudaError_t e = ensure_loaded();
-  if (e != cudaSuccess) return cuda_fail(e);
-  record(prm, 0, s);
-  if ((e = launch_align(a, s)) != cudaSuccess) return cuda_fail(e);
-  record(prm, 1, s);
 
   RowPassArgs r;
   std::memset(&r, 0, sizeof r);
@@ -584,10 +699,26 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   r.d.top_k = kd;
   r.d.cand = ws.cand_d;
   r.d.nucleus = nd ? 1 : 0;
+  attach_pen(r.d, pd, prm->rep_penalty_draft, ws.pen_d, ws.pbase_d, ws.pcnt_d, ws.pstart_d);
+  attach_pen(r.t, pt, prm->rep_penalty_target, ws.pen_t, ws.pbase_t, ws.pcnt_t, ws.pstart_t);
   r.B = batch->B;
   r.n_target = batch->n_target;
+  r.n_draft = batch->n_draft;
   r.target_off = batch->target_off;
   r.target_cols = tcols;
+  r.draft_off = batch->draft_off;
+
+  cudaError_t e = ensure_loaded();
+  if (e != cudaSuccess) return cuda_fail(e);
+  // the penalty's per-request sets, complete before the alignment (launched
+  // without a dependent-launch attribute) and so before the row pass starts
+  if ((pd || pt) &&
+      (e = launch_pen_sets(batch, r.d, r.t, pd, pt, dcols, tcols, ws, s)) != cudaSuccess)
+    return cuda_fail(e);
+  record(prm, 0, s);
+  if ((e = launch_align(a, s)) != cudaSuccess) return cuda_fail(e);
+  record(prm, 1, s);
+
   r.err = ws.err;
   r.epoch = next_epoch();
   r.work = ws.work;       // zeroed by the alignment kernel
@@ -634,6 +765,7 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   d.epoch = r.epoch;
   d.top_p_d = prm->top_p_draft;
   d.top_p_t = prm->top_p_target;
+  d.status_p = (pd || pt) ? ws.pstatus : nullptr;
   if (!filtered) {
     d.warm_ctas = sm_count_current();  // the first CTA on each SM
     if ((e = launch_decide(d, s, pdl)) != cudaSuccess) return cuda_fail(e);
@@ -647,7 +779,8 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   float* qbuf = out->q_hat ? out->q_hat : ws.q_hat;
   attach_kept(d, ws);
   if ((kd > 0 || kt > 0) &&
-      (e = launch_kept_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, s, pdl)) != cudaSuccess)
+      (e = launch_kept_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, s, pdl, batch, d.dt_d,
+                            d.dt_t)) != cudaSuccess)
     return cuda_fail(e);
   if ((nd || nt) &&
       (e = launch_nucleus_sets(r.d, r.rows_d, r.t, r.rows_t, prm, ws, d.dt_d, d.dt_t, batch, tcols,
@@ -700,7 +833,8 @@ tt_status tt_verify_sharded(const tt_batch* batch, const float* q_hat, const tt_
   int32_t V = 0;
   if (!shards_ok(target, rows, &V)) return TT_ERR_INVALID_ARG;
   // one-hot transfer, no filters
-  if (prm->full_q != 0 || prm->top_k_target != 0 || prm->top_p_target < 1.f)
+  if (prm->full_q != 0 || prm->top_k_target != 0 || prm->top_p_target < 1.f ||
+      pen_target(prm))
     return TT_ERR_UNSUPPORTED;
   const ShardWorkspace ws0 = shard_workspace(nullptr, batch, target);
   if (!workspace || workspace_bytes < ws0.bytes ||

@@ -357,6 +357,98 @@ __device__ __forceinline__ void row_topk(const Cand* lists, int nch, int K, int 
   else row_topk_wide(lists, nch, K, Ls, lane, scr, top);
 }
 
+// The top-K of a row under the repetition penalty: its lists' top-K (which
+// leave out the request's penalized columns; -inf entries stand in for them)
+// merged with those columns, each at the row's own value: penalized (z * theta
+// for z < 0, else z / theta, fp32) when the column's first sequence position
+// lies before the row's, raw otherwise. In place in `top`; one warp.
+__device__ void penalize_top(const KeptArgs& a, const RowSet& S, int dt, bool tgt, int64_t row,
+                             int K, int lane, Cand* scr, Cand* top) {
+  const int32_t* off = tgt ? a.target_off : a.draft_off;
+  int lo = 0, hi = a.B - 1;
+  while (lo < hi) {  // the row's request: largest b whose first row is at or before row
+    const int mid = (lo + hi + 1) >> 1;
+    if (int64_t(off[mid]) + (tgt ? mid : 0) <= row) lo = mid;
+    else hi = mid - 1;
+  }
+  const int b = lo;
+  const int64_t j = row - (int64_t(off[b]) + (tgt ? b : 0));  // position of the row
+  const int base = S.pbase[b], cnt = S.pcnt[b];
+  const float th = S.penalty;
+  const char* zrow = S.data + row * S.stride_bytes;
+  const Cand me = lane < K ? top[lane] : Cand{-INFINITY, -1};
+  const bool real = lane < K && me.c >= 0 && me.v > -INFINITY;
+  const int nt = __popc(__ballot_sync(0xffffffffu, real));  // a prefix of the lanes
+  const bool full = nt == K;
+  const float tv = __shfl_sync(0xffffffffu, me.v, K - 1);
+  const int tc = __shfl_sync(0xffffffffu, me.c, K - 1);
+  auto value = [&](const PenEntry& e) -> float {
+    const float z = load_logit_dt(zrow, dt, e.col);
+    return e.first < j ? (z < 0.f ? __fmul_rn(z, th) : __fdiv_rn(z, th)) : z;
+  };
+  __syncwarp();
+  if (real) scr[lane] = me;
+  int n = nt;
+  for (int i0 = 0; i0 < cnt; i0 += 32) {
+    const int i = i0 + lane;
+    Cand c = {-INFINITY, -1};
+    bool q = false;
+    if (i < cnt) {
+      const PenEntry e = S.pen[base + i];
+      c = Cand{value(e), e.col};
+      q = c.v > -INFINITY && (!full || cand_before(c.v, c.c, tv, tc));
+    }
+    const unsigned m = __ballot_sync(0xffffffffu, q);
+    const int pos = n + __popc(m & ((1u << lane) - 1u));
+    if (q && pos < kRowCap) scr[pos] = c;
+    n += __popc(m);
+  }
+  __syncwarp();
+  if (n <= kRowCap) {
+    for (int i = lane; i < n; i += 32) {
+      const Cand ci = scr[i];
+      int r = 0;
+      for (int x = 0; x < n; ++x) r += cand_before(scr[x].v, scr[x].c, ci.v, ci.c);
+      if (r < K) top[r] = ci;
+    }
+    for (int r = n + lane; r < K; r += 32) top[r] = Cand{-INFINITY, -1};
+  } else {
+    // more candidates than the buffer: K rounds of a warp arg-best over the
+    // list entries and the penalized columns
+    float pv = INFINITY;
+    int pc = -1;
+    for (int r = 0; r < K; ++r) {
+      float bv = -INFINITY;
+      int bc = 0x7fffffff;
+      bool f = false;
+      if (real && cand_before(pv, pc, me.v, me.c)) {
+        bv = me.v;
+        bc = me.c;
+        f = true;
+      }
+      for (int i = lane; i < cnt; i += 32) {
+        const PenEntry e = S.pen[base + i];
+        const float v = value(e);
+        if (v > -INFINITY && cand_before(pv, pc, v, e.col) && (!f || cand_before(v, e.col, bv, bc))) {
+          bv = v;
+          bc = e.col;
+          f = true;
+        }
+      }
+      warp_best(bv, bc, f);
+      if (lane == 0) top[r] = f ? Cand{bv, bc} : Cand{-INFINITY, -1};
+      if (f) {
+        pv = bv;
+        pc = bc;
+      } else {
+        pv = -INFINITY;
+        pc = 0x7fffffff;
+      }
+    }
+  }
+  __syncwarp();
+}
+
 // The kept set of a filtered row from its top-K (in shared memory): lane i < n
 // holds kept entry i (column, probability); returns n (0: no finite logit).
 // lse = natural log of the kept set's normaliser sum exp(z / T).
@@ -418,6 +510,8 @@ __global__ void __launch_bounds__(kFThreads) kept_kernel(KeptArgs a) {
     const int K = S.top_k;
     const int Ls = cand_stride(K);
     row_topk(S.cand + row * S.nlist * Ls, S.nlist, K, Ls, lane, s_scr[warp], s_top[warp]);
+    if (S.pen) penalize_top(a, S, tgt ? a.dt_t : a.dt_d, tgt, row, K, lane, s_scr[warp],
+                            s_top[warp]);
     int col;
     float prob, lse;
     const int n = kept_set(s_top[warp], K, S.scale, tgt ? a.top_p_t : a.top_p_d, lane, col,
@@ -471,6 +565,7 @@ __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
       if (i < 0 || i >= k) bad = 1;
     }
   if (__syncthreads_or(bad)) st |= TT_REQ_ID_OUT_OF_RANGE;
+  if (st == 0 && a.status_p) st = a.status_p[b];  // the penalty's histories
   if (st == 0 && a.err && a.err[0] == a.epoch) st = a.err[1];
   if (st != 0) {
     if (!(st & (TT_REQ_BAD_OFFSETS | TT_REQ_TOO_LONG)))
@@ -548,6 +643,7 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
     if (s_in != 0) st = s_in;  // the alignment's verdict comes first
   }
   if (st == 0 && a.status_q) st = a.status_q[b];  // then the transfer's
+  if (st == 0 && a.status_p) st = a.status_p[b];  // then the penalty's histories
   if (a.err && a.err[0] == a.epoch) st = a.err[1];  // the row pass failed
   bad = 0;
   if (st == 0 && a.full_q)

@@ -42,7 +42,7 @@ struct Desc {
   int32_t n_smem; // leading columns delivered by the bulk copy (rest read directly)
   int32_t excl;   // column (within the unit) left out of the sum, -1 = none
   int32_t set;    // 0 draft rows, 1 target rows
-  int32_t pad;
+  int32_t req;    // the row's request when its family has a repetition penalty, else -1
 };
 
 // Stage s is always refilled for the same consumer warp (s mod kConsumerWarps),
@@ -161,6 +161,66 @@ __device__ __forceinline__ int excl_lookup(const RowPassArgs& a, ExclCursor* cur
   if (j < 0 || j >= cur->r1 - cur->r0) return -1;  // the bonus row
   const int c = a.target_cols[cur->t0 + j];
   return (c >= 0 && c < a.t.V) ? c : -1;
+}
+
+// The request of a row, for rows visited mostly in increasing order (kept in
+// shared memory like ExclCursor): target rows of request b are
+// target_off[b] + b .. target_off[b+1] + b, draft rows draft_off[b] ..
+// draft_off[b+1] - 1. -1 outside every request.
+struct ReqCursor {
+  int b;
+  int64_t r0, r1;  // rows of request b: r0 .. r1 inclusive
+};
+
+__device__ __forceinline__ int req_lookup(const int32_t* off, int B, bool tgt, ReqCursor* cur,
+                                          int64_t r) {
+  if (!off || B <= 0) return -1;
+  int b = cur->b;
+  if (b >= 0 && r >= cur->r0 && r <= cur->r1) return b;
+  if (b >= 0 && r == cur->r1 + 1 && b + 1 < B) {
+    ++b;
+  } else {
+    int lo = 0, hi = B - 1;
+    while (lo < hi) {  // largest b whose first row is at or before r
+      const int mid = (lo + hi + 1) >> 1;
+      if (int64_t(off[mid]) + (tgt ? mid : 0) <= r) lo = mid;
+      else hi = mid - 1;
+    }
+    b = lo;
+  }
+  const int64_t r0 = int64_t(off[b]) + (tgt ? b : 0);
+  const int64_t r1 = int64_t(off[b + 1]) + (tgt ? b : -1);
+  cur->b = b;
+  cur->r0 = r0;
+  cur->r1 = r1;
+  return (r >= r0 && r <= r1) ? b : -1;
+}
+
+// Repetition penalty: the request's penalized columns within a unit held in
+// shared memory are set to -inf (they leave its top-k list; the kept-set
+// kernel adds them back with the row's own values); those in the unit's
+// ragged tail, read directly, are returned as lane bits to drop.
+template <int DT>
+__device__ __forceinline__ uint32_t mask_penalized(char* stage, const Desc& d, const RowSet& S,
+                                                   int cps, int lane) {
+  const int u = d.chunk / cps;
+  const int64_t srow = int64_t(d.req) * (S.nch + 1);
+  const int base = S.pbase[d.req];
+  const int lo = S.pstart[srow + u], hi = S.pstart[srow + u + 1];
+  const int c0 = d.chunk * kChunk;
+  uint32_t drop = 0u;
+  for (int i = lo + lane; i < hi; i += 32) {
+    const int x = S.pen[base + i].col - c0;
+    if (x >= 0 && x < d.n_smem) {
+      if constexpr (DT == TT_F32) reinterpret_cast<float*>(stage)[x] = -INFINITY;
+      else reinterpret_cast<uint16_t*>(stage)[x] = 0xff80u;  // bf16 -inf
+    } else if (x >= d.n_smem && x < d.n) {
+      drop |= 1u << (x - d.n_smem);
+    }
+  }
+  drop = __reduce_or_sync(0xffffffffu, drop);
+  __syncwarp();
+  return drop;
 }
 
 template <int DT>
@@ -331,7 +391,7 @@ __device__ __forceinline__ float vec_max(const uint4& w) {
 // every unit, which keeps the stage ring from waiting on one slow warp.
 template <int DT>
 __device__ void select_unit(const char* stage, const Desc& d, const RowView& S, int lane, int K,
-                            Cand* scratch, Cand* out) {
+                            Cand* scratch, Cand* out, uint32_t tail_drop = 0u) {
   constexpr int VEC = DT == TT_F32 ? 4 : 8;  // logits per 16-byte vector
   constexpr int NV = kChunk * 4 / (16 * 32);   // vectors per lane in one stage
   constexpr uint32_t kTailBit = 1u << NV;      // flag of the lane's tail element
@@ -341,7 +401,7 @@ __device__ void select_unit(const char* stage, const Desc& d, const RowView& S, 
   const int nvec = d.n_smem / VEC;  // whole vectors delivered (the copy moves 16-byte units)
   // this lane's vectors v < nvl lie within the copy
   const int nvl = max(0, min(NV, (nvec - lane + 31) >> 5));
-  const bool has_tail = lane < d.n - d.n_smem;
+  const bool has_tail = lane < d.n - d.n_smem && !((tail_drop >> lane) & 1u);
   // the tail element, NaN where the lane has none (NaN never compares >=)
   float zt = kNaN;
   if (has_tail) {
@@ -545,7 +605,9 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       int64_t cached_row = -1, cached_drow = -1;
       int cached_excl = -1;
       __shared__ ExclCursor cursor;
+      __shared__ ReqCursor rcur_d, rcur_t;
       cursor.b = -1;
+      rcur_d.b = rcur_t.b = -1;
       bool cached_need = true;
       // Queues chunk `chunk` of row `row` (tgt: a target row, else a draft
       // row) on the next stage; false once a wait has run out.
@@ -580,6 +642,9 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
           }
           if (!cached_need) return true;  // no target position maps to this row
         }
+        d.req = S->pen ? req_lookup(tgt ? a.target_off : a.draft_off, a.B, tgt,
+                                    tgt ? &rcur_t : &rcur_d, row)
+                       : -1;
         d.chunk = unit * cps;
         const int c0 = d.chunk * kChunk;
         d.n = min(cps * kChunk, S->V - c0);
@@ -714,12 +779,18 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       const RowSet& S = d.set ? a.t : a.d;
       Cand* out = S.cand + (d.row * S.nlist + d.chunk / cps) * cand_stride(S.top_k);
       const RowView V = {a, S.scale};
+      uint32_t drop = 0u;
+      if (S.pen && d.req >= 0) {
+        char* wstage = stages + size_t(s) * R::kStageBytes;
+        drop = (d.set ? DTT : DTD) == TT_F32 ? mask_penalized<TT_F32>(wstage, d, S, cps, lane)
+                                             : mask_penalized<TT_BF16>(wstage, d, S, cps, lane);
+      }
       if constexpr (DTD == DTT) {
-        select_unit<DTT>(stage, d, V, lane, S.top_k, scratch, out);
+        select_unit<DTT>(stage, d, V, lane, S.top_k, scratch, out, drop);
       } else if (d.set) {
-        select_unit<DTT>(stage, d, V, lane, S.top_k, scratch, out);
+        select_unit<DTT>(stage, d, V, lane, S.top_k, scratch, out, drop);
       } else {
-        select_unit<DTD>(stage, d, V, lane, S.top_k, scratch, out);
+        select_unit<DTD>(stage, d, V, lane, S.top_k, scratch, out, drop);
       }
       if (lane == 0 && !(blockIdx.x == 0 && it == a.stall_stage))
         mbar_arrive(&empty[s]);  // the stage's bytes are consumed

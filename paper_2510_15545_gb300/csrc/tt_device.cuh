@@ -54,6 +54,21 @@ struct KeptHead {
   float inv_s;     // 1 / (sum over kept columns of 2^(z * scale - M))
 };
 
+// A column of a request's repetition-penalty set (its history and sequence
+// tokens): the column and the first sequence position holding it (-1 when the
+// history holds it), so that a row at position j penalizes it when first < j.
+// A request's entries are sorted by column, one per column.
+struct PenEntry {
+  int32_t col;
+  int32_t first;
+};
+
+// Sizes of the repetition-penalty arrays of a call (zeros: no penalty).
+struct PenSizes {
+  int n_hist_d = 0, n_hist_t = 0;  // history entries of each family
+  bool on_d = false, on_t = false; // families with a penalty
+};
+
 // The row pass hands out work from kWorkShards counters, each on its own
 // 256-byte line, so that no single L2 address serialises every CTA's draws.
 constexpr int kWorkShards = 8;
@@ -78,6 +93,18 @@ struct Workspace {
   KeptHead* head_t;  // [n_target + B]
   float* um_d;       // [n_draft * nch_d] kept probability mass per chunk of nucleus draft rows
   float* um_t;       // [(n_target + B) * nch_t] the same for nucleus target rows
+  // repetition penalty, per penalized family: each request's sorted penalized
+  // columns (at base[b], cnt[b] entries, capacity its history plus its tokens)
+  // and, per row unit u, the first entry at or past the unit's first column
+  PenEntry* pen_d;    // [n_hist_d + n_draft]
+  int32_t* pbase_d;   // [B]
+  int32_t* pcnt_d;    // [B]
+  int32_t* pstart_d;  // [B * (nch_d + 1)]
+  PenEntry* pen_t;    // [n_hist_t + n_target]
+  int32_t* pbase_t;   // [B]
+  int32_t* pcnt_t;    // [B]
+  int32_t* pstart_t;  // [B * (nch_t + 1)]
+  int32_t* pstatus;   // [B] problems of the histories (TT_REQ_* bits)
   size_t bytes;
 };
 
@@ -86,7 +113,8 @@ struct Workspace {
 __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_draft, int n_target,
                                                       int V_d, int V_t, int k_d = 0,
                                                       int k_t = 0, bool nuc_d = false,
-                                                      bool nuc_t = false) {
+                                                      bool nuc_t = false,
+                                                      PenSizes pen = PenSizes()) {
   Workspace w;
   char* p = static_cast<char*>(base);
   size_t off = 0;
@@ -116,6 +144,20 @@ __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_d
   w.head_t = reinterpret_cast<KeptHead*>(take(ht ? sizeof(KeptHead) * rows_t : 0));
   w.um_d = reinterpret_cast<float*>(take(nuc_d ? sizeof(float) * size_t(n_draft) * n_chunks(V_d) : 0));
   w.um_t = reinterpret_cast<float*>(take(nuc_t ? sizeof(float) * rows_t * n_chunks(V_t) : 0));
+  const size_t pd = pen.on_d ? 1 : 0, pt = pen.on_t ? 1 : 0;
+  w.pen_d = reinterpret_cast<PenEntry*>(
+      take(pd * sizeof(PenEntry) * (size_t(pen.n_hist_d) + size_t(n_draft))));
+  w.pbase_d = reinterpret_cast<int32_t*>(take(pd * sizeof(int32_t) * size_t(B)));
+  w.pcnt_d = reinterpret_cast<int32_t*>(take(pd * sizeof(int32_t) * size_t(B)));
+  w.pstart_d = reinterpret_cast<int32_t*>(
+      take(pd * sizeof(int32_t) * size_t(B) * size_t(n_chunks(V_d) + 1)));
+  w.pen_t = reinterpret_cast<PenEntry*>(
+      take(pt * sizeof(PenEntry) * (size_t(pen.n_hist_t) + size_t(n_target))));
+  w.pbase_t = reinterpret_cast<int32_t*>(take(pt * sizeof(int32_t) * size_t(B)));
+  w.pcnt_t = reinterpret_cast<int32_t*>(take(pt * sizeof(int32_t) * size_t(B)));
+  w.pstart_t = reinterpret_cast<int32_t*>(
+      take(pt * sizeof(int32_t) * size_t(B) * size_t(n_chunks(V_t) + 1)));
+  w.pstatus = reinterpret_cast<int32_t*>(take((pd | pt) * sizeof(int32_t) * size_t(B)));
   w.bytes = off;
   return w;
 }

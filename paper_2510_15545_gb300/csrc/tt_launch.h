@@ -51,6 +51,15 @@ struct RowSet {
   int nlist;            // units (8 KB stages: 2048 fp32 or 4096 bf16 columns) per row
   int nucleus;          // 1: top-p without top-k (the row pass writes partials, as for
                         // unfiltered rows; the nucleus kernel finds each row's kept set)
+  // Repetition penalty (top-k families only; pen = NULL: none): the row pass
+  // leaves each request's penalized columns out of its unit lists, and the
+  // kept-set kernel adds them back with the row's own (penalized or raw) value.
+  const PenEntry* pen;    // sorted penalized columns of request b at pbase[b] (pcnt[b])
+  const int32_t* pbase;
+  const int32_t* pcnt;
+  const int32_t* pstart;  // [B * (nch + 1)]: first entry of each row unit, then pcnt
+  float penalty;          // theta
+  int unit_cols;          // columns per row unit (2048 fp32, 4096 bf16)
 };
 
 struct RowPassArgs {
@@ -58,9 +67,10 @@ struct RowPassArgs {
   int64_t rows_d, rows_t;    // rows of each family to stream (0 = family absent)
   const int32_t* excl;       // [target rows] column left out of the sum, or NULL: found
                              // from target_off / target_cols
-  int B, n_target;
+  int B, n_target, n_draft;
   const int32_t* target_off;
   const int32_t* target_cols;
+  const int32_t* draft_off;  // to find a penalized draft row's request
   int32_t* err;              // err[0] = epoch of a failed call, err[1] = its TT_REQ_* bits
   int32_t epoch;             // identifies this call
   const int32_t* excl_late;  // as excl, but written by the grid this one depends on: read
@@ -108,6 +118,7 @@ struct DecideArgs {
   const KeptHead* head_t;
   const float* um_d;         // per-chunk kept masses of nucleus families
   const float* um_t;
+  const int32_t* status_p;   // problems of the repetition-penalty histories, or NULL
 };
 
 // The kept-set stage of filtered families: one warp per row merges the row's
@@ -127,6 +138,35 @@ struct KeptArgs {
   int B, n_target;         // the batch, to find a nucleus target row's scored column
   const int32_t* target_off;
   const int32_t* target_cols;
+  const int32_t* draft_off;  // and a penalized draft row's request
+  int n_draft;
+};
+
+// The repetition penalty's per-request sets (pen.cu): for each penalized
+// family, every request's history and sequence columns sorted and made unique
+// (with the first sequence position of each), and the start of each row unit.
+struct PenArgs {
+  int B;
+  int on_d, on_t;
+  int V_d, V_t, nch_d, nch_t, unit_d, unit_t, nlist_d, nlist_t;
+  int n_draft, n_target, n_hist_d, n_hist_t;
+  const int32_t* hist_off_d;
+  const int32_t* hist_cols_d;
+  const int32_t* hist_off_t;
+  const int32_t* hist_cols_t;
+  const int32_t* draft_off;
+  const int32_t* draft_cols;
+  const int32_t* target_off;
+  const int32_t* target_cols;
+  PenEntry* pen_d;
+  int32_t* pbase_d;
+  int32_t* pcnt_d;
+  int32_t* pstart_d;
+  PenEntry* pen_t;
+  int32_t* pbase_t;
+  int32_t* pcnt_t;
+  int32_t* pstart_t;
+  int32_t* pstatus;
 };
 
 struct PrepArgs {
@@ -156,6 +196,7 @@ cudaError_t launch_kept(const KeptArgs& args, cudaStream_t stream, int sm_count,
 // over nucleus target rows.
 cudaError_t launch_nucleus(const KeptArgs& args, cudaStream_t stream, int sm_count, bool pdl);
 cudaError_t launch_decide_nucleus(const DecideArgs& args, cudaStream_t stream, bool pdl);
+cudaError_t launch_pen_prep(const PenArgs& args, cudaStream_t stream);
 cudaError_t launch_filter_q(const DecideArgs& args, cudaStream_t stream, bool pdl);
 cudaError_t launch_decide_filtered(const DecideArgs& args, cudaStream_t stream, bool pdl);
 
@@ -166,6 +207,7 @@ cudaError_t preload_rowpass();
 cudaError_t preload_decide();
 cudaError_t preload_filter();
 cudaError_t preload_nucleus();
+cudaError_t preload_pen();
 
 // Records a failed CUDA call for tt_last_cuda_error() and returns TT_ERR_CUDA.
 tt_status record_cuda_error(cudaError_t e);

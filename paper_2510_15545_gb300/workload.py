@@ -216,6 +216,11 @@ class Workload:
     target_cols: np.ndarray  # int32 [n_target]
     draft_logits: torch.Tensor  # [n_draft, V_dl]
     target_logits: torch.Tensor  # [n_target + B, V_tl]
+    # repetition-penalty histories (logits columns, CSR per request); None = none
+    hist_off_d: Optional[np.ndarray] = None
+    hist_cols_d: Optional[np.ndarray] = None
+    hist_off_t: Optional[np.ndarray] = None
+    hist_cols_t: Optional[np.ndarray] = None
 
     @property
     def B(self) -> int:
@@ -258,10 +263,21 @@ class Workload:
             return np.concatenate(xs).astype(np.int32) if xs else np.zeros(0, np.int32)
         dl = self.draft_logits[torch.as_tensor(d_rows, device=self.draft_logits.device)].cpu()
         tl = self.target_logits[torch.as_tensor(t_rows, device=self.target_logits.device)].cpu()
+
+        def hist(off, cols):
+            if off is None:
+                return None, None
+            parts = [cols[off[b]:off[b + 1]] for b in idx]
+            o = np.concatenate([[0], np.cumsum([len(x) for x in parts])]).astype(np.int32)
+            return o, cat(parts)
+        hod, hcd = hist(self.hist_off_d, self.hist_cols_d)
+        hot, hct = hist(self.hist_off_t, self.hist_cols_t)
         return dataclasses.replace(self, draft_off=np.array(d_off, np.int32),
                                    target_off=np.array(t_off, np.int32), draft_ids=cat(d_ids),
                                    target_ids=cat(t_ids), draft_cols=cat(d_cols),
-                                   target_cols=cat(t_cols), draft_logits=dl, target_logits=tl)
+                                   target_cols=cat(t_cols), draft_logits=dl, target_logits=tl,
+                                   hist_off_d=hod, hist_cols_d=hcd, hist_off_t=hot,
+                                   hist_cols_t=hct)
 
     def request(self, b: int) -> dict:
         d0, d1 = int(self.draft_off[b]), int(self.draft_off[b + 1])
@@ -488,3 +504,41 @@ def homogeneous_workload(B: int, k: int, V: int, *, seed: int = 0, device: str =
                     target_off=target_off, target_ids=ids.copy(), draft_cols=ids.copy(),
                     target_cols=ids.copy(), draft_logits=draft_logits.to(dtype),
                     target_logits=tl.to(dtype))
+
+
+def with_histories(wl: Workload, lo: int, hi: int, seed: int = 0) -> Workload:
+    """The workload with seeded repetition-penalty histories: each request gets
+    between lo and hi earlier tokens per family (logits columns), half of them
+    drawn from the request's own rows by the Gumbel-max trick (tokens the rows
+    make likely, as a real context's tokens are) and half uniformly, with
+    repeats allowed."""
+    rng = np.random.default_rng(seed * 7919 + 17)
+    gen = torch.Generator(device=wl.target_logits.device)
+    gen.manual_seed(seed * 104729 + 23)
+
+    def family(off_rows, logits, extra_row):
+        offs, cols = [0], []
+        V = logits.shape[1]
+        for b in range(wl.B):
+            n = int(rng.integers(lo, hi + 1))
+            r0, r1 = int(off_rows[b]) + (b if extra_row else 0), int(off_rows[b + 1]) + (
+                b + 1 if extra_row else 0)
+            n_like = n // 2
+            if n_like > 0 and r1 > r0:
+                rows = torch.as_tensor(rng.integers(r0, r1, size=n_like), device=logits.device)
+                u = torch.rand((n_like, V), generator=gen, device=logits.device).clamp_(1e-12, 1)
+                g = logits[rows].float() - torch.log(-torch.log(u))
+                like = g.argmax(1).cpu().numpy().astype(np.int32)
+            else:
+                like = np.zeros(0, np.int32)
+            uni = rng.integers(0, V, size=n - len(like)).astype(np.int32)
+            h = np.concatenate([like, uni])
+            rng.shuffle(h)
+            cols.append(h)
+            offs.append(offs[-1] + len(h))
+        return np.array(offs, np.int32), (np.concatenate(cols).astype(np.int32) if cols
+                                          else np.zeros(0, np.int32))
+    hod, hcd = family(wl.draft_off, wl.draft_logits, False)
+    hot, hct = family(wl.target_off, wl.target_logits, True)
+    return dataclasses.replace(wl, hist_off_d=hod, hist_cols_d=hcd, hist_off_t=hot,
+                               hist_cols_t=hct)

@@ -24,11 +24,13 @@ def to_np(out: dict) -> dict:
 
 def gpu_step(wl, *, device="cuda", window=None, temp_draft=None, temp_target=None, seed=None,
              full_q=False, draft_probs=None, request_base=0, top_k_draft=0, top_p_draft=1.0,
-             top_k_target=0, top_p_target=1.0) -> dict:
+             top_k_target=0, top_p_target=1.0, rep_penalty_draft=1.0,
+             rep_penalty_target=1.0) -> dict:
     inp = tt.device_inputs(wl, device)
     prm = inp["params"]
     prm.top_k_draft, prm.top_p_draft = top_k_draft, top_p_draft
     prm.top_k_target, prm.top_p_target = top_k_target, top_p_target
+    prm.rep_penalty_draft, prm.rep_penalty_target = rep_penalty_draft, rep_penalty_target
     if window is not None:
         prm.window = window
     if temp_draft is not None:

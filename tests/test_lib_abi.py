@@ -44,12 +44,14 @@ def test_library_is_built_for_sm103a():
 
 def test_struct_layouts_match_the_header():
     # sizes/offsets of the C structs under the LP64 ABI (x86-64 and aarch64 alike)
-    assert ctypes.sizeof(binding._Params) == 56
+    assert ctypes.sizeof(binding._Params) == 64
     assert binding._Params.seed.offset == 16 and binding._Params.events.offset == 32
     assert binding._Params.top_k_draft.offset == 40 and binding._Params.top_p_target.offset == 52
+    assert binding._Params.rep_penalty_target.offset == 60
     assert ctypes.sizeof(binding._Logits) == 32 and binding._Logits.row_stride.offset == 16
     assert ctypes.sizeof(binding._Vocab) == 32 and binding._Vocab.n_bytes.offset == 24
-    assert binding._Batch.draft_off.offset == 24 and ctypes.sizeof(binding._Batch) == 72
+    assert binding._Batch.draft_off.offset == 24 and binding._Batch.hist_off_d.offset == 72
+    assert binding._Batch.n_hist_t.offset == 108 and ctypes.sizeof(binding._Batch) == 112
     assert ctypes.sizeof(binding._StepOut) == 80
     assert ctypes.sizeof(binding._Shards) == 24 and binding._Shards.col0.offset == 16
 
