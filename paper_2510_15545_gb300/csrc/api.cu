@@ -153,6 +153,13 @@ cudaError_t launch_pen_sets(const tt_batch* batch, const RowSet& d, const RowSet
   return launch_pen_prep(a, s);
 }
 
+// A nucleus family's row set: top-kNucList lists of its units and partials
+// of all its columns, from which the nucleus kernels find each row's kept set.
+void attach_nucleus(RowSet& r, bool on) {
+  r.nucleus = on ? 1 : 0;
+  if (on) r.top_k = kNucList;
+}
+
 // A family's row set sees its penalty arrays.
 void attach_pen(RowSet& r, bool on, float theta, PenEntry* pen, const int32_t* pbase,
                 const int32_t* pcnt, const int32_t* pstart) {
@@ -463,7 +470,7 @@ tt_status tt_transfer(const tt_batch* batch, const int32_t* map, const tt_logits
   d.d = from_logits ? rowset(draft, ws.part_d, ws.need_d, prm->temp_draft) : no_rows();
   d.d.top_k = kd;
   d.d.cand = ws.cand_d;
-  d.d.nucleus = nd ? 1 : 0;
+  attach_nucleus(d.d, nd);
   attach_pen(d.d, pd, prm->rep_penalty_draft, ws.pen_d, ws.pbase_d, ws.pcnt_d, ws.pstart_d);
   d.status_p = pd ? ws.pstatus : nullptr;
   d.top_p_d = prm->top_p_draft;
@@ -579,7 +586,7 @@ tt_status tt_verify(const tt_batch* batch, const float* q_hat, const tt_logits* 
   r.t = rowset(target, ws.part_t, nullptr, prm->temp_target);
   r.t.top_k = kt;
   r.t.cand = ws.cand_t;
-  r.t.nucleus = nt ? 1 : 0;
+  attach_nucleus(r.t, nt);
   attach_pen(r.t, pt, prm->rep_penalty_target, ws.pen_t, ws.pbase_t, ws.pcnt_t, ws.pstart_t);
   if (pt && (e = launch_pen_sets(batch, no_rows(), r.t, false, true, nullptr, tcols, ws, s)) !=
                 cudaSuccess)
@@ -695,10 +702,10 @@ tt_status tt_step(const tt_batch* batch, const tt_vocab* vd, const tt_vocab* vt,
   r.rows_d = from_logits ? batch->n_draft : 0;
   r.t.top_k = kt;
   r.t.cand = ws.cand_t;
-  r.t.nucleus = nt ? 1 : 0;
+  attach_nucleus(r.t, nt);
   r.d.top_k = kd;
   r.d.cand = ws.cand_d;
-  r.d.nucleus = nd ? 1 : 0;
+  attach_nucleus(r.d, nd);
   attach_pen(r.d, pd, prm->rep_penalty_draft, ws.pen_d, ws.pbase_d, ws.pcnt_d, ws.pstart_d);
   attach_pen(r.t, pt, prm->rep_penalty_target, ws.pen_t, ws.pbase_t, ws.pcnt_t, ws.pstart_t);
   r.B = batch->B;

@@ -496,7 +496,9 @@ __global__ void __launch_bounds__(kFThreads) kept_kernel(KeptArgs a) {
   __shared__ Cand s_scr[kFWarps][kRowCap];
   __shared__ Cand s_top[kFWarps][TT_MAX_TOP_K];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t rows_d = a.d.top_k > 0 ? a.rows_d : 0, rows_t = a.t.top_k > 0 ? a.rows_t : 0;
+  // (nucleus families' lists are read by the nucleus kernel)
+  const int64_t rows_d = a.d.top_k > 0 && !a.d.nucleus ? a.rows_d : 0;
+  const int64_t rows_t = a.t.top_k > 0 && !a.t.nucleus ? a.rows_t : 0;
   const int64_t total = rows_d + rows_t;
   const int64_t w0 = int64_t(blockIdx.x) * kFWarps + warp, stride = int64_t(gridDim.x) * kFWarps;
   grid_dependency_wait();  // the lists (and the need flags) come from earlier kernels
@@ -791,7 +793,8 @@ cudaError_t preload_filter() {
 }
 
 cudaError_t launch_kept(const KeptArgs& args, cudaStream_t stream, int sm_count, bool pdl) {
-  const int64_t rows = (args.d.top_k > 0 ? args.rows_d : 0) + (args.t.top_k > 0 ? args.rows_t : 0);
+  const int64_t rows = (args.d.top_k > 0 && !args.d.nucleus ? args.rows_d : 0) +
+                       (args.t.top_k > 0 && !args.t.nucleus ? args.rows_t : 0);
   if (rows == 0) return cudaSuccess;
   const int64_t blocks = std::min<int64_t>((rows + kFWarps - 1) / kFWarps, int64_t(sm_count) * 8);
   cudaLaunchConfig_t cfg = {};

@@ -169,34 +169,15 @@ __global__ void __launch_bounds__(kNT) nucleus_kernel(KeptArgs a) {
     const int vec = dt == TT_F32 ? 4 : 8;  // logits per 16-byte vector
     const int nvec = V / vec;              // whole vectors (rows start on 16 bytes)
 
-    // the row maximum: chunk maxima of the partials, and the scored column
-    // (left out of a target row's partials) -- the largest of them
+    // only the rows the merge kernel could not settle from their lists
+    if (head->n != -1) continue;
+    // the row maximum from the partials (nucleus rows' partials hold every column)
     float M = -INFINITY;
     for (int c = tid; c < nch; c += kNT) M = fmaxf(M, S.part[r * nch + c].m);
-    if (tgt && a.target_off && a.B > 0) {
-      // the scored column of target row r: request b owns rows t0 + b .. t1 + b
-      int lo = 0, hi = a.B - 1;
-      while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (int64_t(a.target_off[mid]) + mid <= r) lo = mid;
-        else hi = mid - 1;
-      }
-      const int t0 = a.target_off[lo], t1 = a.target_off[lo + 1];
-      const int64_t j = r - (int64_t(t0) + lo);
-      if (tid == 0 && j >= 0 && j < t1 - t0 && t1 <= a.n_target) {
-        const int c = a.target_cols[t0 + j];
-        if (c >= 0 && c < V) M = fmaxf(M, __fmul_rn(load_dt(row, dt, c), scale));
-      }
-    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
     __syncthreads();
     if (lane == 0) sm.wmax[warp] = __float_as_uint(M) ^ (M < 0.f ? 0xffffffffu : 0x80000000u);
-    for (int c = tid; c < nch; c += kNT) sm.cacc[c] = 0ull;
-    if (tid == 0) {
-      sm.before = 0ull;
-      sm.n_gz = 0;
-    }
     __syncthreads();
     {
       unsigned long long best = 0;
@@ -236,11 +217,19 @@ __global__ void __launch_bounds__(kNT) nucleus_kernel(KeptArgs a) {
 
     // ------------------------------------- the crossing bucket, level by level
     Path cross;
-    cross.b[0] = cross.b[1] = cross.b[2] = 0;
     int level = 0;
     unsigned long long total = 0ull;
     double thr = 0.0;
     bool all_kept = false;
+    float tau = -INFINITY;
+    int tau_col = 0x7fffffff;  // all_kept: every column ranks before (tau, tau_col)
+    for (int c = tid; c < nch; c += kNT) sm.cacc[c] = 0ull;
+    if (tid == 0) {
+      sm.before = 0ull;
+      sm.n_gz = 0;
+    }
+    __syncthreads();
+    cross.b[0] = cross.b[1] = cross.b[2] = 0;
     for (; level < kLevels; ++level) {
       for (int i = tid; i < kBuckets; i += kNT) {
         sm.cnt[i] = 0u;
@@ -324,8 +313,6 @@ __global__ void __launch_bounds__(kNT) nucleus_kernel(KeptArgs a) {
       }
     });
     __syncthreads();
-    float tau = -INFINITY;
-    int tau_col = 0x7fffffff;  // all_kept: every column ranks before (tau, tau_col)
     const int ng = sm.n_gz;
     if (!all_kept) {
       if (ng <= kGather) {
@@ -670,12 +657,156 @@ __global__ void __launch_bounds__(kNT) decide_nucleus_kernel(DecideArgs a) {
 
 static_assert(sizeof(NucSmem) <= 48 * 1024, "fits the default dynamic shared memory");
 
+constexpr int kMWarps = 8;   // warps of a merge CTA (one nucleus row each)
+constexpr int kMLists = 4;   // unit lists a lane owns: rows of up to 128 units
+
+__device__ __forceinline__ bool cand_first(float v1, int c1, float v2, int c2) {
+  return v1 > v2 || (v1 == v2 && c1 < c2);
+}
+
+// The kept set of a nucleus row from its unit lists, one warp per row: the
+// lists (each unit's kNucList largest columns, in order) are merged k-way, and
+// columns are kept in the merged order while the mass before them is below
+// top_p of the row's total (from the partials, which hold every column). The
+// walk stops at the cut; a list consumed to its end while the cut is not yet
+// reached may hide further columns of its unit, and the row is left to
+// nucleus_kernel (head n = -1). Also rows of more than 32 * kMLists units.
+__global__ void __launch_bounds__(kMWarps * 32) nucleus_merge_kernel(KeptArgs a) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t rows_d = a.d.nucleus ? a.rows_d : 0, rows_t = a.t.nucleus ? a.rows_t : 0;
+  const int64_t total = rows_d + rows_t;
+  grid_dependency_wait();  // the lists and partials come from the row pass
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int Ls = cand_stride(kNucList);
+  for (int64_t w = int64_t(blockIdx.x) * kMWarps + warp; w < total;
+       w += int64_t(gridDim.x) * kMWarps) {
+    const bool tgt = w >= rows_d;
+    const int64_t r = tgt ? w - rows_d : w;
+    const RowSet& S = tgt ? a.t : a.d;
+    if (!tgt && S.need && S.need[r] == 0) continue;
+    KeptHead* head = (tgt ? a.head_t : a.head_d) + r;
+    float* um = (tgt ? a.um_t : a.um_d) + r * S.nch;
+    const int nch = S.nch, nl = S.nlist, cps = S.unit_cols / kChunk;
+    const float scale = S.scale, top_p = tgt ? a.top_p_t : a.top_p_d;
+    const Partial* part = S.part + r * nch;
+    // the row's maximum and total 2^(z * scale - M), compensated
+    float M = -INFINITY;
+    for (int c = lane; c < nch; c += 32) M = fmaxf(M, part[c].m);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    F2 T = {0.f, 0.f};
+    if (M > -INFINITY && isfinite(M))
+      for (int c = lane; c < nch; c += 32) {
+        const Partial q = part[c];
+        if (q.m > -INFINITY) T = f2_add(T, F2{q.s * ex2_approx(q.m - M), 0.f});
+      }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+      T = f2_add(T, F2{__shfl_xor_sync(0xffffffffu, T.hi, o), __shfl_xor_sync(0xffffffffu, T.lo, o)});
+    if (!isfinite(M) || !(T.hi > 0.f) || !isfinite(T.hi)) {
+      if (lane == 0) *head = KeptHead{NAN, 0, NAN, -1, M, 0.f};
+      continue;
+    }
+    if (nl > 32 * kMLists) {
+      if (lane == 0) head->n = -1;
+      continue;
+    }
+    const F2 thr = f2_mul_f(T, top_p);
+    const Cand* lists = S.cand + r * int64_t(nl) * Ls;
+    const Cand pad = {-INFINITY, -1};
+    Cand cur[kMLists], nxt[kMLists];
+    int pos[kMLists];
+    float acc[kMLists][2];
+#pragma unroll
+    for (int i = 0; i < kMLists; ++i) {
+      const int u = lane + 32 * i;
+      cur[i] = u < nl ? lists[int64_t(u) * Ls] : pad;
+      nxt[i] = u < nl ? lists[int64_t(u) * Ls + 1] : pad;
+      pos[i] = 1;  // list index of nxt
+      acc[i][0] = acc[i][1] = 0.f;
+    }
+    F2 before = {0.f, 0.f};
+    float tau = -INFINITY;
+    int tau_col = 0x7fffffff, n = 0;
+    bool need_exact = false;
+    for (;;) {
+      // the lane's best current head, then the warp's
+      float bv = -INFINITY;
+      int bc = 0x7fffffff, bi = -1;
+#pragma unroll
+      for (int i = 0; i < kMLists; ++i)
+        if (cur[i].c >= 0 && (bi < 0 || cand_first(cur[i].v, cur[i].c, bv, bc))) {
+          bv = cur[i].v;
+          bc = cur[i].c;
+          bi = i;
+        }
+      float wv = bv;
+      int wc = bc;
+      bool f = bi >= 0;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, wv, o);
+        const int oc = __shfl_xor_sync(0xffffffffu, wc, o);
+        const bool of = __shfl_xor_sync(0xffffffffu, int(f), o) != 0;
+        if (of && (!f || cand_first(ov, oc, wv, wc))) {
+          wv = ov;
+          wc = oc;
+          f = true;
+        }
+      }
+      if (!f || !f2_lt(before, thr)) break;  // every list consumed, or the cut is reached
+      const float e = exp2_scaled(wv, scale, M);
+      before = f2_add(before, F2{e, 0.f});
+      tau = wv;
+      tau_col = wc;
+      ++n;
+      // the owner (columns are distinct) books the mass and advances its list
+      bool exhausted = false;
+      if (bi >= 0 && bc == wc && bv == wv) {
+#pragma unroll
+        for (int i = 0; i < kMLists; ++i)
+          if (i == bi) {
+            const int u = lane + 32 * i;
+            acc[i][(wc / kChunk - u * cps) & 1] += e;
+            cur[i] = nxt[i];
+            ++pos[i];
+            nxt[i] = pos[i] < kNucList ? lists[int64_t(u) * Ls + pos[i]] : pad;
+            // the list's last entry taken: its unit may hold more columns
+            exhausted = pos[i] > kNucList;
+          }
+      }
+      if (__any_sync(0xffffffffu, exhausted) && f2_lt(before, thr)) {
+        need_exact = true;
+        break;
+      }
+    }
+    if (need_exact) {
+      if (lane == 0) head->n = -1;
+      continue;
+    }
+    const float Sk = __fadd_rn(before.hi, before.lo);
+    const float inv_s = __frcp_rn(Sk);
+#pragma unroll
+    for (int i = 0; i < kMLists; ++i) {
+      const int u = lane + 32 * i;
+      if (u >= nl) continue;
+      for (int c = 0; c < cps; ++c) {
+        const int ch = u * cps + c;
+        if (ch < nch) um[ch] = acc[i][c] * inv_s;
+      }
+    }
+    if (lane == 0)
+      *head = KeptHead{(M + lg2_approx(Sk)) * 0.6931471805599453f, n, tau, tau_col, M, inv_s};
+  }
+}
+
 }  // namespace
 
 cudaError_t preload_nucleus() {
   cudaFuncAttributes fa;
-  const cudaError_t e = cudaFuncGetAttributes(&fa, nucleus_kernel);
+  cudaError_t e = cudaFuncGetAttributes(&fa, nucleus_kernel);
   if (e != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, nucleus_merge_kernel)) != cudaSuccess) return e;
   return cudaFuncGetAttributes(&fa, decide_nucleus_kernel);
 }
 
@@ -697,6 +828,22 @@ cudaError_t launch_decide_nucleus(const DecideArgs& args, cudaStream_t stream, b
 cudaError_t launch_nucleus(const KeptArgs& args, cudaStream_t stream, int sm_count, bool pdl) {
   const int64_t rows = (args.d.nucleus ? args.rows_d : 0) + (args.t.nucleus ? args.rows_t : 0);
   if (rows == 0) return cudaSuccess;
+  {  // the merge kernel settles most rows from their lists
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(std::min<int64_t>((rows + kMWarps - 1) / kMWarps,
+                                                  int64_t(sm_count) * 8)));
+    cfg.blockDim = dim3(kMWarps * 32);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, nucleus_merge_kernel, args);
+    if (e != cudaSuccess) return e;
+  }
+  // nucleus_kernel (below) takes the rows it leaves, from their logits
   const int64_t blocks = std::min<int64_t>(rows, int64_t(sm_count) * 2);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(unsigned(blocks));

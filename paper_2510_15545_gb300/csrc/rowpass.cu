@@ -21,6 +21,7 @@
 
 #include "tt_device.cuh"
 #include "tt_launch.h"
+#include "tt_f2.cuh"
 
 namespace tt {
 
@@ -114,9 +115,6 @@ __device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32
           smem_u32(dst)),
       "l"(src), "r"(bytes), "r"(smem_u32(bar))
       : "memory");
-}
-__device__ __forceinline__ void grid_dependency_wait() {
-  asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 __device__ __forceinline__ void grid_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -369,6 +367,55 @@ __device__ __forceinline__ float vec_max(const uint4& w) {
     const uint32_t m = max_bf16x2(max_bf16x2(w.x, w.y), max_bf16x2(w.z, w.w));
     return fmaxf(__uint_as_float(m << 16), __uint_as_float(m & 0xffff0000u));
   }
+}
+
+// Partial of one chunk of a nucleus row (all its columns, the scored one
+// included) from a unit held in shared memory plus its ragged tail read
+// directly: the chunk's largest z * scale and the sum of 2^(s - m), each
+// 16-byte vector's terms added plainly and the vectors' sums in compensated
+// pairs (TwoSum), so that the row's normaliser -- against which the top-p cut
+// is placed -- stays within a few 1e-7 of exact.
+template <int DT>
+__device__ __forceinline__ Partial nuc_chunk_partial(const char* stage, const Desc& d,
+                                                     const char* row, float scale, int c,
+                                                     int lane) {
+  constexpr int VEC = DT == TT_F32 ? 4 : 8;
+  const int lo = c * kChunk;                       // first column of the chunk in the unit
+  const int hi = min(d.n, lo + kChunk);            // its end
+  const int smem_hi = min(hi, d.n_smem);           // columns held in shared memory
+  const int col0 = d.chunk * kChunk;
+  const uint4* sv = reinterpret_cast<const uint4*>(stage);
+  const int v0 = lo / VEC, v1 = smem_hi / VEC;     // whole vectors (lo is a multiple of VEC)
+  const int t = smem_hi + lane;                    // the ragged tail: one column per lane
+  const float zt = (t < hi && t >= d.n_smem) ? load_logit<DT>(row, int64_t(col0) + t) : -INFINITY;
+  float zmax = zt;
+  for (int v = v0 + lane; v < v1; v += 32) zmax = fmaxf(zmax, vec_max<DT>(sv[v]));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) zmax = fmaxf(zmax, __shfl_xor_sync(0xffffffffu, zmax, o));
+  const float m = __fmul_rn(zmax, scale);
+  float hs = 0.f, ls = 0.f;  // compensated sum (hi, lo)
+  if (m > -INFINITY) {
+    auto add = [&](float x) {
+      const float sx = __fadd_rn(hs, x), bb = __fsub_rn(sx, hs);
+      ls = __fadd_rn(ls, __fadd_rn(__fsub_rn(hs, __fsub_rn(sx, bb)), __fsub_rn(x, bb)));
+      hs = sx;
+    };
+    for (int v = v0 + lane; v < v1; v += 32) {  // one vector's terms summed plainly
+      const uint4 w = sv[v];
+      float blk = 0.f;
+#pragma unroll
+      for (int q = 0; q < VEC; ++q) blk += ex2_approx(fmaf(lane_elem<DT>(w, q), scale, -m));
+      add(blk);
+    }
+    if (zt > -INFINITY) add(ex2_approx(fmaf(zt, scale, -m)));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float oh = __shfl_xor_sync(0xffffffffu, hs, o), ol = __shfl_xor_sync(0xffffffffu, ls, o);
+      ls = __fadd_rn(ls, ol);
+      add(oh);
+    }
+  }
+  return Partial{m, __fadd_rn(hs, ls)};
 }
 
 // One consumer warp writes the top-K (value, column) list of one unit held in
@@ -642,9 +689,10 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
           }
           if (!cached_need) return true;  // no target position maps to this row
         }
-        d.req = S->pen ? req_lookup(tgt ? a.target_off : a.draft_off, a.B, tgt,
-                                    tgt ? &rcur_t : &rcur_d, row)
-                       : -1;
+        // (penalized families have top-k lists: the list-selecting variant only)
+        d.req = (SEL && S->pen) ? req_lookup(tgt ? a.target_off : a.draft_off, a.B, tgt,
+                                             tgt ? &rcur_t : &rcur_d, row)
+                                : -1;
         d.chunk = unit * cps;
         const int c0 = d.chunk * kChunk;
         d.n = min(cps * kChunk, S->V - c0);
@@ -791,6 +839,16 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
         select_unit<DTT>(stage, d, V, lane, S.top_k, scratch, out, drop);
       } else {
         select_unit<DTD>(stage, d, V, lane, S.top_k, scratch, out, drop);
+      }
+      if (S.nucleus && d.n > 0) {  // nucleus rows: also the partials of the unit's chunks
+#pragma unroll 1
+        for (int c = 0; c < cps && c * kChunk < d.n; ++c) {
+          const Partial pc =
+              (d.set ? DTT : DTD) == TT_F32
+                  ? nuc_chunk_partial<TT_F32>(stage, d, V.row(d), S.scale, c, lane)
+                  : nuc_chunk_partial<TT_BF16>(stage, d, V.row(d), S.scale, c, lane);
+          if (lane == 0) S.part[d.row * S.nch + d.chunk + c] = pc;
+        }
       }
       if (lane == 0 && !(blockIdx.x == 0 && it == a.stall_stage))
         mbar_arrive(&empty[s]);  // the stage's bytes are consumed

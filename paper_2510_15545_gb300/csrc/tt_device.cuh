@@ -54,6 +54,9 @@ struct KeptHead {
   float inv_s;     // 1 / (sum over kept columns of 2^(z * scale - M))
 };
 
+// List size of the nucleus rows' units (top-p without top-k).
+constexpr int kNucList = 32;
+
 // A column of a request's repetition-penalty set (its history and sequence
 // tokens): the column and the first sequence position holding it (-1 when the
 // history holds it), so that a row at position j penalizes it when first < j.
@@ -124,6 +127,9 @@ __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_d
     return r;
   };
   const size_t rows_t = size_t(n_target) + B;
+  // nucleus families keep top-kNucList lists of their units
+  if (nuc_d && k_d <= 0) k_d = kNucList;
+  if (nuc_t && k_t <= 0) k_t = kNucList;
   w.part_d = reinterpret_cast<Partial*>(take(sizeof(Partial) * size_t(n_draft) * n_chunks(V_d)));
   w.part_t = reinterpret_cast<Partial*>(take(sizeof(Partial) * rows_t * n_chunks(V_t)));
   w.need_d = reinterpret_cast<uint8_t*>(take(size_t(n_draft)));
