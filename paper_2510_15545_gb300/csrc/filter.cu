@@ -350,9 +350,56 @@ __device__ void row_topk_small(const Cand* lists, int nl, int K, int Ls, int lan
   __syncwarp();
 }
 
+// The top-K of a row of two unit lists (a 4096-column fp32 row): the first K
+// places of the merge of two ordered lists. Lane i finds by a binary search
+// over the merge path how many of its first i places list A fills; the
+// entries come from the two lists held one per lane and fetched by shuffles.
+__device__ void row_topk_two(const Cand* lists, int K, int Ls, int lane, Cand* top) {
+  const Cand pad = {-INFINITY, -1};
+  const Cand A = lane < K ? lists[lane] : pad;
+  const Cand Bv = lane < K ? lists[Ls + lane] : pad;
+  // list entries past their real ones (pads) rank last
+  auto a_at = [&](int x) -> Cand {
+    const float v = __shfl_sync(0xffffffffu, A.v, x & 31);
+    const int c = __shfl_sync(0xffffffffu, A.c, x & 31);
+    return Cand{v, c};
+  };
+  auto b_at = [&](int x) -> Cand {
+    const float v = __shfl_sync(0xffffffffu, Bv.v, x & 31);
+    const int c = __shfl_sync(0xffffffffu, Bv.c, x & 31);
+    return Cand{v, c};
+  };
+  auto before = [&](const Cand& x, const Cand& y) -> bool {  // x ranks before y
+    if (x.c < 0) return false;
+    if (y.c < 0) return true;
+    return cand_before(x.v, x.c, y.v, y.c);
+  };
+  // place i: a = entries of A among the first i places (the merge path)
+  const int i = lane;
+  int lo = max(0, i - K), hi = min(i, K);
+#pragma unroll 1
+  for (int step = 0; step < 6; ++step) {  // lo < hi for at most log2(K) + 1 steps
+    const int mid = (lo + hi + 1) >> 1;
+    const bool active = lo < hi;
+    // with mid entries of A taken, A[mid - 1] must rank before B[i - mid]
+    const Cand am = a_at(mid - 1), bm = b_at(i - mid);
+    if (active) {
+      if (i - mid >= K || before(am, bm)) lo = mid;
+      else hi = mid - 1;
+    }
+  }
+  const int a = lo, b = i - a;
+  const Cand ca = a_at(a), cb = b_at(b);
+  const bool take_a = a < K && (b >= K || before(ca, cb));
+  const Cand pick = take_a ? ca : cb;
+  if (lane < K) top[lane] = (take_a ? a < K : b < K) && pick.c >= 0 ? pick : pad;
+  __syncwarp();
+}
+
 __device__ __forceinline__ void row_topk(const Cand* lists, int nch, int K, int Ls, int lane,
                                          Cand* scr, Cand* top) {
-  if (nch * K <= 64) row_topk_small(lists, nch, K, Ls, lane, scr, top);
+  if (nch == 2) row_topk_two(lists, K, Ls, lane, top);
+  else if (nch * K <= 64) row_topk_small(lists, nch, K, Ls, lane, scr, top);
   else if (nch <= 32 * kMergeLists) row_topk_thresh(lists, nch, K, Ls, lane, scr, top);
   else row_topk_wide(lists, nch, K, Ls, lane, scr, top);
 }
@@ -492,7 +539,7 @@ __device__ __forceinline__ float kept_prob(int col, float prob, int c) {
 // draft rows skipped): the row's top-K from its unit lists, then its kept set
 // as K (probability, column) entries in value order, unused ones (0, -1),
 // and the header (lse, kept count).
-__global__ void __launch_bounds__(kFThreads) kept_kernel(KeptArgs a) {
+__global__ void __launch_bounds__(kFThreads, 4) kept_kernel(KeptArgs a) {
   __shared__ Cand s_scr[kFWarps][kRowCap];
   __shared__ Cand s_top[kFWarps][TT_MAX_TOP_K];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;

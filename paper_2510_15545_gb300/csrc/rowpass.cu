@@ -53,7 +53,7 @@ constexpr int kCandCap = 128;   // top-k candidates of one unit a warp keeps in 
 constexpr int kDirectCap = 32;  // vectors at or above tau1 taken directly (more: tau2)
 constexpr int kLevel2Cap = 64;  // vector maxima ranked by counting (more: radix search)
 
-template <int DTD, int DTT, bool SEL>
+template <int DTD, int DTT, int SEL>
 struct Ring {
   static constexpr int kStageBytes = kChunk * 4;  // one fp32 chunk or two bf16 chunks
   static constexpr int kCpsD = DTD == TT_F32 ? 1 : 2;  // chunks per stage, draft rows
@@ -618,7 +618,7 @@ __device__ void select_unit(const char* stage, const Desc& d, const RowView& S, 
   __syncwarp();  // the scratch is free for the next unit
 }
 
-template <int DTD, int DTT, bool SEL>
+template <int DTD, int DTT, int SEL>
 __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
   using R = Ring<DTD, DTT, SEL>;
   extern __shared__ __align__(128) char smem[];
@@ -690,9 +690,9 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
           if (!cached_need) return true;  // no target position maps to this row
         }
         // (penalized families have top-k lists: the list-selecting variant only)
-        d.req = (SEL && S->pen) ? req_lookup(tgt ? a.target_off : a.draft_off, a.B, tgt,
-                                             tgt ? &rcur_t : &rcur_d, row)
-                                : -1;
+        d.req = (SEL == 2 && S->pen) ? req_lookup(tgt ? a.target_off : a.draft_off, a.B, tgt,
+                                                  tgt ? &rcur_t : &rcur_d, row)
+                                     : -1;
         d.chunk = unit * cps;
         const int c0 = d.chunk * kChunk;
         d.n = min(cps * kChunk, S->V - c0);
@@ -828,10 +828,12 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       Cand* out = S.cand + (d.row * S.nlist + d.chunk / cps) * cand_stride(S.top_k);
       const RowView V = {a, S.scale};
       uint32_t drop = 0u;
-      if (S.pen && d.req >= 0) {
-        char* wstage = stages + size_t(s) * R::kStageBytes;
-        drop = (d.set ? DTT : DTD) == TT_F32 ? mask_penalized<TT_F32>(wstage, d, S, cps, lane)
-                                             : mask_penalized<TT_BF16>(wstage, d, S, cps, lane);
+      if constexpr (SEL == 2) {
+        if (S.pen && d.req >= 0) {
+          char* wstage = stages + size_t(s) * R::kStageBytes;
+          drop = (d.set ? DTT : DTD) == TT_F32 ? mask_penalized<TT_F32>(wstage, d, S, cps, lane)
+                                               : mask_penalized<TT_BF16>(wstage, d, S, cps, lane);
+        }
       }
       if constexpr (DTD == DTT) {
         select_unit<DTT>(stage, d, V, lane, S.top_k, scratch, out, drop);
@@ -840,14 +842,16 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
       } else {
         select_unit<DTD>(stage, d, V, lane, S.top_k, scratch, out, drop);
       }
-      if (S.nucleus && d.n > 0) {  // nucleus rows: also the partials of the unit's chunks
+      if constexpr (SEL == 2) {
+        if (S.nucleus && d.n > 0) {  // nucleus rows: also the partials of the unit's chunks
 #pragma unroll 1
-        for (int c = 0; c < cps && c * kChunk < d.n; ++c) {
-          const Partial pc =
-              (d.set ? DTT : DTD) == TT_F32
-                  ? nuc_chunk_partial<TT_F32>(stage, d, V.row(d), S.scale, c, lane)
-                  : nuc_chunk_partial<TT_BF16>(stage, d, V.row(d), S.scale, c, lane);
-          if (lane == 0) S.part[d.row * S.nch + d.chunk + c] = pc;
+          for (int c = 0; c < cps && c * kChunk < d.n; ++c) {
+            const Partial pc =
+                (d.set ? DTT : DTD) == TT_F32
+                    ? nuc_chunk_partial<TT_F32>(stage, d, V.row(d), S.scale, c, lane)
+                    : nuc_chunk_partial<TT_BF16>(stage, d, V.row(d), S.scale, c, lane);
+            if (lane == 0) S.part[d.row * S.nch + d.chunk + c] = pc;
+          }
         }
       }
       if (lane == 0 && !(blockIdx.x == 0 && it == a.stall_stage))
@@ -901,13 +905,13 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
   }
 }
 
-template <int DTD, int DTT, bool SEL>
+template <int DTD, int DTT, int SEL>
 int& resident_per_sm() {
   static int per_sm = 0;
   return per_sm;
 }
 
-template <int DTD, int DTT, bool SEL>
+template <int DTD, int DTT, int SEL>
 cudaError_t preload_t() {
   using R = Ring<DTD, DTT, SEL>;
   cudaError_t e = cudaFuncSetAttribute(rowpass_kernel<DTD, DTT, SEL>,
@@ -925,7 +929,7 @@ cudaError_t preload_t() {
   return cudaSuccess;
 }
 
-template <int DTD, int DTT, bool SEL>
+template <int DTD, int DTT, int SEL>
 cudaError_t launch_rowpass_t(const RowPassArgs& a, cudaStream_t stream, int sm_count, bool pdl) {
   using R = Ring<DTD, DTT, SEL>;
   const int per_sm = resident_per_sm<DTD, DTT, SEL>();
@@ -949,14 +953,20 @@ cudaError_t launch_rowpass_t(const RowPassArgs& a, cudaStream_t stream, int sm_c
 
 template <int DTD, int DTT>
 cudaError_t preload_pair() {
-  cudaError_t e = preload_t<DTD, DTT, false>();
-  return e != cudaSuccess ? e : preload_t<DTD, DTT, true>();
+  cudaError_t e = preload_t<DTD, DTT, 0>();
+  if (e == cudaSuccess) e = preload_t<DTD, DTT, 1>();
+  return e != cudaSuccess ? e : preload_t<DTD, DTT, 2>();
 }
 
+// Variants: 0 partials only; 1 top-k lists for filtered families; 2 lists with
+// the repetition penalty's masking and the nucleus rows' partials (kept apart
+// so that plain filtered rows run the smaller consumer loop).
 template <int DTD, int DTT>
 cudaError_t launch_pair(const RowPassArgs& a, cudaStream_t stream, int sm_count, bool pdl) {
-  if (a.d.top_k > 0 || a.t.top_k > 0) return launch_rowpass_t<DTD, DTT, true>(a, stream, sm_count, pdl);
-  return launch_rowpass_t<DTD, DTT, false>(a, stream, sm_count, pdl);
+  if (a.d.pen || a.t.pen || a.d.nucleus || a.t.nucleus)
+    return launch_rowpass_t<DTD, DTT, 2>(a, stream, sm_count, pdl);
+  if (a.d.top_k > 0 || a.t.top_k > 0) return launch_rowpass_t<DTD, DTT, 1>(a, stream, sm_count, pdl);
+  return launch_rowpass_t<DTD, DTT, 0>(a, stream, sm_count, pdl);
 }
 
 }  // namespace
