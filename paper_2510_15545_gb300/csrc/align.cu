@@ -126,7 +126,8 @@ struct PairSmem {
   uint64_t* tok;  // [K + M] packed bytes (valid when len <= 8)
   int32_t* diag;  // [3 * (K + 2)] rotating anti-diagonals, indexed by i
   uint32_t* path; // [K + M] backtracked cells (i << 16 | j), reverse order
-  uint8_t* tile;  // [K * TW] cost (255: 255 or more, recomputed), then direction
+  uint8_t* tile;  // [K * TW / 2] 4-bit cells, two per byte, row i at (i - 1) * tw:
+                  // cost (15: 15 or more, recomputed), then direction
   uint16_t* len;  // [K + M] token byte lengths
 };
 
@@ -140,7 +141,7 @@ __device__ __forceinline__ PairSmem carve(char* base, int K, int M, int TW) {
   s.path = reinterpret_cast<uint32_t*>(base + off);
   off += sizeof(uint32_t) * (K + M);
   s.tile = reinterpret_cast<uint8_t*>(base + off);
-  off += (size_t(K) * TW + 15) & ~size_t(15);
+  off += (size_t(K) * TW / 2 + 1 + 15) & ~size_t(15);
   s.len = reinterpret_cast<uint16_t*>(base + off);
   return s;
 }
@@ -223,20 +224,22 @@ __device__ __forceinline__ void align_pair(const AlignArgs& a, int b, char* regi
     return lev_rows(a.vd.bytes + a.vd.offsets[di], ld, a.vt.bytes + a.vt.offsets[ti], lt);
   };
 
-  // 1. banded local costs, one byte each (a cost of 255 or more is stored as
-  // 255 and recomputed in the sweep); row i (1-based) holds j = jlo(i) .. jhi(i).
-  // Each lane takes two cells per step: when both are short tokens their two
-  // bit-parallel evaluations run interleaved.
-  for (int idx = lane; idx < k * tw; idx += 64) {
+  // 1. banded local costs, four bits each (a cost of 15 or more -- possible
+  // only for tokens of more than 8 bytes -- is stored as 15 and recomputed in
+  // the sweep); row i (1-based) holds j = jlo(i) .. jhi(i) at (i - 1) * tw.
+  // Each lane takes the two cells of one byte per step: when both are short
+  // tokens their two bit-parallel evaluations run interleaved.
+  for (int q = lane; 2 * q < k * tw; q += 32) {
     int ii[2], cc[2], jj[2];
     bool ok[2];
+    ii[0] = (2 * q) / tw + 1;
+    cc[0] = 2 * q - (ii[0] - 1) * tw;
+    ii[1] = cc[0] + 1 == tw ? ii[0] + 1 : ii[0];
+    cc[1] = cc[0] + 1 == tw ? 0 : cc[0] + 1;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const int id = idx + 32 * h;
-      ii[h] = id / tw + 1;
-      cc[h] = id - (ii[h] - 1) * tw;
       jj[h] = max(1, ii[h] - W0) + cc[h];
-      ok[h] = id < k * tw && jj[h] <= min(m, ii[h] + W0);
+      ok[h] = 2 * q + h < k * tw && jj[h] <= min(m, ii[h] + W0);
     }
     int d[2] = {0, 0};
     const bool short0 = ok[0] && sm.len[ii[0] - 1] <= 8 && sm.len[k + jj[0] - 1] <= 8;
@@ -260,10 +263,19 @@ __device__ __forceinline__ void align_pair(const AlignArgs& a, int b, char* regi
       if (ok[0]) d[0] = token_cost(ii[0], jj[0]);
       if (ok[1]) d[1] = token_cost(ii[1], jj[1]);
     }
-#pragma unroll
-    for (int h = 0; h < 2; ++h)
-      if (ok[h]) sm.tile[size_t(ii[h] - 1) * TW + cc[h]] = uint8_t(min(d[h], 255));
+    sm.tile[q] = uint8_t((ok[0] ? min(d[0], 15) : 0) | ((ok[1] ? min(d[1], 15) : 0) << 4));
   }
+  __syncwarp();  // every cost is in the tile before the sweep reads it
+
+  // A cell's cost nibble and, once its predecessor is chosen, its direction:
+  // set by one XOR on the 32-bit word holding it (the other nibbles of the
+  // word belong to cells of other diagonals, which other lanes may be setting).
+  uint32_t* tile32 = reinterpret_cast<uint32_t*>(sm.tile);
+  auto cell_of = [&](int i, int j) { return (i - 1) * tw + (j - max(1, i - W0)); };
+  auto nibble = [&](int p) { return (sm.tile[p >> 1] >> ((p & 1) * 4)) & 15; };
+  auto set_dir = [&](int p, int stored, int dir) {
+    atomicXor(&tile32[p >> 3], uint32_t(stored ^ dir) << ((p & 7) * 4));
+  };
 
   // 2. anti-diagonal sweep. A diagonal s = i + j holds the cells
   // i = lo(s) .. hi(s); each depends on the two diagonals before it.
@@ -290,11 +302,11 @@ __device__ __forceinline__ void align_pair(const AlignArgs& a, int b, char* regi
         int best = (sd >= 0 && sd < n2) ? dg0 : kInf, dir = 0;
         if (up < best) { best = up; dir = 1; }
         if (left < best) { best = left; dir = 2; }
-        uint8_t* cell = sm.tile + size_t(i - 1) * TW + (j - max(1, i - W0));
-        int cost = *cell;
-        if (cost == 255) cost = token_cost(i, j);
+        const int p = cell_of(i, j);
+        const int stored = nibble(p);
+        const int cost = stored == 15 ? token_cost(i, j) : stored;
         v = best >= kInf ? kInf : best + cost;
-        *cell = uint8_t(dir);
+        set_dir(p, stored, dir);
       }
       v2 = v1;
       lo2 = lo1;
@@ -325,11 +337,11 @@ __device__ __forceinline__ void align_pair(const AlignArgs& a, int b, char* regi
         int best = dg, dir = 0;
         if (up < best) { best = up; dir = 1; }
         if (left < best) { best = left; dir = 2; }
-        uint8_t* cell = sm.tile + size_t(i - 1) * TW + (j - max(1, i - W0));
-        int cost = *cell;
-        if (cost == 255) cost = token_cost(i, j);
+        const int p = cell_of(i, j);
+        const int stored = nibble(p);
+        const int cost = stored == 15 ? token_cost(i, j) : stored;
         cur[i] = best >= kInf ? kInf : best + cost;
-        *cell = uint8_t(dir);
+        set_dir(p, stored, dir);
       }
       if (lane == 0) {  // guards: neighbours just outside the diagonal read as infinite
         if (lo - 1 >= 0) cur[lo - 1] = kInf;
@@ -346,7 +358,7 @@ __device__ __forceinline__ void align_pair(const AlignArgs& a, int b, char* regi
     int i = k, j = m;
     while (i > 0 && j > 0 && L < k + m) {
       sm.path[L++] = (uint32_t(i) << 16) | uint32_t(j);
-      const int dir = sm.tile[size_t(i - 1) * TW + (j - max(1, i - W0))];
+      const int dir = nibble(cell_of(i, j));
       if (dir == 0) { --i; --j; }
       else if (dir == 1) { --i; }
       else { --j; }
@@ -383,7 +395,7 @@ __device__ __forceinline__ void align_pair(const AlignArgs& a, int b, char* regi
 // Before the row pass, at most one CTA per SM whose warps loop over the pairs
 // (the row pass's CTAs fit beside it and stream target rows while the pairs
 // are aligned); alone, one warp per pair (launch_align).
-__global__ void __launch_bounds__(kAlignWarpsMax * 32)
+__global__ void __launch_bounds__(kAlignWarpsMax * 32, 4)
     align_kernel(AlignArgs a) {
   extern __shared__ __align__(16) char smem_raw[];
   // the row pass may start streaming target rows now; it waits for this grid
@@ -404,7 +416,8 @@ __global__ void __launch_bounds__(kAlignWarpsMax * 32)
 
 size_t align_smem_per_warp(int max_k, int max_m, int tile_w) {
   size_t n = sizeof(uint64_t) * (max_k + max_m) + sizeof(int32_t) * 3 * (max_k + 2) +
-             sizeof(uint32_t) * (max_k + max_m) + ((size_t(max_k) * tile_w + 15) & ~size_t(15)) +
+             sizeof(uint32_t) * (max_k + max_m) +
+             ((size_t(max_k) * tile_w / 2 + 1 + 15) & ~size_t(15)) +
              sizeof(uint16_t) * (max_k + max_m);
   return (n + 15) & ~size_t(15);
 }
@@ -427,13 +440,16 @@ cudaError_t launch_align(const AlignArgs& args, cudaStream_t stream) {
       cudaDeviceGetAttribute(&n_sm[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     n_sm[dev] = 148;
   // A grid followed by the row pass (it zeroes the row pass's work counters)
-  // takes at most one CTA per SM, whose warps loop over the pairs, so that the
-  // row pass's CTAs fit beside it and stream target rows while it runs; an
-  // alignment on its own takes one warp per pair and as many CTAs as fit.
-  const int per_pair = (args.B + args.warps_per_block - 1) / args.warps_per_block;
-  const int blocks = args.work ? std::min(per_pair, n_sm[dev]) : per_pair;
-  const size_t smem = args.smem_per_warp * size_t(args.warps_per_block);
-  align_kernel<<<blocks, args.warps_per_block * 32, smem, stream>>>(args);
+  // takes at most one CTA of at most kAlignWarpsStep warps per SM, whose warps
+  // loop over the pairs, so that three row-pass CTAs fit beside it and stream
+  // target rows while it runs; an alignment on its own takes one warp per pair
+  // and as many CTAs as fit.
+  AlignArgs a = args;
+  if (a.work) a.warps_per_block = std::min(a.warps_per_block, kAlignWarpsStep);
+  const int per_pair = (a.B + a.warps_per_block - 1) / a.warps_per_block;
+  const int blocks = a.work ? std::min(per_pair, n_sm[dev]) : per_pair;
+  const size_t smem = a.smem_per_warp * size_t(a.warps_per_block);
+  align_kernel<<<blocks, a.warps_per_block * 32, smem, stream>>>(a);
   return cudaGetLastError();
 }
 

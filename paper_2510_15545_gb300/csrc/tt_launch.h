@@ -12,6 +12,7 @@ namespace tt {
 struct Partial;
 
 constexpr int kAlignWarpsMax = 8;             // warps (pairs at a time) per align CTA
+constexpr int kAlignWarpsStep = 4;            // the same inside tt_step, beside the row pass
 constexpr int kAlignSmemMax = 200 * 1024;     // dynamic shared memory cap of one align CTA
 constexpr int kMaxChunksPerRow = 1024;        // rows up to 1024 * 2048 = 2,097,152 columns
 
