@@ -60,6 +60,9 @@ def parse_args(argv=None):
     ap.add_argument("--top-p", type=float, default=1.0,
                     help="top-p filter (after the top-k when --top-k is set; over the whole row "
                          "when it is not; 1 = off)")
+    ap.add_argument("--rep-penalty", type=float, default=1.0,
+                    help="repetition penalty of draft and target rows (1 = off; needs --top-k); "
+                         "each request gets a seeded history of 64-1024 earlier tokens per family")
     ap.add_argument("--shards", type=int, default=0,
                     help="also time the vocabulary-sharded verification with the target "
                          "rows split into this many column slices (1-8), against the "
@@ -225,6 +228,14 @@ def profiled_traffic(workload: str, top_k: int = 0):
         return None
 
 
+def run_traffic(workload: str, args):
+    """profiled_traffic for this run's filters: nucleus (top-p without top-k)
+    and penalty rows run another row-pass variant, with no committed summary."""
+    if args.rep_penalty != 1.0 or (args.top_k <= 0 and args.top_p < 1.0):
+        return None
+    return profiled_traffic(workload, args.top_k)
+
+
 def algorithmic_bytes(wl, mp) -> dict:
     """Bytes the step must read once: every distinct mapped draft row and all
     m_b + 1 target rows of every request."""
@@ -250,11 +261,23 @@ def step_launches(args) -> int:
     """Kernels one tt_step launches: alignment, row pass and decision; with
     filters also the kept sets of top-k families, the nucleus kernel of
     top-p-only families and the transfer of q_hat before the decision."""
+    pen = 1 if args.rep_penalty != 1.0 else 0  # the penalty's per-request sets
     if args.top_k > 0:
-        return 5
+        return 5 + pen
     if args.top_p < 1.0:
-        return 5
+        return 6  # the nucleus merge and the exact nucleus kernel
     return 3
+
+
+def filters_config(args):
+    """The sampling filters of the run for the config key (None without any)."""
+    if args.top_k <= 0 and args.top_p >= 1.0 and args.rep_penalty == 1.0:
+        return None
+    f = {"top_k": args.top_k, "top_p": args.top_p}
+    if args.rep_penalty != 1.0:
+        f["rep_penalty"] = args.rep_penalty
+        f["history"] = "64-1024 tokens per request and family"
+    return f
 
 
 def step_kwargs(args) -> dict:
@@ -262,6 +285,8 @@ def step_kwargs(args) -> dict:
     the temperature override and the sampling filters of both families."""
     kw = {"top_k_draft": args.top_k, "top_k_target": args.top_k,
           "top_p_draft": args.top_p, "top_p_target": args.top_p}
+    if args.rep_penalty != 1.0:
+        kw["rep_penalty_draft"] = kw["rep_penalty_target"] = args.rep_penalty
     if args.temp is not None:
         kw["temp_draft"] = kw["temp_target"] = args.temp
     return kw
@@ -357,6 +382,8 @@ def prepare_step(tt, W, name, args, rank, dev, stream):
     step with every output (mapped draft rows, acceptance, the parity sample),
     and a prepared call for the timed loop."""
     wl = W.make_workload(name, B=args.batch, seed=rank, device=str(dev))
+    if args.rep_penalty != 1.0:
+        wl = W.with_histories(wl, 64, 1024, seed=rank)
     inp = tt.device_inputs(wl, dev)
     prm = inp["params"]
     prm.request_base = request_base(rank, wl.B)
@@ -364,6 +391,7 @@ def prepare_step(tt, W, name, args, rank, dev, stream):
         prm.temp_draft = prm.temp_target = args.temp
     prm.top_k_draft = prm.top_k_target = args.top_k
     prm.top_p_draft = prm.top_p_target = args.top_p
+    prm.rep_penalty_draft = prm.rep_penalty_target = args.rep_penalty
     full = tt.tt_step(inp["batch"], inp["vd"], inp["vt"], inp["draft_logits"],
                       inp["target_logits"], prm)
     import torch
@@ -441,7 +469,7 @@ def extra_workload(tt, W, name, args, rank, ws, dev, stream, clocks, peak):
          "hbm_gbs_step": ab["total"] / (sec / K) / 1e9,
          "step_frac_of_8tbs": ab["total"] / (sec / K) / 8e12,
          "rowpass_gbs": row_gbs, "rowpass_frac": row_gbs / peak,
-         "rowpass_traffic": profiled_traffic(name, args.top_k),
+         "rowpass_traffic": run_traffic(name, args),
          "stage_ms": st, "dtw_pairs_per_s": wl.B / (align_alone_ms / 1e3),
          "accept_rate": float(acc.sum() / max(1, m.sum())), "clocks": clocks.summary(h0, h1)}
     del wl, inp, full, call
@@ -521,7 +549,7 @@ def run_mine(args):
     peak, peak_kind = measured_hbm_peak()
     achieved = ab["total"] / (row_ms / 1e3) / 1e9
     step_gbs = ab["total"] / (sec / K) / 1e9
-    traffic = profiled_traffic(name, args.top_k)
+    traffic = run_traffic(name, args)
 
     e2e = None
     if not args.no_e2e:
@@ -569,8 +597,7 @@ def run_mine(args):
                    "logits_cols": [int(dl_shape[1]), int(tl_shape[1])],
                    "target_tokens_per_gpu": wl.n_target, "window": prm.window,
                    "temperature": [prm.temp_draft, prm.temp_target],
-                   "filters": ({"top_k": args.top_k, "top_p": args.top_p} if filtered
-                               else None),
+                   "filters": filters_config(args),
                    "parallelism": "dp%d (independent requests per GPU)" % ws,
                    "l2": "inputs %.0f MB exceed the 129 MB L2; no flush between steps"
                          % (in_bytes / 1e6) if ab["total"] > L2_BYTES else "inputs fit in L2",
@@ -844,6 +871,8 @@ def run_reference(args):
     # oracle reads each request's rows copied to the host
     gen_dev = "cuda" if torch.cuda.is_available() else "cpu"
     wl = W.make_workload(name, B=args.batch, seed=0, device=gen_dev)
+    if args.rep_penalty != 1.0:
+        wl = W.with_histories(wl, 64, 1024, seed=0)
     per_worker = {"b1_g4_v32k": 1, "b64_g8_v152k": 2, "b256_g16_v152k_bf16": 1,
                   "dtw_4096x64": 8, "b1024_g8_v201k_bf16": 1}.get(name, 1)
     n = host_cores()
@@ -881,8 +910,7 @@ def run_reference(args):
                                        int(wl.target_logits.shape[1])],
                        "target_tokens_per_gpu": wl.n_target, "window": spec.window,
                        "temperature": temps,
-                       "filters": ({"top_k": args.top_k, "top_p": args.top_p}
-                                   if args.top_k > 0 else None),
+                       "filters": filters_config(args),
                        "parallelism": "oracle processes on the host cores",
                        "requests_per_step": per_step},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": n, "kind": "oracle",

@@ -124,8 +124,11 @@ typedef struct {
      below top_p (top_p >= 1 = off), and renormalise the kept set. Every
      probability of the step is then the filtered one: q_hat, p_hat, the accept
      ratio, the residual and the bonus row; lse is the log-normaliser of each
-     target row's kept set. top_p < 1 needs top_k >= 1 (TT_ERR_UNSUPPORTED
-     otherwise); in full-q mode either both families are filtered or neither. */
+     target row's kept set. top_p < 1 with top_k = 0 keeps a nucleus over the
+     whole row (the shortest prefix, larger logit then smaller column first,
+     whose mass reaches top_p); in full-q mode either both families are
+     filtered or neither, and no family may be a nucleus one
+     (TT_ERR_UNSUPPORTED). */
   int32_t top_k_draft;
   float top_p_draft;
   int32_t top_k_target;

@@ -160,3 +160,23 @@ def test_cpu_leg_counts_boundary_cases_and_mismatches(monkeypatch):
     full["next_token"][1] = (int(o["next_token"][1]) + 7) % wl.target_logits.shape[1]
     cpu, cpu_all, bnd = bench.cpu_baseline_leg(wl, full, args, bench.step_kwargs(args))
     assert bnd["mismatches"] == 1 and bnd["first_mismatches"]
+
+
+def test_launch_count_traffic_and_filters_key_follow_the_run_filters():
+    """gpu_launches counts the kernels each filter family launches (nucleus:
+    merge and exact kernels; penalty: its per-request sets), and only runs
+    whose row-pass variant has a committed summary may carry its traffic."""
+    p = bench.parse_args
+    assert bench.step_launches(p([])) == 3
+    assert bench.step_launches(p(["--top-k", "20", "--top-p", "0.95"])) == 5
+    assert bench.step_launches(p(["--top-p", "0.9"])) == 6
+    assert bench.step_launches(p(["--top-k", "20", "--rep-penalty", "1.1"])) == 6
+    assert bench.run_traffic("no_such_workload", p(["--top-p", "0.9"])) is None
+    assert bench.run_traffic("no_such_workload",
+                             p(["--top-k", "20", "--rep-penalty", "1.1"])) is None
+    assert bench.filters_config(p([])) is None
+    assert bench.filters_config(p(["--top-p", "0.9"])) == {"top_k": 0, "top_p": 0.9}
+    f = bench.filters_config(p(["--top-k", "20", "--rep-penalty", "1.1"]))
+    assert f["rep_penalty"] == 1.1 and f["top_k"] == 20
+    kw = bench.step_kwargs(p(["--top-k", "20", "--rep-penalty", "1.1"]))
+    assert kw["rep_penalty_draft"] == kw["rep_penalty_target"] == 1.1
