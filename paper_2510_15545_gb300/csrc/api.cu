@@ -153,12 +153,10 @@ cudaError_t launch_pen_sets(const tt_batch* batch, const RowSet& d, const RowSet
   return launch_pen_prep(a, s);
 }
 
-// A nucleus family's row set: top-kNucList lists of its units and partials
-// of all its columns, from which the nucleus kernels find each row's kept set.
-void attach_nucleus(RowSet& r, bool on) {
-  r.nucleus = on ? 1 : 0;
-  if (on) r.top_k = kNucList;
-}
+// A nucleus family's row set: the row pass writes the compensated partials of
+// all its columns, and the nucleus kernel finds each row's kept set from them
+// and the row's logits.
+void attach_nucleus(RowSet& r, bool on) { r.nucleus = on ? 1 : 0; }
 
 // A family's row set sees its penalty arrays.
 void attach_pen(RowSet& r, bool on, float theta, PenEntry* pen, const int32_t* pbase,

@@ -10,7 +10,14 @@
 // 2^(z * scale - M) / S and its mass per 2048-column chunk.
 //
 // nucleus_kernel finds it exactly, one CTA per row, from the row's logits and
-// the row pass's partials (which give the row maximum M):
+// the row pass's compensated partials of all its columns (which give the row
+// maximum M and the row's total):
+//  0. usually in one pass over the row: every column within kCandDelta = 14
+//     log2 units of M is gathered in shared memory (on the paper's settings
+//     the cut lies within about 13 units), the candidates' fixed-point masses
+//     are binned as in step 1, and the crossing bucket is walked as in step 3
+//     (one lane per candidate when it holds at most 32). Rows whose candidates
+//     overflow the buffer or do not reach the cut take steps 1-4:
 //  1. a histogram of delta = M - z * scale in buckets of 1/32 (log2 units) over
 //     [0, 40), with counts and masses 2^-delta in 40-bit fixed point, so that
 //     sums are exact in any order (columns at delta >= 40 weigh less than
@@ -49,7 +56,21 @@ constexpr float kDeltaMax = 40.f;      // level-0 range of delta (log2 units)
 constexpr float kBucketsPerUnit = 32.f;  // level-0 buckets per log2 unit
 constexpr int kLevels = 3;             // the level-0 histogram and two refinements
 constexpr int kRefine = 256;           // a crossing bucket with more columns is split again
-constexpr int kGather = 2048;          // crossing-bucket columns held in shared memory
+constexpr int kGather = 4096;          // columns held in shared memory (candidates, crossing bucket)
+constexpr float kCandDelta = 14.f;     // candidates: delta below this (log2 units)
+constexpr int kCross = 256;            // candidates of the crossing bucket held apart
+constexpr int kRegion = kGather / kNW;  // candidates per warp's region of the buffer
+// Rows of at most kWarpRowMax columns: one warp per row (nucleus_warp_kernel),
+// candidates within kWCandDelta log2 units of the maximum, at most kWCap.
+constexpr int kWarpRowMax = 8192;
+constexpr float kWCandDelta = 12.f;
+constexpr int kWCap = 512;
+constexpr int kWBuckets = int(kWCandDelta) * 32 + 32;
+constexpr int kWWarps = 8;
+constexpr int kWChunks = kWarpRowMax / kChunk;
+// buckets of the candidates' delta (a little past kCandDelta: the fp32 delta of
+// a candidate may round up to it)
+constexpr int kCandBuckets = int(kCandDelta) * 32 + 32;
 constexpr float kFix = 1099511627776.f;  // 2^40: fixed-point scale of the masses
 
 __device__ __forceinline__ float load_dt(const char* row, int dt, int64_t col) {
@@ -86,16 +107,24 @@ __device__ __forceinline__ int path_cmp(const Path& p, const Path& cross, int le
 }
 
 
-// Shared memory of one nucleus CTA (about 40 KB, under the default 48 KB).
+// Shared memory of one nucleus CTA (about 58 KB: three CTAs fit on an SM).
 struct NucSmem {
   unsigned int cnt[kBuckets];
   unsigned long long mass[kBuckets];
   unsigned long long cacc[kMaxChunksPerRow];  // kept mass per chunk
-  Cand gz[kGather];                           // gathered crossing-bucket columns (z, column)
+  Cand gz[kGather];                           // gathered columns (z, column)
+  Cand gc[kCross];                            // candidates of the crossing bucket
   unsigned long long wsum[kNW];
   unsigned long long wmax[kNW];
+  F2 wf2[kNW];
   int wcnt[kNW];
   int n_gz;
+  int n_gc;
+  int wn[kNW];  // candidates per warp region
+  int todo[kNT];  // rows of the current tile left to this kernel
+  int n_todo;
+  float tau_v;  // the last kept column, found by one warp
+  int tau_c;
   int cross;  // crossing bucket of the current level (-1: no bucket reaches the cut)
   unsigned long long before;  // mass of the columns ranked before the current range
 };
@@ -114,14 +143,28 @@ __device__ __forceinline__ unsigned long long block_sum_u64(unsigned long long v
   return t;
 }
 
-// Block-wide (largest value below `below`, how many columns hold it) over the
-// gathered columns.
-__device__ __forceinline__ void block_max_count(const NucSmem& sm, NucSmem& s, int n, float below,
+// Block-wide compensated sum of one pair per thread (the same on every thread).
+__device__ __forceinline__ F2 block_sum_f2(F2 v, NucSmem& s, int lane, int warp) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1)
+    v = f2_add(v, F2{__shfl_xor_sync(0xffffffffu, v.hi, o), __shfl_xor_sync(0xffffffffu, v.lo, o)});
+  __syncthreads();
+  if (lane == 0) s.wf2[warp] = v;
+  __syncthreads();
+  F2 t = {0.f, 0.f};
+#pragma unroll
+  for (int w = 0; w < kNW; ++w) t = f2_add(t, s.wf2[w]);
+  return t;
+}
+
+// Block-wide (largest value below `below`, how many columns hold it) over
+// n gathered columns.
+__device__ __forceinline__ void block_max_count(const Cand* arr, NucSmem& s, int n, float below,
                                                 int tid, float& vmax, int& count) {
   const int lane = tid & 31, warp = tid >> 5;
   float v = -INFINITY;
   for (int i = tid; i < n; i += kNT) {
-    const float z = sm.gz[i].v;
+    const float z = arr[i].v;
     if (z < below) v = fmaxf(v, z);
   }
 #pragma unroll
@@ -135,7 +178,7 @@ __device__ __forceinline__ void block_max_count(const NucSmem& sm, NucSmem& s, i
   const uint32_t key = uint32_t(best);
   vmax = __uint_as_float(key & 0x80000000u ? key ^ 0x80000000u : ~key);
   int c = 0;
-  for (int i = tid; i < n; i += kNT) c += sm.gz[i].v == vmax;
+  for (int i = tid; i < n; i += kNT) c += arr[i].v == vmax;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
   __syncthreads();
@@ -146,17 +189,500 @@ __device__ __forceinline__ void block_max_count(const NucSmem& sm, NucSmem& s, i
   for (int w = 0; w < kNW; ++w) count += s.wcnt[w];
 }
 
-// One CTA per nucleus row (grid-stride over draft rows, then target rows).
-__global__ void __launch_bounds__(kNT) nucleus_kernel(KeptArgs a) {
+__device__ __forceinline__ uint32_t max_bf16x2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+// Largest logit of a 16-byte vector (4 fp32 or 8 bf16 logits).
+__device__ __forceinline__ float vector_max(const uint4& w, int dt) {
+  if (dt == TT_F32)
+    return fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)),
+                 fmaxf(__uint_as_float(w.z), __uint_as_float(w.w)));
+  const uint32_t m = max_bf16x2(max_bf16x2(w.x, w.y), max_bf16x2(w.z, w.w));
+  return fmaxf(__uint_as_float(m << 16), __uint_as_float(m & 0xffff0000u));
+}
+
+// One pass over a row's nvec whole 16-byte vectors by NTHR threads (this one
+// is t), U loads in flight per thread: hit(v, w) for every vector w (the
+// row's v-th) holding a logit above zc, found from the vector's maximum in a
+// few instructions.
+template <int NTHR, int U, class Hit>
+__device__ __forceinline__ void scan_row(const uint4* rv, int nvec, int dt, float zc, int t,
+                                         Hit&& hit) {
+  for (int v0 = t; v0 < nvec; v0 += NTHR * U) {
+    uint4 w[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int v = v0 + u * NTHR;
+      if (v < nvec) w[u] = ld_stream_v4(rv + v);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int v = v0 + u * NTHR;
+      if (v < nvec && vector_max(w[u], dt) > zc) hit(v, w[u]);
+    }
+  }
+}
+
+// The logits above zc of vector w (the row's v-th), passed to take(z, column).
+template <class Take>
+__device__ __forceinline__ void vector_candidates(const uint4& w, int dt, int v, float zc,
+                                                  Take&& take) {
+  const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+  if (dt == TT_F32) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float z = __uint_as_float(ww[q]);
+      if (z > zc) take(z, v * 4 + q);
+    }
+  } else {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float z0 = __uint_as_float(ww[q] << 16), z1 = __uint_as_float(ww[q] & 0xffff0000u);
+      if (z0 > zc) take(z0, v * 8 + 2 * q);
+      if (z1 > zc) take(z1, v * 8 + 2 * q + 1);
+    }
+  }
+}
+
+// The cut among n gathered columns that hold it, `before` being the mass
+// ranked before all of them: runs of equal logits from the largest; a run holds
+// the cut or lies wholly before it, and the number of its columns kept follows
+// from the run's mass (k columns kept while before + k' * mv < thr for
+// k' < k), the smallest columns of the run first. Every thread calls; the last
+// kept column is (tau, tau_col) on every thread.
+__device__ void walk_runs(const Cand* arr, int n, unsigned long long before, double thr,
+                          NucSmem& sm, float M, float scale, float& tau, int& tau_col) {
+  const int tid = threadIdx.x;
+  float below = INFINITY;
+  for (int guard = 0; guard < n; ++guard) {
+    float v;
+    int cv;
+    block_max_count(arr, sm, n, below, tid, v, cv);
+    if (cv == 0) break;  // (not reached: the columns' mass reaches thr)
+    const unsigned long long mv =
+        (unsigned long long)__float2ull_rn(exp2_scaled(v, scale, M) * kFix);
+    const double need = thr - double(before);  // > 0
+    if (double(before) + double(mv) * double(cv) >= thr || mv == 0ull) {
+      // kept: the first k columns of the run, k = ceil(need / mv) (at least 1)
+      long long k = mv == 0ull ? cv : (long long)ceil(need / double(mv));
+      k = k < 1 ? 1 : (k > cv ? cv : k);
+      // the k-th smallest column among the run (ranks by counting)
+      for (int i = tid; i < n; i += kNT) {
+        const Cand e = arr[i];
+        if (e.v != v) continue;
+        int rank = 0;
+        for (int j = 0; j < n; ++j) rank += (arr[j].v == v && arr[j].c < e.c);
+        if (rank == k - 1) sm.cross = e.c;  // exactly one thread
+      }
+      __syncthreads();
+      tau = v;
+      tau_col = sm.cross;
+      __syncthreads();
+      return;
+    }
+    before += mv * (unsigned long long)cv;
+    below = v;
+  }
+}
+
+// The kept set of a nucleus row from one pass over its logits, when the cut
+// lies among the columns within kCandDelta log2 units of the row maximum M
+// (a column there weighs at least 2^-kCandDelta of the maximum's mass): those
+// columns are gathered in shared memory, their masses (40-bit fixed point)
+// binned by delta at 1/32 log2 unit, and the bucket where the running mass,
+// largest logits first, reaches top_p of the row's total (from the partials)
+// is walked by value. Every column above zc is a candidate, so the walk over
+// the candidates in rank order is the walk over the whole row down to zc, and
+// a cut reached among them is the row's cut. Returns false -- and the caller
+// runs the histogram levels over the whole row -- when the candidates overflow
+// the buffer, their mass stays below the cut, or the crossing bucket holds
+// more than kCross of them. On true, sm.cacc holds the kept masses per chunk.
+// Every thread calls and gets the same result.
+__device__ bool candidate_cut(const Partial* part, NucSmem& sm, const char* row, int dt, int V,
+                              int nvec, int vec, int nch, float M, float scale, float top_p,
+                              float& tau, int& tau_col) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // the row's total 2^(z * scale - M), compensated, from the partials
+  F2 T = {0.f, 0.f};
+  for (int c = tid; c < nch; c += kNT) {
+    const Partial q = part[c];
+    if (q.m > -INFINITY) T = f2_add(T, F2{__fmul_rn(q.s, ex2_approx(q.m - M)), 0.f});
+  }
+  T = block_sum_f2(T, sm, lane, warp);
+  const double Td = double(T.hi) + double(T.lo);
+  if (!(Td > 0.0) || !isfinite(Td)) return false;
+  const double thr = double(top_p) * Td * double(kFix);
+  const float zc = __fdiv_rn(__fsub_rn(M, kCandDelta), scale);  // candidates: z > zc
+
+  if (tid == 0) {
+    sm.n_gc = 0;
+    sm.cross = -1;
+  }
+  if (tid < kNW) sm.wn[tid] = 0;
+  for (int c = tid; c < nch; c += kNT) sm.cacc[c] = 0ull;
+  for (int i = tid; i < kCandBuckets; i += kNT) sm.mass[i] = 0ull;
+  __syncthreads();
+  // ------------------------------------ one pass over the row: the candidates
+  // A vector holding a logit above zc has its candidates appended at once by
+  // its lane (the row is not read again: the rows in flight across the GPU
+  // exceed L2), each warp to its own region of the buffer (kRegion entries;
+  // the columns are spread over the warps, so a region overflows only when
+  // the whole buffer nearly would).
+  Cand* region = sm.gz + warp * kRegion;
+  auto take = [&](float z, int x) {
+    const int i = atomicAdd(&sm.wn[warp], 1);
+    if (i < kRegion) region[i] = Cand{z, x};
+  };
+  scan_row<kNT, 8>(reinterpret_cast<const uint4*>(row), nvec, dt, zc, tid,
+                   [&](int v, const uint4& w) { vector_candidates(w, dt, v, zc, take); });
+  for (int x = nvec * vec + tid; x < V; x += kNT) {  // the ragged tail
+    const float z = load_dt(row, dt, x);
+    if (z > zc) take(z, x);
+  }
+  __syncthreads();
+  bool over = false;
+  int ng = 0;
+#pragma unroll
+  for (int x = 0; x < kNW; ++x) {
+    ng += sm.wn[x];
+    over |= sm.wn[x] > kRegion;
+  }
+  if (over) return false;
+  // every gathered candidate, region by region
+  auto for_cands = [&](auto&& fn) {
+    for (int x = 0; x < kNW; ++x) {
+      const int n = sm.wn[x];
+      for (int i = tid; i < n; i += kNT) fn(sm.gz[x * kRegion + i]);
+    }
+  };
+
+  // ------------------------ candidate masses binned by delta (1/32 log2 unit)
+  auto fixm = [&](float z) {
+    return (unsigned long long)__float2ull_rn(exp2_scaled(z, scale, M) * kFix);
+  };
+  auto bucket = [&](float z) {  // non-increasing in z
+    const float f = __fsub_rn(M, __fmul_rn(z, scale)) * kBucketsPerUnit;
+    return f > 0.f ? min(kCandBuckets - 1, int(f)) : 0;
+  };
+  for_cands([&](const Cand& e) { atomicAdd(&sm.mass[bucket(e.v)], fixm(e.v)); });
+  __syncthreads();
+  // the first bucket whose inclusive running mass reaches thr (thread t owns a
+  // contiguous run of buckets)
+  constexpr int kPer = (kCandBuckets + kNT - 1) / kNT;
+  const int b0 = tid * kPer, b1 = min(kCandBuckets, b0 + kPer);
+  unsigned long long loc = 0ull;
+  for (int i = b0; i < b1; ++i) loc += sm.mass[i];
+  unsigned long long incl = loc;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned long long n = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += n;
+  }
+  if (lane == 31) sm.wsum[warp] = incl;
+  __syncthreads();
+  unsigned long long wbase = 0ull;
+#pragma unroll
+  for (int x = 0; x < kNW; ++x)
+    if (x < warp) wbase += sm.wsum[x];
+  unsigned long long run = wbase + incl - loc;
+  for (int i = b0; i < b1; ++i) {
+    const unsigned long long nx = run + sm.mass[i];
+    if (double(nx) >= thr && double(run) < thr) sm.cross = i;  // one bucket at most
+    run = nx;
+  }
+  __syncthreads();
+  const int cb = sm.cross;
+  if (cb < 0) return false;  // the candidates' mass stays below the cut
+  unsigned long long pre = 0ull;
+  for (int i = tid; i < cb; i += kNT) pre += sm.mass[i];
+  const unsigned long long before = block_sum_u64(pre, sm, lane, warp);
+  // the crossing bucket's candidates, apart
+  for_cands([&](const Cand& e) {
+    if (bucket(e.v) == cb) {
+      const int j = atomicAdd(&sm.n_gc, 1);
+      if (j < kCross) sm.gc[j] = e;
+    }
+  });
+  __syncthreads();
+  const int nc = sm.n_gc;
+  if (nc > kCross) return false;
+  if (nc <= 32) {
+    // one lane per candidate: a candidate is kept when the mass ranked before
+    // it (larger logit, then smaller column) is below thr; the last kept one
+    // has the most mass before it (every candidate's mass is positive)
+    if (warp == 0) {
+      const bool has = lane < nc;
+      const Cand e = has ? sm.gc[lane] : Cand{-INFINITY, 0x7fffffff};
+      const unsigned long long me = has ? fixm(e.v) : 0ull;
+      unsigned long long pm = 0ull;
+      for (int j = 0; j < nc; ++j) {
+        const float vj = __shfl_sync(0xffffffffu, e.v, j);
+        const int cj = __shfl_sync(0xffffffffu, e.c, j);
+        const unsigned long long mj = __shfl_sync(0xffffffffu, me, j);
+        if (vj > e.v || (vj == e.v && cj < e.c)) pm += mj;
+      }
+      const bool kept = has && double(before + pm) < thr;
+      unsigned long long key = kept ? pm + 1ull : 0ull;
+      int src = lane;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const unsigned long long ok = __shfl_xor_sync(0xffffffffu, key, o);
+        const int os = __shfl_xor_sync(0xffffffffu, src, o);
+        if (ok > key || (ok == key && os < src)) {
+          key = ok;
+          src = os;
+        }
+      }
+      if (lane == src) {
+        sm.tau_v = e.v;
+        sm.tau_c = e.c;
+      }
+    }
+    __syncthreads();
+    tau = sm.tau_v;
+    tau_col = sm.tau_c;
+  } else {
+    walk_runs(sm.gc, nc, before, thr, sm, M, scale, tau, tau_col);
+  }
+  // the kept candidates join their chunks
+  for_cands([&](const Cand& e) {
+    if (e.v > tau || (e.v == tau && e.c <= tau_col)) atomicAdd(&sm.cacc[e.c / kChunk], fixm(e.v));
+  });
+  return ng > 0;
+}
+
+// Shared memory of one warp of nucleus_warp_kernel (about 7.7 KB).
+struct NucWarpSmem {
+  Cand cand[kWCap];
+  unsigned long long mass[kWBuckets];
+  Cand gc[32];
+  unsigned long long cacc[kWChunks];
+  int n, ngc;
+};
+
+// The kept set of a narrow nucleus row (at most kWarpRowMax columns), one warp
+// per row: the candidate way of candidate_cut at warp scale -- the columns
+// within kWCandDelta log2 units of the row maximum gathered, their fixed-point
+// masses binned by delta at 1/32 log2 unit, the crossing bucket ranked one
+// candidate per lane. A row whose candidates overflow kWCap, do not reach the
+// cut or put more than 32 in the crossing bucket gets head n = -1 and is left
+// to nucleus_kernel.
+__global__ void __launch_bounds__(kWWarps * 32, 3) nucleus_warp_kernel(KeptArgs a) {
+  extern __shared__ __align__(16) char wsm_raw[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  NucWarpSmem& sm = reinterpret_cast<NucWarpSmem*>(wsm_raw)[warp];
+  const int64_t rows_d = (a.d.nucleus && a.d.V <= kWarpRowMax) ? a.rows_d : 0;
+  const int64_t rows_t = (a.t.nucleus && a.t.V <= kWarpRowMax) ? a.rows_t : 0;
+  grid_dependency_wait();  // the partials (and the need flags) come from earlier kernels
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  for (int64_t w = int64_t(blockIdx.x) * kWWarps + warp; w < rows_d + rows_t;
+       w += int64_t(gridDim.x) * kWWarps) {
+    const bool tgt = w >= rows_d;
+    const int64_t r = tgt ? w - rows_d : w;
+    const RowSet& S = tgt ? a.t : a.d;
+    if (!tgt && S.need && S.need[r] == 0) continue;
+    const int dt = tgt ? a.dt_t : a.dt_d;
+    const float top_p = tgt ? a.top_p_t : a.top_p_d;
+    KeptHead* head = (tgt ? a.head_t : a.head_d) + r;
+    float* um = (tgt ? a.um_t : a.um_d) + r * S.nch;
+    const int V = S.V, nch = S.nch;
+    const float scale = S.scale;
+    const char* row = S.data + r * S.stride_bytes;
+    const int vec = dt == TT_F32 ? 4 : 8;
+    const int nvec = V / vec;
+    const Partial* part = S.part + r * nch;
+    // the row maximum and total from the partials (compensated)
+    float M = -INFINITY;
+    for (int c = lane; c < nch; c += 32) M = fmaxf(M, part[c].m);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    if (!isfinite(M)) {
+      if (lane == 0) *head = KeptHead{NAN, 0, NAN, -1, M, 0.f};
+      continue;
+    }
+    F2 T = {0.f, 0.f};
+    for (int c = lane; c < nch; c += 32) {
+      const Partial q = part[c];
+      if (q.m > -INFINITY) T = f2_add(T, F2{__fmul_rn(q.s, ex2_approx(q.m - M)), 0.f});
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+      T = f2_add(T, F2{__shfl_xor_sync(0xffffffffu, T.hi, o), __shfl_xor_sync(0xffffffffu, T.lo, o)});
+    const double Td = double(T.hi) + double(T.lo);
+    if (!(Td > 0.0) || !isfinite(Td)) {
+      if (lane == 0) head->n = -1;
+      continue;
+    }
+    const double thr = double(top_p) * Td * double(kFix);
+    const float zc = __fdiv_rn(__fsub_rn(M, kWCandDelta), scale);  // candidates: z > zc
+    auto fixm = [&](float z) {
+      return (unsigned long long)__float2ull_rn(exp2_scaled(z, scale, M) * kFix);
+    };
+    auto bucket = [&](float z) {  // non-increasing in z
+      const float f = __fsub_rn(M, __fmul_rn(z, scale)) * kBucketsPerUnit;
+      return f > 0.f ? min(kWBuckets - 1, int(f)) : 0;
+    };
+    if (lane == 0) {
+      sm.n = 0;
+      sm.ngc = 0;
+    }
+    for (int i = lane; i < kWBuckets; i += 32) sm.mass[i] = 0ull;
+    if (lane < kWChunks) sm.cacc[lane] = 0ull;
+    __syncwarp();
+    // one pass over the row; a vector holding candidates has them appended at
+    // once by its lane
+    auto take = [&](float z, int x) {
+      const int i = atomicAdd(&sm.n, 1);
+      if (i < kWCap) sm.cand[i] = Cand{z, x};
+    };
+    scan_row<32, 8>(reinterpret_cast<const uint4*>(row), nvec, dt, zc, lane,
+                    [&](int v, const uint4& w) { vector_candidates(w, dt, v, zc, take); });
+    for (int x = nvec * vec + lane; x < V; x += 32) {  // the ragged tail
+      const float z = load_dt(row, dt, x);
+      if (z > zc) take(z, x);
+    }
+    __syncwarp();
+    const int n = sm.n;
+    if (n > kWCap || n == 0) {
+      if (lane == 0) head->n = -1;
+      __syncwarp();
+      continue;
+    }
+    for (int i = lane; i < n; i += 32) {
+      const Cand e = sm.cand[i];
+      atomicAdd(&sm.mass[bucket(e.v)], fixm(e.v));
+    }
+    __syncwarp();
+    // the first bucket whose inclusive running mass reaches thr (lane l owns a
+    // contiguous run of buckets)
+    constexpr int kPer = (kWBuckets + 31) / 32;
+    const int b0 = lane * kPer, b1 = min(kWBuckets, b0 + kPer);
+    unsigned long long loc = 0ull;
+    for (int i = b0; i < b1; ++i) loc += sm.mass[i];
+    unsigned long long incl = loc;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned long long y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    unsigned long long run = incl - loc, before = 0ull;
+    int cb = kWBuckets;
+    for (int i = b0; i < b1; ++i) {
+      const unsigned long long nx = run + sm.mass[i];
+      if (double(nx) >= thr && double(run) < thr) {
+        cb = i;
+        before = run;
+      }
+      run = nx;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const int ocb = __shfl_xor_sync(0xffffffffu, cb, o);
+      const unsigned long long ob = __shfl_xor_sync(0xffffffffu, before, o);
+      if (ocb < cb) {
+        cb = ocb;
+        before = ob;
+      }
+    }
+    if (cb >= kWBuckets) {  // the candidates' mass stays below the cut
+      if (lane == 0) head->n = -1;
+      __syncwarp();
+      continue;
+    }
+    for (int i = lane; i < n; i += 32) {
+      const Cand e = sm.cand[i];
+      if (bucket(e.v) == cb) {
+        const int j = atomicAdd(&sm.ngc, 1);
+        if (j < 32) sm.gc[j] = e;
+      }
+    }
+    __syncwarp();
+    const int nc = sm.ngc;
+    if (nc > 32) {
+      if (lane == 0) head->n = -1;
+      __syncwarp();
+      continue;
+    }
+    // one lane per candidate of the crossing bucket (see candidate_cut)
+    const bool has = lane < nc;
+    const Cand e = has ? sm.gc[lane] : Cand{-INFINITY, 0x7fffffff};
+    const unsigned long long me = has ? fixm(e.v) : 0ull;
+    unsigned long long pm = 0ull;
+    for (int j = 0; j < nc; ++j) {
+      const float vj = __shfl_sync(0xffffffffu, e.v, j);
+      const int cj = __shfl_sync(0xffffffffu, e.c, j);
+      const unsigned long long mj = __shfl_sync(0xffffffffu, me, j);
+      if (vj > e.v || (vj == e.v && cj < e.c)) pm += mj;
+    }
+    const bool kept = has && double(before + pm) < thr;
+    unsigned long long key = kept ? pm + 1ull : 0ull;
+    int src = lane;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long ok = __shfl_xor_sync(0xffffffffu, key, o);
+      const int os = __shfl_xor_sync(0xffffffffu, src, o);
+      if (ok > key || (ok == key && os < src)) {
+        key = ok;
+        src = os;
+      }
+    }
+    const float tau = __shfl_sync(0xffffffffu, e.v, src);
+    const int tau_col = __shfl_sync(0xffffffffu, e.c, src);
+    // the kept candidates join their chunks; the header
+    for (int i = lane; i < n; i += 32) {
+      const Cand c = sm.cand[i];
+      if (c.v > tau || (c.v == tau && c.c <= tau_col))
+        atomicAdd(&sm.cacc[c.c / kChunk], fixm(c.v));
+    }
+    __syncwarp();
+    unsigned long long tot = lane < nch ? sm.cacc[lane] : 0ull;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+    const double Sd = double(tot) / double(kFix);  // kept normaliser relative to 2^M
+    if (lane < nch) um[lane] = float(double(sm.cacc[lane]) / double(kFix) / Sd);
+    if (lane == 0) {
+      const float lse = float((double(M) + log2(Sd)) * 0.6931471805599453);
+      *head = KeptHead{lse, 1, tau, tau_col, M, float(1.0 / Sd)};
+    }
+    __syncwarp();  // shared memory is reused by the warp's next row
+  }
+}
+
+// One CTA per nucleus row: every row of a family wider than kWarpRowMax, and
+// the rows of a narrower family that nucleus_warp_kernel left (head n = -1),
+// found 256 rows at a time. Tiles of draft rows, then of target rows,
+// grid-stride.
+__global__ void __launch_bounds__(kNT, 3) nucleus_kernel(KeptArgs a) {
   extern __shared__ __align__(16) char nsm_raw[];
   NucSmem& sm = *reinterpret_cast<NucSmem*>(nsm_raw);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t rows_d = a.d.nucleus ? a.rows_d : 0, rows_t = a.t.nucleus ? a.rows_t : 0;
+  const int tsz_d = a.d.V <= kWarpRowMax ? kNT : 1, tsz_t = a.t.V <= kWarpRowMax ? kNT : 1;
+  const int64_t nt_d = (rows_d + tsz_d - 1) / tsz_d, nt_t = (rows_t + tsz_t - 1) / tsz_t;
   grid_dependency_wait();  // the partials (and the need flags) come from earlier kernels
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  for (int64_t w = blockIdx.x; w < rows_d + rows_t; w += gridDim.x) {
-    const bool tgt = w >= rows_d;
-    const int64_t r = tgt ? w - rows_d : w;
+  for (int64_t tile = blockIdx.x; tile < nt_d + nt_t; tile += gridDim.x) {
+  const bool tgt = tile >= nt_d;
+  const int tsz = tgt ? tsz_t : tsz_d;
+  const int64_t r0 = (tgt ? tile - nt_d : tile) * tsz;
+  int n_todo = 1;
+  if (tsz > 1) {  // the narrow rows the warp kernel could not settle
+    __syncthreads();
+    if (tid == 0) sm.n_todo = 0;
+    __syncthreads();
+    const int64_t rr = r0 + tid;
+    const RowSet& SF = tgt ? a.t : a.d;
+    const KeptHead* hf = tgt ? a.head_t : a.head_d;
+    if (rr < (tgt ? rows_t : rows_d) && (tgt || !SF.need || SF.need[rr] != 0) && hf[rr].n == -1)
+      sm.todo[atomicAdd(&sm.n_todo, 1)] = tid;
+    __syncthreads();
+    n_todo = sm.n_todo;
+  }
+  for (int k = 0; k < n_todo; ++k) {
+    const int64_t r = tsz > 1 ? r0 + sm.todo[k] : r0;
     const RowSet& S = tgt ? a.t : a.d;
     if (!tgt && S.need && S.need[r] == 0) continue;
     const int dt = tgt ? a.dt_t : a.dt_d;
@@ -169,8 +695,6 @@ __global__ void __launch_bounds__(kNT) nucleus_kernel(KeptArgs a) {
     const int vec = dt == TT_F32 ? 4 : 8;  // logits per 16-byte vector
     const int nvec = V / vec;              // whole vectors (rows start on 16 bytes)
 
-    // only the rows the merge kernel could not settle from their lists
-    if (head->n != -1) continue;
     // the row maximum from the partials (nucleus rows' partials hold every column)
     float M = -INFINITY;
     for (int c = tid; c < nch; c += kNT) M = fmaxf(M, S.part[r * nch + c].m);
@@ -215,14 +739,17 @@ __global__ void __launch_bounds__(kNT) nucleus_kernel(KeptArgs a) {
       return (unsigned long long)__float2ull_rn(exp2_scaled(z, scale, M) * kFix);
     };
 
+    float tau = -INFINITY;
+    int tau_col = 0x7fffffff;  // all kept: every column ranks before (tau, tau_col)
+    const bool settled = candidate_cut(S.part + r * nch, sm, row, dt, V, nvec, vec, nch, M,
+                                       scale, top_p, tau, tau_col);
+    if (!settled) {
     // ------------------------------------- the crossing bucket, level by level
     Path cross;
     int level = 0;
     unsigned long long total = 0ull;
     double thr = 0.0;
     bool all_kept = false;
-    float tau = -INFINITY;
-    int tau_col = 0x7fffffff;  // all_kept: every column ranks before (tau, tau_col)
     for (int c = tid; c < nch; c += kNT) sm.cacc[c] = 0ull;
     if (tid == 0) {
       sm.before = 0ull;
@@ -316,36 +843,7 @@ __global__ void __launch_bounds__(kNT) nucleus_kernel(KeptArgs a) {
     const int ng = sm.n_gz;
     if (!all_kept) {
       if (ng <= kGather) {
-        // runs of equal logits from the largest; a run holds the cut or lies before it
-        unsigned long long before = sm.before;
-        float below = INFINITY;
-        for (int guard = 0; guard < ng; ++guard) {
-          float v;
-          int cv;
-          block_max_count(sm, sm, ng, below, tid, v, cv);
-          if (cv == 0) break;  // (not reached: the bucket's mass reaches thr)
-          const unsigned long long mv = fixm(v);
-          const double need = thr - double(before);  // > 0
-          if (double(before) + double(mv) * double(cv) >= thr || mv == 0ull) {
-            // kept: the first k columns of the run, k = ceil(need / mv) (at least 1)
-            long long k = mv == 0ull ? cv : (long long)ceil(need / double(mv));
-            k = k < 1 ? 1 : (k > cv ? cv : k);
-            // the k-th smallest column among the run (ranks by counting)
-            for (int i = tid; i < ng; i += kNT) {
-              const Cand e = sm.gz[i];
-              if (e.v != v) continue;
-              int rank = 0;
-              for (int j = 0; j < ng; ++j) rank += (sm.gz[j].v == v && sm.gz[j].c < e.c);
-              if (rank == k - 1) sm.cross = e.c;  // exactly one thread
-            }
-            __syncthreads();
-            tau = v;
-            tau_col = sm.cross;
-            break;
-          }
-          before += mv * (unsigned long long)cv;
-          below = v;
-        }
+        walk_runs(sm.gz, ng, sm.before, thr, sm, M, scale, tau, tau_col);
         // the kept columns of the crossing bucket join their chunks
         for (int i = tid; i < ng; i += kNT) {
           const Cand e = sm.gz[i];
@@ -425,6 +923,7 @@ __global__ void __launch_bounds__(kNT) nucleus_kernel(KeptArgs a) {
         });
       }
     }
+    }  // !settled
     __syncthreads();
     // ---------------------------------------------- header and chunk masses
     unsigned long long tot = 0ull;
@@ -438,6 +937,7 @@ __global__ void __launch_bounds__(kNT) nucleus_kernel(KeptArgs a) {
       *head = KeptHead{lse, tot > 0ull ? 1 : 0, tau, tau_col, M, inv_s};
     }
     __syncthreads();  // shared memory is reused by the next row
+  }
   }
 }
 
@@ -655,158 +1155,20 @@ __global__ void __launch_bounds__(kNT) decide_nucleus_kernel(DecideArgs a) {
   }
 }
 
-static_assert(sizeof(NucSmem) <= 48 * 1024, "fits the default dynamic shared memory");
-
-constexpr int kMWarps = 8;   // warps of a merge CTA (one nucleus row each)
-constexpr int kMLists = 4;   // unit lists a lane owns: rows of up to 128 units
-
-__device__ __forceinline__ bool cand_first(float v1, int c1, float v2, int c2) {
-  return v1 > v2 || (v1 == v2 && c1 < c2);
-}
-
-// The kept set of a nucleus row from its unit lists, one warp per row: the
-// lists (each unit's kNucList largest columns, in order) are merged k-way, and
-// columns are kept in the merged order while the mass before them is below
-// top_p of the row's total (from the partials, which hold every column). The
-// walk stops at the cut; a list consumed to its end while the cut is not yet
-// reached may hide further columns of its unit, and the row is left to
-// nucleus_kernel (head n = -1). Also rows of more than 32 * kMLists units.
-__global__ void __launch_bounds__(kMWarps * 32) nucleus_merge_kernel(KeptArgs a) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t rows_d = a.d.nucleus ? a.rows_d : 0, rows_t = a.t.nucleus ? a.rows_t : 0;
-  const int64_t total = rows_d + rows_t;
-  grid_dependency_wait();  // the lists and partials come from the row pass
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  const int Ls = cand_stride(kNucList);
-  for (int64_t w = int64_t(blockIdx.x) * kMWarps + warp; w < total;
-       w += int64_t(gridDim.x) * kMWarps) {
-    const bool tgt = w >= rows_d;
-    const int64_t r = tgt ? w - rows_d : w;
-    const RowSet& S = tgt ? a.t : a.d;
-    if (!tgt && S.need && S.need[r] == 0) continue;
-    KeptHead* head = (tgt ? a.head_t : a.head_d) + r;
-    float* um = (tgt ? a.um_t : a.um_d) + r * S.nch;
-    const int nch = S.nch, nl = S.nlist, cps = S.unit_cols / kChunk;
-    const float scale = S.scale, top_p = tgt ? a.top_p_t : a.top_p_d;
-    const Partial* part = S.part + r * nch;
-    // the row's maximum and total 2^(z * scale - M), compensated
-    float M = -INFINITY;
-    for (int c = lane; c < nch; c += 32) M = fmaxf(M, part[c].m);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    F2 T = {0.f, 0.f};
-    if (M > -INFINITY && isfinite(M))
-      for (int c = lane; c < nch; c += 32) {
-        const Partial q = part[c];
-        if (q.m > -INFINITY) T = f2_add(T, F2{q.s * ex2_approx(q.m - M), 0.f});
-      }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
-      T = f2_add(T, F2{__shfl_xor_sync(0xffffffffu, T.hi, o), __shfl_xor_sync(0xffffffffu, T.lo, o)});
-    if (!isfinite(M) || !(T.hi > 0.f) || !isfinite(T.hi)) {
-      if (lane == 0) *head = KeptHead{NAN, 0, NAN, -1, M, 0.f};
-      continue;
-    }
-    if (nl > 32 * kMLists) {
-      if (lane == 0) head->n = -1;
-      continue;
-    }
-    const F2 thr = f2_mul_f(T, top_p);
-    const Cand* lists = S.cand + r * int64_t(nl) * Ls;
-    const Cand pad = {-INFINITY, -1};
-    Cand cur[kMLists], nxt[kMLists];
-    int pos[kMLists];
-    float acc[kMLists][2];
-#pragma unroll
-    for (int i = 0; i < kMLists; ++i) {
-      const int u = lane + 32 * i;
-      cur[i] = u < nl ? lists[int64_t(u) * Ls] : pad;
-      nxt[i] = u < nl ? lists[int64_t(u) * Ls + 1] : pad;
-      pos[i] = 1;  // list index of nxt
-      acc[i][0] = acc[i][1] = 0.f;
-    }
-    F2 before = {0.f, 0.f};
-    float tau = -INFINITY;
-    int tau_col = 0x7fffffff, n = 0;
-    bool need_exact = false;
-    for (;;) {
-      // the lane's best current head, then the warp's
-      float bv = -INFINITY;
-      int bc = 0x7fffffff, bi = -1;
-#pragma unroll
-      for (int i = 0; i < kMLists; ++i)
-        if (cur[i].c >= 0 && (bi < 0 || cand_first(cur[i].v, cur[i].c, bv, bc))) {
-          bv = cur[i].v;
-          bc = cur[i].c;
-          bi = i;
-        }
-      float wv = bv;
-      int wc = bc;
-      bool f = bi >= 0;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, wv, o);
-        const int oc = __shfl_xor_sync(0xffffffffu, wc, o);
-        const bool of = __shfl_xor_sync(0xffffffffu, int(f), o) != 0;
-        if (of && (!f || cand_first(ov, oc, wv, wc))) {
-          wv = ov;
-          wc = oc;
-          f = true;
-        }
-      }
-      if (!f || !f2_lt(before, thr)) break;  // every list consumed, or the cut is reached
-      const float e = exp2_scaled(wv, scale, M);
-      before = f2_add(before, F2{e, 0.f});
-      tau = wv;
-      tau_col = wc;
-      ++n;
-      // the owner (columns are distinct) books the mass and advances its list
-      bool exhausted = false;
-      if (bi >= 0 && bc == wc && bv == wv) {
-#pragma unroll
-        for (int i = 0; i < kMLists; ++i)
-          if (i == bi) {
-            const int u = lane + 32 * i;
-            acc[i][(wc / kChunk - u * cps) & 1] += e;
-            cur[i] = nxt[i];
-            ++pos[i];
-            nxt[i] = pos[i] < kNucList ? lists[int64_t(u) * Ls + pos[i]] : pad;
-            // the list's last entry taken: its unit may hold more columns
-            exhausted = pos[i] > kNucList;
-          }
-      }
-      if (__any_sync(0xffffffffu, exhausted) && f2_lt(before, thr)) {
-        need_exact = true;
-        break;
-      }
-    }
-    if (need_exact) {
-      if (lane == 0) head->n = -1;
-      continue;
-    }
-    const float Sk = __fadd_rn(before.hi, before.lo);
-    const float inv_s = __frcp_rn(Sk);
-#pragma unroll
-    for (int i = 0; i < kMLists; ++i) {
-      const int u = lane + 32 * i;
-      if (u >= nl) continue;
-      for (int c = 0; c < cps; ++c) {
-        const int ch = u * cps + c;
-        if (ch < nch) um[ch] = acc[i][c] * inv_s;
-      }
-    }
-    if (lane == 0)
-      *head = KeptHead{(M + lg2_approx(Sk)) * 0.6931471805599453f, n, tau, tau_col, M, inv_s};
-  }
-}
+static_assert(3 * (sizeof(NucSmem) + 1024) <= 227 * 1024, "three nucleus CTAs fit on an SM");
+static_assert(3 * (kWWarps * sizeof(NucWarpSmem) + 1024) <= 227 * 1024,
+              "three warp-kernel CTAs fit on an SM");
 
 }  // namespace
 
 cudaError_t preload_nucleus() {
-  cudaFuncAttributes fa;
-  cudaError_t e = cudaFuncGetAttributes(&fa, nucleus_kernel);
+  cudaError_t e = cudaFuncSetAttribute(nucleus_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       int(sizeof(NucSmem)));
   if (e != cudaSuccess) return e;
-  if ((e = cudaFuncGetAttributes(&fa, nucleus_merge_kernel)) != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(nucleus_warp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           int(kWWarps * sizeof(NucWarpSmem)));
+  if (e != cudaSuccess) return e;
+  cudaFuncAttributes fa;
   return cudaFuncGetAttributes(&fa, decide_nucleus_kernel);
 }
 
@@ -828,23 +1190,25 @@ cudaError_t launch_decide_nucleus(const DecideArgs& args, cudaStream_t stream, b
 cudaError_t launch_nucleus(const KeptArgs& args, cudaStream_t stream, int sm_count, bool pdl) {
   const int64_t rows = (args.d.nucleus ? args.rows_d : 0) + (args.t.nucleus ? args.rows_t : 0);
   if (rows == 0) return cudaSuccess;
-  {  // the merge kernel settles most rows from their lists
+  const int64_t narrow = (args.d.nucleus && args.d.V <= kWarpRowMax ? args.rows_d : 0) +
+                         (args.t.nucleus && args.t.V <= kWarpRowMax ? args.rows_t : 0);
+  if (narrow > 0) {  // narrow rows: one warp each first
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(unsigned(std::min<int64_t>((rows + kMWarps - 1) / kMWarps,
-                                                  int64_t(sm_count) * 8)));
-    cfg.blockDim = dim3(kMWarps * 32);
-    cfg.dynamicSmemBytes = 0;
+    cfg.gridDim = dim3(unsigned(std::min<int64_t>((narrow + kWWarps - 1) / kWWarps,
+                                                  int64_t(sm_count) * 3)));
+    cfg.blockDim = dim3(kWWarps * 32);
+    cfg.dynamicSmemBytes = kWWarps * sizeof(NucWarpSmem);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, nucleus_merge_kernel, args);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, nucleus_warp_kernel, args);
     if (e != cudaSuccess) return e;
   }
-  // nucleus_kernel (below) takes the rows it leaves, from their logits
-  const int64_t blocks = std::min<int64_t>(rows, int64_t(sm_count) * 2);
+  // three CTAs of about 59 KB per SM, each streaming one row at a time
+  const int64_t blocks = std::min<int64_t>(rows, int64_t(sm_count) * 3);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(unsigned(blocks));
   cfg.blockDim = dim3(kNT);

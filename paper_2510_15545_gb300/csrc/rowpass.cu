@@ -823,6 +823,24 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
     const char* stage = stages + size_t(s) * R::kStageBytes;
     const int cps = d.set ? R::kCpsT : R::kCpsD;
     const int esz = (d.set ? DTT : DTD) == TT_F32 ? 4 : 2;
+    if constexpr (SEL == 2) {
+      const RowSet& S = d.set ? a.t : a.d;
+      if (S.nucleus) {  // nucleus rows: the compensated partials of all the unit's columns
+        const RowView V = {a, S.scale};
+#pragma unroll 1
+        for (int c = 0; c < cps && c * kChunk < d.n; ++c) {
+          const Partial pc =
+              (d.set ? DTT : DTD) == TT_F32
+                  ? nuc_chunk_partial<TT_F32>(stage, d, V.row(d), S.scale, c, lane)
+                  : nuc_chunk_partial<TT_BF16>(stage, d, V.row(d), S.scale, c, lane);
+          if (lane == 0) S.part[d.row * S.nch + d.chunk + c] = pc;
+        }
+        __syncwarp();
+        if (lane == 0 && !(blockIdx.x == 0 && it == a.stall_stage))
+          mbar_arrive(&empty[s]);  // the stage's bytes are consumed
+        continue;
+      }
+    }
     if (SEL && (d.set ? a.t : a.d).top_k > 0) {  // filtered rows: the unit's top-k list
       const RowSet& S = d.set ? a.t : a.d;
       Cand* out = S.cand + (d.row * S.nlist + d.chunk / cps) * cand_stride(S.top_k);
@@ -841,18 +859,6 @@ __global__ void __launch_bounds__(kThreads, 3) rowpass_kernel(RowPassArgs a) {
         select_unit<DTT>(stage, d, V, lane, S.top_k, scratch, out, drop);
       } else {
         select_unit<DTD>(stage, d, V, lane, S.top_k, scratch, out, drop);
-      }
-      if constexpr (SEL == 2) {
-        if (S.nucleus && d.n > 0) {  // nucleus rows: also the partials of the unit's chunks
-#pragma unroll 1
-          for (int c = 0; c < cps && c * kChunk < d.n; ++c) {
-            const Partial pc =
-                (d.set ? DTT : DTD) == TT_F32
-                    ? nuc_chunk_partial<TT_F32>(stage, d, V.row(d), S.scale, c, lane)
-                    : nuc_chunk_partial<TT_BF16>(stage, d, V.row(d), S.scale, c, lane);
-            if (lane == 0) S.part[d.row * S.nch + d.chunk + c] = pc;
-          }
-        }
       }
       if (lane == 0 && !(blockIdx.x == 0 && it == a.stall_stage))
         mbar_arrive(&empty[s]);  // the stage's bytes are consumed

@@ -127,9 +127,6 @@ __host__ __device__ inline Workspace workspace_layout(void* base, int B, int n_d
     return r;
   };
   const size_t rows_t = size_t(n_target) + B;
-  // nucleus families keep top-kNucList lists of their units
-  if (nuc_d && k_d <= 0) k_d = kNucList;
-  if (nuc_t && k_t <= 0) k_t = kNucList;
   w.part_d = reinterpret_cast<Partial*>(take(sizeof(Partial) * size_t(n_draft) * n_chunks(V_d)));
   w.part_t = reinterpret_cast<Partial*>(take(sizeof(Partial) * rows_t * n_chunks(V_t)));
   w.need_d = reinterpret_cast<uint8_t*>(take(size_t(n_draft)));

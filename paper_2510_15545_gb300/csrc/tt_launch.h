@@ -50,9 +50,9 @@ struct RowSet {
   int top_k;            // > 0: filtered rows, the row pass writes top-k lists to cand
   Cand* cand;           // [n_rows * nlist * cand_stride(top_k)]: one list per row unit
   int nlist;            // units (8 KB stages: 2048 fp32 or 4096 bf16 columns) per row
-  int nucleus;          // 1: top-p without top-k: the row pass writes each unit's
-                        // top-kNucList list (top_k = kNucList) and the partials of
-                        // all its columns; the nucleus kernels find each row's kept set
+  int nucleus;          // 1: top-p without top-k (top_k = 0): the row pass writes the
+                        // compensated partials of all its columns; the nucleus
+                        // kernel finds each row's kept set
   // Repetition penalty (top-k families only; pen = NULL: none): the row pass
   // leaves each request's penalized columns out of its unit lists, and the
   // kept-set kernel adds them back with the row's own (penalized or raw) value.
