@@ -25,14 +25,21 @@ namespace tt {
 
 namespace {
 
-// Bit i set iff byte i of the packed string P equals c.
+// Bit i set iff byte i of the packed string P equals c. Each half's bytes of
+// P ^ c...c are tested for zero exactly (the high bit of a byte of
+// ~(((t & 0x7f..) + 0x7f..) | t | 0x7f..) is set iff the byte of t is 0); the
+// eight flags, at bits 8y (low half) and 8y + 4 (high half) after the shifts,
+// are gathered into bits 0..7 by one multiply: the multiplier's bits 7, 14,
+// 21, 28 send flag bit q to q + 7 .. q + 28, and each product bit receives at
+// most one term (the flags lie 4 apart, the shifts differ mod 4), so nothing
+// carries and bits 28..35 hold the flags in byte order.
 __device__ __forceinline__ uint32_t eq_mask8(uint64_t P, uint32_t c) {
-  uint32_t cc = c * 0x01010101u;
-  uint32_t lo = __vcmpeq4(uint32_t(P), cc), hi = __vcmpeq4(uint32_t(P >> 32), cc);
-  // gather the low bit of each 0x00/0xFF byte into 4 consecutive bits
-  uint32_t blo = (((lo & 0x01010101u) * 0x00204081u) >> 21) & 0xFu;
-  uint32_t bhi = (((hi & 0x01010101u) * 0x00204081u) >> 21) & 0xFu;
-  return blo | (bhi << 4);
+  const uint32_t cc = c * 0x01010101u;
+  const uint32_t tl = uint32_t(P) ^ cc, th = uint32_t(P >> 32) ^ cc;
+  const uint32_t zl = ~(((tl & 0x7f7f7f7fu) + 0x7f7f7f7fu) | tl | 0x7f7f7f7fu);
+  const uint32_t zh = ~(((th & 0x7f7f7f7fu) + 0x7f7f7f7fu) | th | 0x7f7f7f7fu);
+  const uint32_t f = (zl >> 7) | (zh >> 3);
+  return uint32_t((uint64_t(f) * 0x10204080ull) >> 28) & 0xFFu;
 }
 
 // Edit distance of two byte strings of at most 8 bytes, packed little-endian,
@@ -122,6 +129,13 @@ __device__ int lev_rows(const uint8_t* s, int ns, const uint8_t* t, int nt) {
   return row[ns];
 }
 
+// Bytes of a K x TW tile of 4-bit cells, in whole 32-bit words (the sweep
+// and the tile fill update cells through the words holding them), rounded to
+// 16 bytes.
+__host__ __device__ __forceinline__ size_t tile_bytes(int K, int TW) {
+  return ((size_t(K) * TW + 7) / 8 * 4 + 15) & ~size_t(15);
+}
+
 struct PairSmem {
   uint64_t* tok;  // [K + M] packed bytes (valid when len <= 8)
   int32_t* diag;  // [3 * (K + 2)] rotating anti-diagonals, indexed by i
@@ -141,7 +155,7 @@ __device__ __forceinline__ PairSmem carve(char* base, int K, int M, int TW) {
   s.path = reinterpret_cast<uint32_t*>(base + off);
   off += sizeof(uint32_t) * (K + M);
   s.tile = reinterpret_cast<uint8_t*>(base + off);
-  off += (size_t(K) * TW / 2 + 1 + 15) & ~size_t(15);
+  off += tile_bytes(K, TW);
   s.len = reinterpret_cast<uint16_t*>(base + off);
   return s;
 }
@@ -187,8 +201,13 @@ __device__ __forceinline__ void align_pair(const AlignArgs& a, int b, char* regi
           flag |= TT_REQ_TOO_LONG;
         } else {
           ln = uint16_t(n);
-          if (n <= 8)
-            for (int y = 0; y < n; ++y) packed |= uint64_t(v.bytes[o0 + y]) << (8 * y);
+          if (n <= 8) {  // all loads issued before any is used
+            uint8_t by[8];
+#pragma unroll
+            for (int y = 0; y < 8; ++y) by[y] = y < n ? v.bytes[o0 + y] : uint8_t(0);
+#pragma unroll
+            for (int y = 0; y < 8; ++y) packed |= uint64_t(by[y]) << (8 * y);
+          }
         }
       }
       sm.len[x] = ln;
@@ -417,7 +436,7 @@ __global__ void __launch_bounds__(kAlignWarpsMax * 32, 4)
 size_t align_smem_per_warp(int max_k, int max_m, int tile_w) {
   size_t n = sizeof(uint64_t) * (max_k + max_m) + sizeof(int32_t) * 3 * (max_k + 2) +
              sizeof(uint32_t) * (max_k + max_m) +
-             ((size_t(max_k) * tile_w / 2 + 1 + 15) & ~size_t(15)) +
+             tile_bytes(max_k, tile_w) +
              sizeof(uint16_t) * (max_k + max_m);
   return (n + 15) & ~size_t(15);
 }
