@@ -60,6 +60,9 @@ constexpr int kGather = 4096;          // columns held in shared memory (candida
 constexpr float kCandDelta = 14.f;     // candidates: delta below this (log2 units)
 constexpr int kCross = 256;            // candidates of the crossing bucket held apart
 constexpr int kRegion = kGather / kNW;  // candidates per warp's region of the buffer
+constexpr int kUnitBins = 16;          // candidate counts per whole log2 unit of delta
+constexpr int kRetryCands = 3200;      // candidates a second pass may take (of kGather)
+constexpr float kMinBar = 8.f;         // lowest bar of a second pass
 // Rows of at most kWarpRowMax columns: one warp per row (nucleus_warp_kernel),
 // candidates within kWCandDelta log2 units of the maximum, at most kWCap.
 constexpr int kWarpRowMax = 8192;
@@ -121,6 +124,7 @@ struct NucSmem {
   int n_gz;
   int n_gc;
   int wn[kNW];  // candidates per warp region
+  float ucnt[kUnitBins];  // estimated candidates per whole log2 unit of delta
   int todo[kNT];  // rows of the current tile left to this kernel
   int n_todo;
   float tau_v;  // the last kept column, found by one warp
@@ -315,13 +319,21 @@ __device__ bool candidate_cut(const Partial* part, NucSmem& sm, const char* row,
   const double Td = double(T.hi) + double(T.lo);
   if (!(Td > 0.0) || !isfinite(Td)) return false;
   const double thr = double(top_p) * Td * double(kFix);
-  const float zc = __fdiv_rn(__fsub_rn(M, kCandDelta), scale);  // candidates: z > zc
-
+  // Candidates: z > zc, zc = (M - bar) / scale. The first pass uses the bar
+  // kCandDelta and also counts its candidates per whole log2 unit of delta;
+  // when they overflow the buffer, a second pass takes the largest lower
+  // whole bar whose candidates fit (a row whose cut lies below that bar is
+  // still settled; the others take the histogram levels).
+  float bar = kCandDelta;
+  bool over = false;
+  for (int attempt = 0; attempt < 2; ++attempt) {
+  const float zc = __fdiv_rn(__fsub_rn(M, bar), scale);  // candidates: z > zc
   if (tid == 0) {
     sm.n_gc = 0;
     sm.cross = -1;
   }
   if (tid < kNW) sm.wn[tid] = 0;
+  if (tid < kUnitBins) sm.ucnt[tid] = 0.f;
   for (int c = tid; c < nch; c += kNT) sm.cacc[c] = 0ull;
   for (int i = tid; i < kCandBuckets; i += kNT) sm.mass[i] = 0ull;
   __syncthreads();
@@ -343,14 +355,37 @@ __device__ bool candidate_cut(const Partial* part, NucSmem& sm, const char* row,
     if (z > zc) take(z, x);
   }
   __syncthreads();
-  bool over = false;
-  int ng = 0;
+  over = false;
 #pragma unroll
+  for (int x = 0; x < kNW; ++x) over |= sm.wn[x] > kRegion;
+  if (!over || attempt == 1) break;
+  // The buffer holds the first candidates of each warp's columns, a sample of
+  // all of them whose spread in delta (per whole log2 unit) estimates theirs:
+  // the largest whole bar below this one whose estimated candidates fit with
+  // room to spare in every warp's region.
   for (int x = 0; x < kNW; ++x) {
-    ng += sm.wn[x];
-    over |= sm.wn[x] > kRegion;
+    const int held = min(sm.wn[x], kRegion);
+    const float weight = float(sm.wn[x]) / float(max(held, 1));  // candidates per held one
+    for (int i = tid; i < held; i += kNT) {
+      const float dd = __fsub_rn(M, __fmul_rn(sm.gz[x * kRegion + i].v, scale));
+      atomicAdd(&sm.ucnt[min(kUnitBins - 1, max(0, int(dd)))], weight);
+    }
+  }
+  __syncthreads();
+  float nb = 0.f, below = 0.f;
+  for (int d = 0; d < int(bar); ++d) {
+    below += sm.ucnt[d];
+    if (below > float(kRetryCands)) break;
+    nb = float(d + 1);
+  }
+  __syncthreads();  // every thread has read the counts before they are cleared
+  if (!(nb >= kMinBar && nb < bar)) break;
+  bar = nb;
   }
   if (over) return false;
+  int ng = 0;
+#pragma unroll
+  for (int x = 0; x < kNW; ++x) ng += sm.wn[x];
   // every gathered candidate, region by region
   auto for_cands = [&](auto&& fn) {
     for (int x = 0; x < kNW; ++x) {
