@@ -169,3 +169,28 @@ def test_full_size_nucleus_step_sampled(name, n_sample):
         g = dict(out)
         g["_target_off"], g["_draft_off"] = wl.target_off, wl.draft_off
         compare(sw, g, o, req_index=[b])
+
+
+def crowded_rows(wl, seed=21):
+    """Target logits whose rows hold a small nucleus near the maximum (a column
+    at 0 and a few within 3 log2 units at T = 0.6) and 5000 columns between 12.5
+    and 13.5 log2 units below it, the rest far below: at top-p 0.5 the cut lies
+    in the nucleus, while more than 4096 columns lie within 14 units."""
+    rng = np.random.default_rng(seed)
+    R, V = wl.target_logits.shape
+    scale = 1.4426950408889634 / 0.6
+    z = np.full((R, V), -40.0, np.float32)
+    for r in range(R):
+        cols = rng.permutation(V)
+        z[r, cols[0]] = 0.0
+        z[r, cols[1:5]] = -rng.uniform(0.5, 3.0, 4) / scale
+        z[r, cols[5:5005]] = -rng.uniform(12.5, 13.5, 5000) / scale
+    return dataclasses.replace(wl, target_logits=torch.as_tensor(z))
+
+
+def test_rows_that_overflow_the_first_candidate_bar():
+    """The nucleus kernel's second candidate pass (a lower whole bar estimated
+    from the held candidates) settles these rows; compared with the oracle."""
+    wl = crowded_rows(_wl("b64_g8_v152k", 6, seed=13))
+    f = dict(temp_target=0.6, top_p_target=0.5)
+    compare(wl, gpu_step(wl, **f), oracle_step(wl, **f))

@@ -10,6 +10,7 @@ of them; other rows take the full histogram levels. The paper's settings
 workload; rows of coarse integer logits take the histogram levels and rows
 with one dominant logit a single candidate, so the GPU tests cover both."""
 import dataclasses
+import os
 
 import numpy as np
 import torch
@@ -74,3 +75,28 @@ def test_coarse_integer_rows_take_the_histogram_levels():
     dominant = np.zeros(len(way), bool)
     dominant[::3] = True
     assert way[dominant].all() and not way[~dominant].any()
+
+
+def test_crowded_rows_take_the_second_candidate_pass():
+    """The rows of test_gpu_nucleus.crowded_rows: more than 4096 candidates
+    within 14 log2 units, so the first pass overflows; the count below each
+    whole bar (the kernel estimates it from the candidates it holds) gives the
+    largest bar with at most 3200, and the second pass at that bar holds the
+    cut with every warp's candidates within its region."""
+    import sys
+    sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+    import importlib
+    gn = importlib.import_module("test_gpu_nucleus")
+    wl = gn.crowded_rows(W.make_workload("b64_g8_v152k", B=6, seed=13))
+    z = wl.target_logits.numpy().astype(np.float64) * (LOG2E / 0.6)
+    d = z.max(1, keepdims=True) - z
+    m = np.exp2(-d)
+    V = d.shape[1]
+    for r in range(len(d)):
+        assert (d[r] < 14).sum() > 4096                     # the first pass overflows
+        bar = max(b for b in range(8, 14) if (d[r] < b).sum() <= 3200)
+        cols = np.nonzero(d[r] < bar)[0]
+        tid = (cols // 4) % 256                              # fp32: 4 columns per vector
+        assert np.bincount(tid // 32, minlength=8).max() <= 512
+        assert m[r][cols].sum() >= 0.5 * m[r].sum()          # the cut lies below the bar
+        assert V > 8192                                      # the CTA kernel's rows
