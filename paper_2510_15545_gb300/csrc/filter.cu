@@ -584,7 +584,11 @@ __device__ __forceinline__ int load_kept(const Cand* kept, const KeptHead* head,
 
 // ------------------------------------------------------- q_hat, filtered
 
-__global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
+// NT threads per CTA: 256, or 128 when the batch has more requests than the
+// GPU holds at once (more requests per SM, fewer threads idle at barriers).
+template <int NT>
+__global__ void __launch_bounds__(NT) filter_q_kernel(DecideArgs a) {
+  constexpr int NW = NT / 32;
   __shared__ int s_map[TT_MAX_M];
   __shared__ float s_q[TT_MAX_M];
   const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -602,13 +606,13 @@ __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
   }
   int bad = 0;
   if (st == 0)
-    for (int i = tid; i < k; i += kFThreads) {
+    for (int i = tid; i < k; i += NT) {
       const int col = a.draft_cols[d0 + i];
       if (col < 0 || col >= a.d.V) bad = 1;
     }
   grid_dependency_wait();
   if (st == 0)
-    for (int j = tid; j < m; j += kFThreads) {
+    for (int j = tid; j < m; j += NT) {
       const int i = a.map[t0 + j];
       s_map[j] = i;
       if (i < 0 || i >= k) bad = 1;
@@ -618,13 +622,13 @@ __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
   if (st == 0 && a.err && a.err[0] == a.epoch) st = a.err[1];
   if (st != 0) {
     if (!(st & (TT_REQ_BAD_OFFSETS | TT_REQ_TOO_LONG)))
-      for (int j = tid; j < m; j += kFThreads) a.q_hat_out[t0 + j] = 0.f;
+      for (int j = tid; j < m; j += NT) a.q_hat_out[t0 + j] = 0.f;
     if (tid == 0) a.status[b] = st;
     return;
   }
   // one warp per run of equal map entries (the copy rule reuses its q)
   int nonfinite = 0;
-  for (int j = warp; j < m; j += kFWarps) {
+  for (int j = warp; j < m; j += NW) {
     if (j > 0 && s_map[j] == s_map[j - 1]) continue;
     const int64_t row = int64_t(d0) + s_map[j];
     float q;
@@ -645,7 +649,7 @@ __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
     if (lane == 0) s_q[j] = q;
   }
   const int nf = __syncthreads_or(nonfinite);
-  for (int j = tid; j < m; j += kFThreads) {
+  for (int j = tid; j < m; j += NT) {
     int f = j;
     while (f > 0 && s_map[f - 1] == s_map[j]) --f;
     a.q_hat_out[t0 + j] = s_q[f];
@@ -655,7 +659,9 @@ __global__ void __launch_bounds__(kFThreads) filter_q_kernel(DecideArgs a) {
 
 // ------------------------------------------------ decision, filtered target
 
-__global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a) {
+template <int NT>
+__global__ void __launch_bounds__(NT) decide_filtered_kernel(DecideArgs a) {
+  constexpr int NW = NT / 32;
   __shared__ float s_p[TT_MAX_M];
   __shared__ int s_a, s_nf, s_pick;
   const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -681,7 +687,7 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
   }
   int bad = 0;
   if (st == 0)
-    for (int j = tid; j < m; j += kFThreads) {
+    for (int j = tid; j < m; j += NT) {
       const int col = a.target_cols[t0 + j];
       if (col < 0 || col >= a.t.V) bad = 1;
     }
@@ -696,7 +702,7 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
   if (a.err && a.err[0] == a.epoch) st = a.err[1];  // the row pass failed
   bad = 0;
   if (st == 0 && a.full_q)
-    for (int j = tid; j < m; j += kFThreads) {
+    for (int j = tid; j < m; j += NT) {
       const int i = a.map[t0 + j];
       if (i < 0 || i >= k) bad = 1;
     }
@@ -710,7 +716,7 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
     return;
   }
   // target rows 0..m: kept sets, p_hat, lse; one warp per row
-  for (int j = warp; j <= m; j += kFWarps) {
+  for (int j = warp; j <= m; j += NW) {
     const int64_t row = int64_t(t0) + b + j;
     int col;
     float prob, lse;
@@ -736,7 +742,7 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
   }
   // accept while u_j q_j < p_j (u < 1 exactly)
   const uint64_t req = a.request_base + uint64_t(b);
-  for (int j = tid; j < m; j += kFThreads) {
+  for (int j = tid; j < m; j += NT) {
     const float u = float(philox_uniform(a.seed, uint64_t(j), 0, req));
     if (!(u * a.q_hat_in[t0 + j] < s_p[j])) atomicMin(&s_a, j);
   }
@@ -814,11 +820,11 @@ __global__ void __launch_bounds__(kFThreads) decide_filtered_kernel(DecideArgs a
 }
 
 template <typename Kern>
-cudaError_t launch_f(Kern kernel, const DecideArgs& args, cudaStream_t stream, bool pdl) {
+cudaError_t launch_f(Kern kernel, int nt, const DecideArgs& args, cudaStream_t stream, bool pdl) {
   if (args.B == 0) return cudaSuccess;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(unsigned(args.B));
-  cfg.blockDim = dim3(kFThreads);
+  cfg.blockDim = dim3(nt);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
@@ -835,8 +841,10 @@ cudaError_t preload_filter() {
   cudaFuncAttributes fa;
   cudaError_t e;
   if ((e = cudaFuncGetAttributes(&fa, kept_kernel)) != cudaSuccess) return e;
-  if ((e = cudaFuncGetAttributes(&fa, filter_q_kernel)) != cudaSuccess) return e;
-  return cudaFuncGetAttributes(&fa, decide_filtered_kernel);
+  if ((e = cudaFuncGetAttributes(&fa, filter_q_kernel<128>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, filter_q_kernel<256>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, decide_filtered_kernel<128>)) != cudaSuccess) return e;
+  return cudaFuncGetAttributes(&fa, decide_filtered_kernel<256>);
 }
 
 cudaError_t launch_kept(const KeptArgs& args, cudaStream_t stream, int sm_count, bool pdl) {
@@ -857,12 +865,17 @@ cudaError_t launch_kept(const KeptArgs& args, cudaStream_t stream, int sm_count,
   return cudaLaunchKernelEx(&cfg, kept_kernel, args);
 }
 
+// 128 threads per request when the batch has more than four requests per SM
+static bool f_small_ctas(const DecideArgs& a) { return int64_t(a.B) > int64_t(4) * a.sm_count; }
+
 cudaError_t launch_filter_q(const DecideArgs& args, cudaStream_t stream, bool pdl) {
-  return launch_f(filter_q_kernel, args, stream, pdl);
+  if (f_small_ctas(args)) return launch_f(filter_q_kernel<128>, 128, args, stream, pdl);
+  return launch_f(filter_q_kernel<256>, 256, args, stream, pdl);
 }
 
 cudaError_t launch_decide_filtered(const DecideArgs& args, cudaStream_t stream, bool pdl) {
-  return launch_f(decide_filtered_kernel, args, stream, pdl);
+  if (f_small_ctas(args)) return launch_f(decide_filtered_kernel<128>, 128, args, stream, pdl);
+  return launch_f(decide_filtered_kernel<256>, 256, args, stream, pdl);
 }
 
 }  // namespace tt
