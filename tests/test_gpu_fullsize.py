@@ -23,8 +23,12 @@ def _lib():
 
 
 @pytest.mark.parametrize("name,n_sample", [("b64_g8_v152k", 10), ("b256_g16_v152k_bf16", 12),
-                                           ("b1024_g8_v201k_bf16", 6)])
+                                           ("b1024_g8_v201k_bf16", 6), ("dtw_4096x64", 12)])
 def test_full_size_step_sampled(name, n_sample):
+    """One full-size tt_step as the benchmark launches it (the decision kernel
+    at 256 threads per request, or 128 for the 1024-request and the
+    4096-request DTW batches): every request's invariants, a sample against
+    the oracle."""
     wl = W.make_workload(name, seed=0, device="cuda")
     inp = tt.device_inputs(wl, "cuda")
     out = to_np(tt.tt_step(inp["batch"], inp["vd"], inp["vt"], inp["draft_logits"],
