@@ -54,9 +54,6 @@ struct KeptHead {
   float inv_s;     // 1 / (sum over kept columns of 2^(z * scale - M))
 };
 
-// List size of the nucleus rows' units (top-p without top-k).
-constexpr int kNucList = 32;
-
 // A column of a request's repetition-penalty set (its history and sequence
 // tokens): the column and the first sequence position holding it (-1 when the
 // history holds it), so that a row at position j penalizes it when first < j.
