@@ -300,10 +300,12 @@ __device__ void walk_runs(const Cand* arr, int n, unsigned long long before, dou
 // largest logits first, reaches top_p of the row's total (from the partials)
 // is walked by value. Every column above zc is a candidate, so the walk over
 // the candidates in rank order is the walk over the whole row down to zc, and
-// a cut reached among them is the row's cut. Returns false -- and the caller
-// runs the histogram levels over the whole row -- when the candidates overflow
-// the buffer, their mass stays below the cut, or the crossing bucket holds
-// more than kCross of them. On true, sm.cacc holds the kept masses per chunk.
+// a cut reached among them is the row's cut. Candidates that overflow the
+// buffer at the first bar are gathered again at a lower one (below). Returns
+// false -- and the caller runs the histogram levels over the whole row -- when
+// the candidates still overflow the buffer, their mass stays below the cut, or
+// the crossing bucket holds more than kCross of them. On true, sm.cacc holds
+// the kept masses per chunk.
 // Every thread calls and gets the same result.
 __device__ bool candidate_cut(const Partial* part, NucSmem& sm, const char* row, int dt, int V,
                               int nvec, int vec, int nch, float M, float scale, float top_p,
@@ -320,67 +322,67 @@ __device__ bool candidate_cut(const Partial* part, NucSmem& sm, const char* row,
   if (!(Td > 0.0) || !isfinite(Td)) return false;
   const double thr = double(top_p) * Td * double(kFix);
   // Candidates: z > zc, zc = (M - bar) / scale. The first pass uses the bar
-  // kCandDelta and also counts its candidates per whole log2 unit of delta;
-  // when they overflow the buffer, a second pass takes the largest lower
-  // whole bar whose candidates fit (a row whose cut lies below that bar is
-  // still settled; the others take the histogram levels).
+  // kCandDelta; when its candidates overflow the buffer, a second pass takes
+  // the largest lower whole bar whose candidates, estimated from the ones the
+  // buffer holds, fit (a row whose cut lies below that bar is still settled;
+  // the others take the histogram levels).
   float bar = kCandDelta;
   bool over = false;
   for (int attempt = 0; attempt < 2; ++attempt) {
-  const float zc = __fdiv_rn(__fsub_rn(M, bar), scale);  // candidates: z > zc
-  if (tid == 0) {
-    sm.n_gc = 0;
-    sm.cross = -1;
-  }
-  if (tid < kNW) sm.wn[tid] = 0;
-  if (tid < kUnitBins) sm.ucnt[tid] = 0.f;
-  for (int c = tid; c < nch; c += kNT) sm.cacc[c] = 0ull;
-  for (int i = tid; i < kCandBuckets; i += kNT) sm.mass[i] = 0ull;
-  __syncthreads();
-  // ------------------------------------ one pass over the row: the candidates
-  // A vector holding a logit above zc has its candidates appended at once by
-  // its lane (the row is not read again: the rows in flight across the GPU
-  // exceed L2), each warp to its own region of the buffer (kRegion entries;
-  // the columns are spread over the warps, so a region overflows only when
-  // the whole buffer nearly would).
-  Cand* region = sm.gz + warp * kRegion;
-  auto take = [&](float z, int x) {
-    const int i = atomicAdd(&sm.wn[warp], 1);
-    if (i < kRegion) region[i] = Cand{z, x};
-  };
-  scan_row<kNT, 8>(reinterpret_cast<const uint4*>(row), nvec, dt, zc, tid,
-                   [&](int v, const uint4& w) { vector_candidates(w, dt, v, zc, take); });
-  for (int x = nvec * vec + tid; x < V; x += kNT) {  // the ragged tail
-    const float z = load_dt(row, dt, x);
-    if (z > zc) take(z, x);
-  }
-  __syncthreads();
-  over = false;
-#pragma unroll
-  for (int x = 0; x < kNW; ++x) over |= sm.wn[x] > kRegion;
-  if (!over || attempt == 1) break;
-  // The buffer holds the first candidates of each warp's columns, a sample of
-  // all of them whose spread in delta (per whole log2 unit) estimates theirs:
-  // the largest whole bar below this one whose estimated candidates fit with
-  // room to spare in every warp's region.
-  for (int x = 0; x < kNW; ++x) {
-    const int held = min(sm.wn[x], kRegion);
-    const float weight = float(sm.wn[x]) / float(max(held, 1));  // candidates per held one
-    for (int i = tid; i < held; i += kNT) {
-      const float dd = __fsub_rn(M, __fmul_rn(sm.gz[x * kRegion + i].v, scale));
-      atomicAdd(&sm.ucnt[min(kUnitBins - 1, max(0, int(dd)))], weight);
+    const float zc = __fdiv_rn(__fsub_rn(M, bar), scale);  // candidates: z > zc
+    if (tid == 0) {
+      sm.n_gc = 0;
+      sm.cross = -1;
     }
-  }
-  __syncthreads();
-  float nb = 0.f, below = 0.f;
-  for (int d = 0; d < int(bar); ++d) {
-    below += sm.ucnt[d];
-    if (below > float(kRetryCands)) break;
-    nb = float(d + 1);
-  }
-  __syncthreads();  // every thread has read the counts before they are cleared
-  if (!(nb >= kMinBar && nb < bar)) break;
-  bar = nb;
+    if (tid < kNW) sm.wn[tid] = 0;
+    if (tid < kUnitBins) sm.ucnt[tid] = 0.f;
+    for (int c = tid; c < nch; c += kNT) sm.cacc[c] = 0ull;
+    for (int i = tid; i < kCandBuckets; i += kNT) sm.mass[i] = 0ull;
+    __syncthreads();
+    // ------------------------------------ one pass over the row: the candidates
+    // A vector holding a logit above zc has its candidates appended at once by
+    // its lane (the row is not read again: the rows in flight across the GPU
+    // exceed L2), each warp to its own region of the buffer (kRegion entries;
+    // the columns are spread over the warps, so a region overflows only when
+    // the whole buffer nearly would).
+    Cand* region = sm.gz + warp * kRegion;
+    auto take = [&](float z, int x) {
+      const int i = atomicAdd(&sm.wn[warp], 1);
+      if (i < kRegion) region[i] = Cand{z, x};
+    };
+    scan_row<kNT, 8>(reinterpret_cast<const uint4*>(row), nvec, dt, zc, tid,
+                     [&](int v, const uint4& w) { vector_candidates(w, dt, v, zc, take); });
+    for (int x = nvec * vec + tid; x < V; x += kNT) {  // the ragged tail
+      const float z = load_dt(row, dt, x);
+      if (z > zc) take(z, x);
+    }
+    __syncthreads();
+    over = false;
+#pragma unroll
+    for (int x = 0; x < kNW; ++x) over |= sm.wn[x] > kRegion;
+    if (!over || attempt == 1) break;
+    // The buffer holds the first candidates of each warp's columns, a sample of
+    // all of them whose spread in delta (per whole log2 unit) estimates theirs:
+    // the largest whole bar below this one whose estimated candidates fit with
+    // room to spare in every warp's region.
+    for (int x = 0; x < kNW; ++x) {
+      const int held = min(sm.wn[x], kRegion);
+      const float weight = float(sm.wn[x]) / float(max(held, 1));  // candidates per held one
+      for (int i = tid; i < held; i += kNT) {
+        const float dd = __fsub_rn(M, __fmul_rn(sm.gz[x * kRegion + i].v, scale));
+        atomicAdd(&sm.ucnt[min(kUnitBins - 1, max(0, int(dd)))], weight);
+      }
+    }
+    __syncthreads();
+    float nb = 0.f, below = 0.f;
+    for (int d = 0; d < int(bar); ++d) {
+      below += sm.ucnt[d];
+      if (below > float(kRetryCands)) break;
+      nb = float(d + 1);
+    }
+    __syncthreads();  // every thread has read the counts before they are cleared
+    if (!(nb >= kMinBar && nb < bar)) break;
+    bar = nb;
   }
   if (over) return false;
   int ng = 0;
