@@ -175,3 +175,21 @@ def test_binding_fails_loudly_without_the_library(monkeypatch, tmp_path):
     monkeypatch.setattr(binding, "lib_path", lambda: str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="not built"):
         binding.load()
+
+
+def test_workspace_of_filter_families(lib):
+    """Host sizing of the workspace with sampling filters: top-k families add
+    their per-unit lists (k rounded up to even entries of 8 bytes per 8 KB
+    unit) and kept sets; nucleus families (top-p without top-k) add only a
+    float per 2048-column chunk and a header per row, no lists."""
+    b = tt.Batch.from_host([0, 8], list(range(8)), [0, 10], list(range(10)), device="cpu")
+    V = 151936
+    plain = tt.tt_workspace_bytes(b, V, V, tt.Params())
+    topk = tt.tt_workspace_bytes(b, V, V, tt.Params(top_k_draft=20, top_k_target=20))
+    nuc = tt.tt_workspace_bytes(b, V, V, tt.Params(top_p_draft=0.9, top_p_target=0.9))
+    units = (V + 2047) // 2048  # fp32 sizing: 2048 columns per unit
+    rows = 8 + 10 + 1           # draft rows, target rows (with the bonus row)
+    lists = rows * units * 20 * 8
+    assert topk - plain >= lists
+    assert plain < nuc < plain + rows * (units * 4 + 64) + 8 * 256
+    assert nuc < topk
